@@ -1,0 +1,117 @@
+"""Float64 CPU oracle for the Free Energy Mixer forward read (softmax prior).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may use this package; the library under
+``paper_2602_07160_gb300`` never does, and the two share no code.
+
+The arithmetic lives in ``fem_oracle.c`` (plain C99, double precision,
+optionally OpenMP over rows).  This module compiles it with gcc and calls it
+through ctypes.  ``bruteforce.py`` holds an independent 50-digit mpmath
+statement of the same read used to pin the C code.
+
+Definition followed (Sec. 2.3, Eq. "fem-free-energy-main"; App. C,
+Eq. "softmax-prior"): o_{t,j} = (1/beta_j) log sum_{i in M_t} p_t(i)
+exp(beta_j v_{i,j}) with p_t = softmax(q_t . k_i / sqrt(d)) over the masked
+support M_t, beta_j = 0 meaning the prior mean; lse_t = LSE_i s_{t,i}.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "fem_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False, src: str = _SRC, out: str = _LIB_PATH) -> str:
+    """Compile the C oracle (gcc -O2, no fast-math, OpenMP when available)."""
+    if not force and os.path.exists(out) and os.path.getmtime(out) >= os.path.getmtime(src):
+        return out
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    base = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-fno-fast-math", src, "-o", out, "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True, capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    return out
+
+
+def load(path: str | None = None):
+    """Build if needed and return the ctypes handle of the oracle library."""
+    global _lib
+    if path is not None:
+        return _bind(ctypes.CDLL(path))
+    with _lock:
+        if _lib is None:
+            _lib = _bind(ctypes.CDLL(build()))
+        return _lib
+
+
+def _bind(lib):
+    dp = ctypes.POINTER(ctypes.c_double)
+    i64 = ctypes.c_int64
+    lib.fem_oracle_fwd.argtypes = [dp, dp, dp, dp, i64, i64, i64, i64, ctypes.c_int, dp, dp, ctypes.c_int]
+    lib.fem_oracle_fwd.restype = ctypes.c_int
+    lib.fem_oracle_rows.argtypes = [dp, dp, dp, dp, i64, i64, i64, i64, ctypes.c_int,
+                                    ctypes.POINTER(ctypes.c_int64), i64, dp, dp, ctypes.c_int]
+    lib.fem_oracle_rows.restype = ctypes.c_int
+    lib.fem_oracle_max_threads.argtypes = []
+    lib.fem_oracle_max_threads.restype = ctypes.c_int
+    return lib
+
+
+def _f64(x) -> np.ndarray:
+    if hasattr(x, "detach"):  # torch tensor: upcast its exact values
+        x = x.detach().to("cpu").double().numpy()
+    return np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
+
+
+def max_threads(lib=None) -> int:
+    return int((lib or load()).fem_oracle_max_threads())
+
+
+def fem_read(q, k, v, beta, causal: bool, nthreads: int = 0, lib=None):
+    """The whole read.  q, k, v: [B, H, T, d]; beta: [H, d].
+
+    Returns (out [B, H, T, d], lse [B, H, T]) as float64 numpy arrays."""
+    lib = lib or load()
+    q, k, v, beta = _f64(q), _f64(k), _f64(v), _f64(beta)
+    B, H, T, d = q.shape
+    assert k.shape == q.shape and v.shape == q.shape and beta.shape == (H, d)
+    out = np.empty((B, H, T, d), dtype=np.float64)
+    lse = np.empty((B, H, T), dtype=np.float64)
+    rc = lib.fem_oracle_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), B, H, T, d, int(bool(causal)),
+                            _ptr(out), _ptr(lse), int(nthreads))
+    if rc != 0:
+        raise ValueError(f"fem_oracle_fwd failed with code {rc}")
+    return out, lse
+
+
+def fem_read_rows(q, k, v, beta, causal: bool, rows, nthreads: int = 0, lib=None):
+    """Selected rows.  rows: flat indices (b*H + h)*T + t.
+
+    Returns (out [n, d], lse [n]) as float64 numpy arrays."""
+    lib = lib or load()
+    q, k, v, beta = _f64(q), _f64(k), _f64(v), _f64(beta)
+    B, H, T, d = q.shape
+    rows = np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+    out = np.empty((rows.size, d), dtype=np.float64)
+    lse = np.empty((rows.size,), dtype=np.float64)
+    rc = lib.fem_oracle_rows(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), B, H, T, d, int(bool(causal)),
+                             rows.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), rows.size,
+                             _ptr(out), _ptr(lse), int(nthreads))
+    if rc != 0:
+        raise ValueError(f"fem_oracle_rows failed with code {rc}")
+    return out, lse
