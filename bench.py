@@ -1,0 +1,395 @@
+#!/usr/bin/env python
+"""Benchmark of the Free Energy Mixer forward read on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl fem|reference]
+                    [--workload lm_causal_d128]
+
+One step is one full read (value statistics pre-pass, tensor-core kernel,
+exact fix-up) of the workload's synthetic inputs, resident in HBM.  Prints
+one JSON line: the metric (TFLOP/s with the flash-attention FLOP count,
+causal-halved), the tensor-core roofline of the dominant kernel (timed with
+CUDA events on its launch stream), the end-to-end figure through the
+host-buffer C-ABI call (copies included), the float64 oracle timed on a
+bounded sample on the host cores, and the SM clocks seen during the timed
+region.  ``--impl reference`` times the oracle itself, as the reference arm.
+
+Under torchrun (N > 1) every rank reads its own copy of the workload (weak
+scaling, no collective on the data path); the step time is the maximum over
+ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "FEM fwd TFLOP/s and tensor-pipe % of GB300 peak (causal, T=8192, d=128, bf16)"
+UNIT = "TFLOP/s"
+L2_BYTES = 129 * 1024 * 1024
+FALLBACK_BF16_TFLOPS = 1900.0
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fem_tc_traffic.txt")
+TC_SOURCE = os.path.join(ROOT, "paper_2602_07160_gb300", "csrc", "fem_tc.cu")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["fem", "reference"], default="fem")
+    ap.add_argument("--workload", default="lm_causal_d128")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle CPU-baseline budget")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--shape", default=None,
+                    help="B,H,T override of the workload sizes (profiling aid; the JSON config reports them)")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (timing only)
+# ---------------------------------------------------------------------------
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_dist(world, backend="nccl"):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return dist if world > 1 else None
+
+
+def barrier(dist, device=None):
+    if dist is not None:
+        if device is not None:
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+def max_over_ranks(dist, value: float, device=None) -> float:
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.3)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons, power = [], 0.0, set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                p = [x.strip() for x in line.split(",")]
+                if len(p) < 9:
+                    continue
+                try:
+                    sm.append(float(p[1]))
+                    smax = max(smax, float(p[2]))
+                    power.append(float(p[3]))
+                except ValueError:
+                    continue
+                for n, flag in zip(names, p[5:9]):
+                    if flag.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        loaded = [x for x in sm if x >= 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+# ---------------------------------------------------------------------------
+# peaks, traffic record
+# ---------------------------------------------------------------------------
+def bf16_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), "measured (MEASURED_PEAKS.json bf16_tflops, burst)"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_BF16_TFLOPS, "fallback (1.9 PFLOP/s bf16 burst)"
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the tensor-core kernel from a committed ncu
+    summary, if that summary was taken on the current kernel source."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            rec = dict(line.strip().split("=", 1) for line in f if "=" in line and not line.startswith("#"))
+        sha = hashlib.sha256(open(TC_SOURCE, "rb").read()).hexdigest()[:16]
+        if rec.get("source_sha") != sha or rec.get("workload") != workload:
+            return None
+        return float(rec["dram_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+# ---------------------------------------------------------------------------
+# the oracle on a bounded sample (CPU baseline and reference arm)
+# ---------------------------------------------------------------------------
+def row_flops(w, rows):
+    import numpy as np
+    t = np.asarray(rows) % w.T
+    keys = (t + 1) if w.causal else np.full_like(t, w.T)
+    return float((4.0 * w.d * keys).sum())
+
+
+class OracleSampler:
+    def __init__(self, w, q, k, v, beta, seed=1):
+        import numpy as np
+        import oracle
+        self.w = w
+        self.oracle = oracle
+        self.lib = oracle.load()
+        self.arrays = [np.ascontiguousarray(x.double().numpy()) for x in (q, k, v, beta)]
+        self.rng = np.random.default_rng(seed)
+        self.threads = oracle.max_threads(self.lib)
+
+    def rows(self, n):
+        w = self.w
+        return self.rng.choice(w.B * w.H * w.T, size=n, replace=False)
+
+    def run(self, rows):
+        q, k, v, beta = self.arrays
+        t = time.perf_counter()
+        self.oracle.fem_read_rows(q, k, v, beta, self.w.causal, rows, lib=self.lib)
+        return time.perf_counter() - t
+
+    def rows_for_seconds(self, seconds):
+        probe = self.rows(64)
+        dt = max(self.run(probe), 1e-3)
+        per_flop = dt / row_flops(self.w, probe)
+        mean_row_flops = 4.0 * self.w.d * ((self.w.T + 1) / 2 if self.w.causal else self.w.T)
+        return max(16, int(seconds / per_flop / mean_row_flops))
+
+    def measure(self, seconds):
+        batch = self.rows_for_seconds(min(2.0, seconds))
+        flops, dt, n = 0.0, 0.0, 0
+        while dt < seconds:
+            rows = self.rows(batch)
+            dt += self.run(rows)
+            flops += row_flops(self.w, rows)
+            n += batch
+        return flops / dt / 1e12, n, dt
+
+
+# ---------------------------------------------------------------------------
+# arms
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2602_07160_gb300 import workloads as W
+    w = W.WORKLOADS[args.workload]
+    q, k, v, beta = W.make_inputs(w)
+    s = OracleSampler(w, q, k, v, beta)
+    step_s = max(0.5, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
+    n = s.rows_for_seconds(step_s)
+    for _ in range(args.warmup):
+        s.run(s.rows(n))
+    flops, secs = 0.0, 0.0
+    for _ in range(args.steps):
+        rows = s.rows(n)
+        secs += s.run(rows)
+        flops += row_flops(w, rows)
+    value = flops / secs / 1e12
+    sample = f"{n} uniformly drawn rows of the workload per step ({args.steps} steps)"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": dict(w.describe(), l2="inputs larger than L2"),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": s.threads, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_fem(args):
+    import numpy as np
+    import torch
+
+    from paper_2602_07160_gb300 import build as fem_build
+    from paper_2602_07160_gb300 import fem
+    from paper_2602_07160_gb300 import workloads as W
+
+    world, rank, local = dist_env()
+    dist = init_dist(world)
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    fem_build.build()
+    fem.load()
+
+    w = W.WORKLOADS[args.workload]
+    if args.shape:
+        import dataclasses
+        B_, H_, T_ = (int(x) for x in args.shape.split(","))
+        w = dataclasses.replace(w, B=B_, H=H_, T=T_, name=f"{w.name}@B{B_}H{H_}T{T_}")
+    if w.dtype != "bf16":
+        raise SystemExit("bench times the bf16 tensor-core read; pick a bf16 workload")
+    q, k, v, beta = W.make_inputs(w, seed=rank)  # sizes come from w (overridable with --shape)
+    qd, kd, vd, bd = (x.to(device) for x in (q, k, v, beta))
+    out = torch.empty(q.shape, dtype=torch.float32, device=device)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=device)
+    stream = torch.cuda.current_stream(device)
+
+    def step():
+        fem.fem_fwd(qd, kd, vd, bd, causal=w.causal, out=out, lse=lse, stream=stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    fem.check_device_error(stream)
+
+    # sanity parity on a few sampled rows (oracle, float64) before timing
+    parity = None
+    if rank == 0:
+        import oracle
+        rows = np.random.default_rng(123).choice(w.B * w.H * w.T, size=48, replace=False)
+        rows = np.unique(np.concatenate([rows, np.arange(16)]))
+        ref, _ = oracle.fem_read_rows(q, k, v, beta, w.causal, rows)
+        got = out.reshape(-1, w.d)[torch.from_numpy(rows).to(device)].double().cpu().numpy()
+        parity = {"rows": int(rows.size), "max_abs": float(np.abs(got - ref).max())}
+
+    # ---- timed region: K reads, inputs resident (403 MB of Q/K/V > 129 MB L2)
+    K = args.steps
+    k_start = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    k_stop = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    for e in k_start + k_stop:
+        e.record(stream)  # materialise the CUDA events
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_stop = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
+    barrier(dist, device)
+    torch.cuda.synchronize(device)
+    if clocks:
+        clocks.start()
+        time.sleep(0.2)
+    t_start.record(stream)
+    for i in range(K):
+        fem.set_kernel_events(k_start[i], k_stop[i])
+        step()
+    t_stop.record(stream)
+    torch.cuda.synchronize(device)
+    barrier(dist, device)
+    clk = clocks.stop() if clocks else None
+    fem.check_device_error(stream)
+    ms_step = t_start.elapsed_time(t_stop) / K
+    ms_step = max_over_ranks(dist, ms_step, device)
+    kernel_ms = [a.elapsed_time(b) for a, b in zip(k_start, k_stop)]
+    tc_ms = statistics.mean(kernel_ms)
+    fixup_entries = fem.last_fixup_rows(stream)
+
+    value = w.flops * world / (ms_step * 1e-3) / 1e12
+    peak, peak_src = bf16_peak()
+    achieved = w.flops / (tc_ms * 1e-3) / 1e12
+    traffic = recorded_traffic(w.name)
+
+    # ---- end to end through the host-buffer C ABI call
+    e2e = None
+    if not args.no_e2e:
+        hq, hk, hv, hb = (x.pin_memory() for x in (q, k, v, beta))
+        hout = torch.empty(q.shape, dtype=torch.float32).pin_memory()
+        hlse = torch.empty(q.shape[:3], dtype=torch.float32).pin_memory()
+        fem.fem_fwd_host(hq, hk, hv, hb, causal=w.causal, out=hout, lse=hlse, stream=stream)
+        barrier(dist, device)
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            fem.fem_fwd_host(hq, hk, hv, hb, causal=w.causal, out=hout, lse=hlse, stream=stream)
+        e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+        e2e_s = max_over_ranks(dist, e2e_s, device)
+        h2d = sum(x.numel() * x.element_size() for x in (hq, hk, hv, hb))
+        d2h = hout.numel() * 4 + hlse.numel() * 4
+        e2e = {"value": w.flops * world / e2e_s / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "steps": args.e2e_steps}
+
+    # ---- the oracle on the host cores (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        s = OracleSampler(w, q, k, v, beta)
+        val, n, dt = s.measure(args.cpu_seconds)
+        cpu = {"value": val, "unit": UNIT, "cores": s.threads, "kind": "oracle",
+               "sample": f"{n} uniformly drawn rows of the workload, {dt:.1f} s of float64 C/OpenMP"}
+
+    if rank == 0:
+        in_bytes = sum(x.numel() * x.element_size() for x in (q, k, v))
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+            "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
+            "config": dict(w.describe(), pv_operands="fp16", parallelism=f"replicas{world}" if world > 1 else "single",
+                           l2=f"inputs larger than L2 ({in_bytes / 1e6:.0f} MB of Q/K/V vs 129 MB L2)",
+                           parity_sample=parity, fixup_entries=fixup_entries),
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                         "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
+                         "kernel": "fem_tc_kernel", "kernel_ms": tc_ms},
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+            "clocks": clk,
+            "gpu_launches": K * (3 if w.causal else 2),
+        }
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_fem(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,136 @@
+/*
+ * fem.h -- C ABI of libfem.so: the forward free-energy read of the Free
+ * Energy Mixer (arXiv 2602.07160) with a softmax prior, on sm_103a GPUs.
+ *
+ * The read (Sec. 2.3, Eq. "fem-free-energy-main"; softmax prior of App. C,
+ * Eq. "softmax-prior"; masked scaled scores of Sec. 1):
+ *
+ *   s_{t,i} = q_t . k_i / sqrt(d),  i in M_t = {0..t} (causal) or {0..T-1}
+ *   o_{t,j} = (1/beta_j) ( LSE_i(s_{t,i} + beta_j v_{i,j}) - LSE_i s_{t,i} )
+ *           = (1/beta_j) log sum_{i in M_t} softmax(s_t)_i exp(beta_j v_{i,j})
+ *   lse_t   = LSE_i s_{t,i}   (natural log; LSE_i(s + beta v) = lse + beta o)
+ *
+ * beta_j = 0 is the continuous beta -> 0 limit, the prior mean
+ * sum_i p_t(i) v_{i,j} (Prop. "app-baseline").  beta_j < 0 is outside the
+ * method and a precondition violation (device memory is not inspected).
+ *
+ * Conventions for every entry point:
+ *  - Layout: q, k, v are [B, H, T, d] contiguous, d fastest; beta is [H, d]
+ *    float32 (per head, per channel, shared over batch and time); out is
+ *    [B, H, T, d] float32; lse is [B, H, T] float32 or NULL.
+ *  - Ownership: the caller owns every buffer.  Device pointers must be
+ *    16-byte aligned.  The library keeps no pointer after a call returns.
+ *  - Streams: `stream` is a cudaStream_t (NULL = legacy default stream).
+ *    Device work is enqueued asynchronously on it; outputs are valid once the
+ *    stream reaches the end of the call's work.
+ *  - Errors: argument errors are reported synchronously and nothing is
+ *    enqueued.  A CUDA launch or allocation failure returns FEM_ERR_CUDA or
+ *    FEM_ERR_NO_MEMORY.  A kernel that gives up on a bounded wait records
+ *    the fact in a per-device error word and exits cleanly; read it with
+ *    fem_check_device_error().  No exception crosses the ABI.
+ *  - Threads: entry points may be called from several host threads; calls
+ *    share only the per-device error word and fix-up counter.
+ */
+#ifndef FEM_H
+#define FEM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FEM_OK = 0,
+    FEM_ERR_INVALID_ARG = 1,  /* null pointer, non-positive size, misalignment */
+    FEM_ERR_UNSUPPORTED = 2,  /* a head dimension the path does not implement */
+    FEM_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed */
+    FEM_ERR_TIMEOUT = 4,      /* a kernel gave up on a bounded wait */
+    FEM_ERR_NO_MEMORY = 5     /* workspace allocation failed / too small */
+} fem_status;
+
+/*
+ * fem_fwd -- the read for bf16 inputs (the tensor-core path).
+ *   q, k, v : device, bf16 [B, H, T, d]
+ *   beta    : device, float32 [H, d], beta >= 0
+ *   out     : device, float32 [B, H, T, d]
+ *   lse     : device, float32 [B, H, T], or NULL
+ *   B, H, T : >= 1;  d in {64, 128};  causal: 0 (full prior) or 1
+ * Allocates its workspace stream-ordered (cudaMallocAsync/cudaFreeAsync on
+ * `stream`).  Accuracy: the score contraction takes bf16 q, k; the second
+ * contraction takes the prior weights and the per-channel value bank in fp16
+ * (11-bit significand); both accumulate in fp32.
+ */
+int fem_fwd(const void *q, const void *k, const void *v, const float *beta,
+            float *out, float *lse, int B, int H, int T, int d, int causal,
+            void *stream);
+
+/*
+ * fem_fwd_workspace_bytes -- bytes of device workspace fem_fwd_ws needs for
+ * these sizes (0 on invalid sizes).
+ */
+size_t fem_fwd_workspace_bytes(int B, int H, int T, int d, int causal);
+
+/*
+ * fem_fwd_ws -- fem_fwd with a caller-owned device workspace of at least
+ * fem_fwd_workspace_bytes() bytes, 256-byte aligned.  Performs no allocation.
+ * The workspace must not be used by another call that overlaps on the GPU.
+ */
+int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta,
+               float *out, float *lse, int B, int H, int T, int d, int causal,
+               void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * fem_fwd_f32 -- the read for float32 inputs on CUDA cores (exact fp32
+ * arithmetic with a per-row, per-channel shift).  Same layout and rules as
+ * fem_fwd with q, k, v float32; 1 <= d <= 256.  No workspace.
+ */
+int fem_fwd_f32(const float *q, const float *k, const float *v,
+                const float *beta, float *out, float *lse, int B, int H, int T,
+                int d, int causal, void *stream);
+
+/*
+ * fem_fwd_host -- fem_fwd on HOST buffers: copies q, k, v, beta to the
+ * device, runs the read and copies out (and lse, if non-NULL) back, all on
+ * `stream`, then synchronises it.  Host buffers should be pinned for full
+ * copy bandwidth.  Device buffers come from cudaMallocAsync on `stream` and
+ * are freed before return.  Returns after the results are in host memory.
+ */
+int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
+                 float *out, float *lse, int B, int H, int T, int d, int causal,
+                 void *stream);
+
+/*
+ * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
+ * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
+ * on a bounded wait since the last check (the word is cleared), or
+ * FEM_ERR_CUDA if the synchronisation failed.
+ */
+int fem_check_device_error(void *stream);
+
+/*
+ * fem_last_fixup_rows -- synchronises `stream` and returns the number of
+ * (row, 32-channel group) entries the last bf16 read on the current device
+ * recomputed exactly (causal rows whose visible values lie far below the
+ * shared value-bank shift).  Diagnostic; -1 on error.
+ */
+int fem_last_fixup_rows(void *stream);
+
+/*
+ * fem_set_kernel_events -- diagnostic timing hook.  With both arguments
+ * non-NULL (caller-owned cudaEvent_t handles), the next bf16 read issued by
+ * the calling host thread records `start` on its stream immediately before
+ * its tensor-core kernel and `stop` immediately after it, then forgets the
+ * events.  Passing NULL clears a pending request.  Always FEM_OK.
+ */
+int fem_set_kernel_events(void *start, void *stop);
+
+/* fem_status_str -- a static string naming a status code. */
+const char *fem_status_str(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FEM_H */

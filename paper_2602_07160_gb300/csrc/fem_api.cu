@@ -1,0 +1,282 @@
+// C ABI of libfem.so (declared in include/fem.h): argument checks, workspace
+// layout, TMA tensor maps and the launch sequence of the FEM read.
+//
+// bf16 path, in stream order:
+//   1. value_stats  (one read of V): channel modes, shift schedule, fix-up list
+//   2. fem_tc       (tcgen05): the read for every row and channel
+//   3. fixup        (causal only): exact fp32 recompute of the listed entries
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "fem.h"
+#include "fem_launch.h"
+
+namespace fem {
+namespace {
+
+__device__ unsigned g_error_word;
+__device__ int g_last_fixup;
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+  bool ready = false;
+  unsigned *err = nullptr;
+  int *last_fixup = nullptr;
+  int num_sms = 0;
+};
+
+std::mutex g_mutex;
+thread_local cudaEvent_t t_ev_start = nullptr, t_ev_stop = nullptr;
+DeviceState g_dev[kMaxDevices];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int map_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return FEM_OK;
+  if (e == cudaErrorMemoryAllocation) return FEM_ERR_NO_MEMORY;
+  return FEM_ERR_CUDA;
+}
+
+// Per-device addresses of the error word and fix-up counter, SM count and the
+// tensor-map encoder, set up once with the device current.
+int device_state(DeviceState **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FEM_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceState &s = g_dev[dev];
+  if (!s.ready) {
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&s.err), g_error_word) != cudaSuccess) return FEM_ERR_CUDA;
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&s.last_fixup), g_last_fixup) != cudaSuccess)
+      return FEM_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return FEM_ERR_CUDA;
+    if (!g_encode) {
+      cudaDriverEntryPointQueryResult q;
+      void *fn = nullptr;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || !fn)
+        return FEM_ERR_CUDA;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    s.ready = true;
+  }
+  *out = &s;
+  return FEM_OK;
+}
+
+// [d, T, B*H] bf16 tensor, boxes of 64 channels x 128 rows, 128-byte swizzle.
+int make_map(CUtensorMap *map, const void *base, int BH, int T, int d) {
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(BH)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(T) * d * 2};
+  cuuint32_t box[3] = {64, 128, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? FEM_OK : FEM_ERR_CUDA;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct WsLayout {
+  size_t chan, cpre, fixups, count, total;
+};
+
+bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
+  if (B <= 0 || H <= 0 || T <= 0 || d <= 0) return false;
+  const size_t BH = static_cast<size_t>(B) * H;
+  const size_t n_kt = (static_cast<size_t>(T) + kBlockK - 1) / kBlockK;
+  const size_t groups = (static_cast<size_t>(d) + 31) / 32;
+  size_t off = 0;
+  w->chan = off;
+  off += round256(BH * d * sizeof(ChanInfo));
+  w->cpre = off;
+  off += round256(BH * n_kt * d * sizeof(float));
+  w->fixups = off;
+  off += causal ? round256(BH * n_kt * kBlockQ * groups * sizeof(FixupEntry)) : 0;
+  w->count = off;
+  off += 256;
+  w->total = off;
+  return true;
+}
+
+int check_common(const void *q, const void *k, const void *v, const float *beta, const float *out, const float *lse,
+                 int B, int H, int T, int d, int causal) {
+  if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || T <= 0 || d <= 0) return FEM_ERR_INVALID_ARG;
+  if (causal != 0 && causal != 1) return FEM_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out)) return FEM_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(beta) & 3u) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return FEM_ERR_INVALID_ARG;
+  const long long rows = static_cast<long long>(B) * H * T;
+  if (rows >= (1ll << 31) || static_cast<long long>(B) * H > 65535) return FEM_ERR_UNSUPPORTED;
+  return FEM_OK;
+}
+
+}  // namespace
+}  // namespace fem
+
+using namespace fem;
+
+extern "C" {
+
+const char *fem_status_str(int status) {
+  switch (status) {
+    case FEM_OK: return "FEM_OK";
+    case FEM_ERR_INVALID_ARG: return "FEM_ERR_INVALID_ARG";
+    case FEM_ERR_UNSUPPORTED: return "FEM_ERR_UNSUPPORTED";
+    case FEM_ERR_CUDA: return "FEM_ERR_CUDA";
+    case FEM_ERR_TIMEOUT: return "FEM_ERR_TIMEOUT";
+    case FEM_ERR_NO_MEMORY: return "FEM_ERR_NO_MEMORY";
+    default: return "FEM_ERR_UNKNOWN";
+  }
+}
+
+size_t fem_fwd_workspace_bytes(int B, int H, int T, int d, int causal) {
+  WsLayout w;
+  if (!ws_layout(B, H, T, d, causal ? 1 : 0, &w)) return 0;
+  return w.total;
+}
+
+int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
+               int T, int d, int causal, void *workspace, size_t workspace_bytes, void *stream) {
+  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  WsLayout w;
+  ws_layout(B, H, T, d, causal, &w);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return FEM_ERR_INVALID_ARG;
+  if (workspace_bytes < w.total) return FEM_ERR_NO_MEMORY;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
+
+  const int BH = B * H;
+  CUtensorMap tq, tk, tv;
+  if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
+  if ((rc = make_map(&tk, k, BH, T, d)) != FEM_OK) return rc;
+  if ((rc = make_map(&tv, v, BH, T, d)) != FEM_OK) return rc;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  ChanInfo *chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
+  float *cpre = reinterpret_cast<float *>(ws + w.cpre);
+  FixupEntry *fix = reinterpret_cast<FixupEntry *>(ws + w.fixups);
+  int *count = reinterpret_cast<int *>(ws + w.count);
+
+  cudaError_t e = cudaMemsetAsync(count, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = launch_value_stats(v, beta, BH, H, T, d, causal, chan, cpre, fix, count, s);
+  const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
+  t_ev_start = t_ev_stop = nullptr;
+  if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
+  if (e == cudaSuccess) e = launch_tc(d, tq, tk, tv, beta, chan, cpre, out, lse, BH, H, T, causal, ds->err, s);
+  if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
+  if (e == cudaSuccess) {
+    if (causal)
+      e = launch_fixup(q, k, v, beta, out, H, T, d, fix, count, ds->last_fixup, ds->num_sms, s);
+    else
+      e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
+  }
+  return map_cuda(e);
+}
+
+int fem_fwd(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
+            int T, int d, int causal, void *stream) {
+  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  const size_t bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  void *ws = nullptr;
+  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
+  if (e != cudaSuccess) return map_cuda(e);
+  rc = fem_fwd_ws(q, k, v, beta, out, lse, B, H, T, d, causal, ws, bytes, stream);
+  e = cudaFreeAsync(ws, s);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(e);
+}
+
+int fem_fwd_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse, int B,
+                int H, int T, int d, int causal, void *stream) {
+  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (d > 256) return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  return map_cuda(launch_f32(q, k, v, beta, out, lse, B, H, T, d, causal, static_cast<cudaStream_t>(stream)));
+}
+
+int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B,
+                 int H, int T, int d, int causal, void *stream) {
+  if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || T <= 0 || d <= 0 || (causal != 0 && causal != 1)) return FEM_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  const size_t n = static_cast<size_t>(B) * H * T * d;
+  const size_t rows = static_cast<size_t>(B) * H * T;
+  const size_t in_b = round256(n * 2), beta_b = round256(static_cast<size_t>(H) * d * 4), out_b = round256(n * 4),
+               lse_b = round256(rows * 4), ws_b = fem_fwd_workspace_bytes(B, H, T, d, causal);
+  const size_t total = 3 * in_b + beta_b + out_b + lse_b + ws_b;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t *buf = nullptr;
+  cudaError_t e = cudaMallocAsync(reinterpret_cast<void **>(&buf), total, s);
+  if (e != cudaSuccess) return map_cuda(e);
+  uint8_t *dq = buf, *dk = dq + in_b, *dv = dk + in_b, *db = dv + in_b, *dout = db + beta_b, *dlse = dout + out_b,
+          *dws = dlse + lse_b;
+  e = cudaMemcpyAsync(dq, q, n * 2, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(dk, k, n * 2, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(dv, v, n * 2, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(db, beta, static_cast<size_t>(H) * d * 4, cudaMemcpyHostToDevice, s);
+  int rc = map_cuda(e);
+  if (rc == FEM_OK)
+    rc = fem_fwd_ws(dq, dk, dv, reinterpret_cast<float *>(db), reinterpret_cast<float *>(dout),
+                    lse ? reinterpret_cast<float *>(dlse) : nullptr, B, H, T, d, causal, dws, ws_b, stream);
+  if (rc == FEM_OK) {
+    e = cudaMemcpyAsync(out, dout, n * 4, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && lse) e = cudaMemcpyAsync(lse, dlse, rows * 4, cudaMemcpyDeviceToHost, s);
+    rc = map_cuda(e);
+  }
+  cudaError_t ef = cudaFreeAsync(buf, s);
+  cudaError_t es = cudaStreamSynchronize(s);
+  if (rc != FEM_OK) return rc;
+  if (ef != cudaSuccess) return map_cuda(ef);
+  return map_cuda(es);
+}
+
+int fem_set_kernel_events(void *start, void *stop) {
+  if (start && stop) {
+    t_ev_start = static_cast<cudaEvent_t>(start);
+    t_ev_stop = static_cast<cudaEvent_t>(stop);
+  } else {
+    t_ev_start = t_ev_stop = nullptr;
+  }
+  return FEM_OK;
+}
+
+int fem_check_device_error(void *stream) {
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return FEM_ERR_CUDA;
+  unsigned word = 0;
+  if (cudaMemcpy(&word, ds->err, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return FEM_ERR_CUDA;
+  if (word) {
+    const unsigned zero = 0;
+    if (cudaMemcpy(ds->err, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return FEM_ERR_CUDA;
+    return FEM_ERR_TIMEOUT;
+  }
+  return FEM_OK;
+}
+
+int fem_last_fixup_rows(void *stream) {
+  DeviceState *ds = nullptr;
+  if (device_state(&ds) != FEM_OK) return -1;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return -1;
+  int n = 0;
+  if (cudaMemcpy(&n, ds->last_fixup, sizeof(n), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+  return n;
+}
+
+}  // extern "C"

@@ -1,0 +1,128 @@
+// The FEM read for fp32 inputs on CUDA cores, exact to fp32 rounding.
+//
+// One warp per output row t; lane l owns channels l, l+32, ...  For every key
+// i in the support the warp forms s_{t,i} = q_t . k_i / sqrt(d) (lane-partial
+// dot product, butterfly sum) and folds key i into
+//   L   = sum_i P_i,                          P_i = exp(s_i - m)
+//   A_j = sum_i P_i exp(beta_j (v_ij - c_j))
+//   W_j = sum_i P_i expm1(beta_j (v_ij - c_j)) / beta_j   (v_ij - c_j at beta 0)
+// with a running row maximum m and an exact running per-channel maximum c_j
+// of the visible values (the per-channel stabilisation of App. E, per row).
+// When m grows by dm, L, A and W scale by exp(-dm); when c_j grows to c',
+// with r = exp(beta (c - c')), A <- r A and W <- r W + expm1(beta (c - c'))/beta L
+// (the joint rescale of the two running shifts).  The read is then
+//   o = c + log1p(beta W / L) / beta   when beta W / L > -1/2 (no cancellation),
+//   o = c + log(A / L) / beta          otherwise,
+//   o = c + W / L                      at beta = 0 (the prior mean),
+// which is (1/beta) log sum_i p_t(i) exp(beta v_ij) (Sec. 2.3).
+#include "fem_common.cuh"
+#include "fem_launch.h"
+
+namespace fem {
+
+constexpr int kSimtMaxPerLane = 8;  // d <= 256
+
+__device__ __forceinline__ float expm1_over_beta(float b, float x) {
+  // expm1(b x) / b, continuous at b = 0
+  return b != 0.f ? expm1f(b * x) / b : x;
+}
+
+__global__ void __launch_bounds__(128) fem_f32_kernel(const float *__restrict__ q, const float *__restrict__ k,
+                                                       const float *__restrict__ v, const float *__restrict__ beta,
+                                                       float *__restrict__ out, float *__restrict__ lse, int H,
+                                                       int T, int d, int causal, long long n_rows) {
+  const int lane = threadIdx.x & 31;
+  const long long row = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (row >= n_rows) return;
+  const long long bh = row / T;
+  const int t = static_cast<int>(row % T);
+  const int h = static_cast<int>(bh % H);
+  const int n = causal ? t + 1 : T;
+  const int per = (d + 31) / 32;
+  const float inv_sqrt_d = rsqrtf(static_cast<float>(d));
+  const float *kb = k + bh * T * d;
+  const float *vb = v + bh * T * d;
+
+  float qv[kSimtMaxPerLane], bj[kSimtMaxPerLane], c[kSimtMaxPerLane], A[kSimtMaxPerLane], W[kSimtMaxPerLane];
+#pragma unroll
+  for (int u = 0; u < kSimtMaxPerLane; ++u) {
+    const int j = lane + 32 * u;
+    const bool ok = u < per && j < d;
+    qv[u] = ok ? q[row * d + j] : 0.f;
+    bj[u] = ok ? beta[h * d + j] : 0.f;
+    c[u] = -INFINITY;
+    A[u] = 0.f;
+    W[u] = 0.f;
+  }
+  float m = -INFINITY, L = 0.f;
+
+  for (int i = 0; i < n; ++i) {
+    const float *kr = kb + static_cast<long long>(i) * d;
+    float part = 0.f;
+#pragma unroll
+    for (int u = 0; u < kSimtMaxPerLane; ++u) {
+      const int j = lane + 32 * u;
+      if (u < per && j < d) part = fmaf(qv[u], kr[j], part);
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+    const float s = part * inv_sqrt_d;
+    if (s > m) {
+      const float alpha = expf(m - s);  // 0 when m = -inf
+      L *= alpha;
+#pragma unroll
+      for (int u = 0; u < kSimtMaxPerLane; ++u) {
+        A[u] *= alpha;
+        W[u] *= alpha;
+      }
+      m = s;
+    }
+    const float p = expf(s - m);
+    const float *vr = vb + static_cast<long long>(i) * d;
+#pragma unroll
+    for (int u = 0; u < kSimtMaxPerLane; ++u) {
+      const int j = lane + 32 * u;
+      if (!(u < per && j < d)) continue;
+      const float x = vr[j];
+      const float b = bj[u];
+      if (x > c[u]) {
+        if (c[u] != -INFINITY) {
+          const float r = expf(b * (c[u] - x));
+          W[u] = r * W[u] + expm1_over_beta(b, c[u] - x) * L;
+          A[u] *= r;
+        }
+        c[u] = x;
+      }
+      A[u] += p * expf(b * (x - c[u]));
+      W[u] += p * expm1_over_beta(b, x - c[u]);
+    }
+    L += p;
+  }
+
+#pragma unroll
+  for (int u = 0; u < kSimtMaxPerLane; ++u) {
+    const int j = lane + 32 * u;
+    if (!(u < per && j < d)) continue;
+    const float b = bj[u];
+    float o;
+    if (b == 0.f) {
+      o = c[u] + W[u] / L;
+    } else {
+      const float z = b * W[u] / L;
+      o = z > -0.5f ? c[u] + log1pf(z) / b : c[u] + logf(A[u] / L) / b;
+    }
+    out[row * d + j] = o;
+  }
+  if (lse && lane == 0) lse[row] = m + logf(L);
+}
+
+cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
+                       int B, int H, int T, int d, int causal, cudaStream_t stream) {
+  const long long n_rows = static_cast<long long>(B) * H * T;
+  const long long blocks = (n_rows + 3) / 4;
+  fem_f32_kernel<<<static_cast<unsigned>(blocks), 128, 0, stream>>>(q, k, v, beta, out, lse, H, T, d, causal,
+                                                                    n_rows);
+  return cudaGetLastError();
+}
+
+}  // namespace fem

@@ -1,0 +1,176 @@
+"""Python binding of libfem.so (argument marshalling only).
+
+Every function here checks shapes, dtypes and devices of torch tensors,
+passes raw pointers and sizes to the C ABI of ``include/fem.h`` and raises on
+a non-zero status.  All arithmetic of the read runs in the library's CUDA
+kernels; there is no other implementation behind these names.  If the
+library is not built, ``load()`` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libfem.so")
+_lock = threading.Lock()
+_lib = None
+
+STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "FEM_ERR_CUDA",
+          4: "FEM_ERR_TIMEOUT", 5: "FEM_ERR_NO_MEMORY"}
+
+EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
+           "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str"]
+
+
+class FemError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        super().__init__(f"{fn} returned {STATUS.get(status, status)}")
+        self.status = status
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load(path: str | None = None):
+    """Load libfem.so (built by ``paper_2602_07160_gb300.build``) and bind its ABI."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or _LIB_PATH
+        if not os.path.exists(p):
+            raise RuntimeError(f"{p} is not built; run `python -m paper_2602_07160_gb300.build`")
+        lib = ctypes.CDLL(p)
+        vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        sig = [vp, vp, vp, vp, vp, vp, i, i, i, i, i]
+        lib.fem_fwd.argtypes = sig + [vp]
+        lib.fem_fwd_ws.argtypes = sig + [vp, sz, vp]
+        lib.fem_fwd_f32.argtypes = sig + [vp]
+        lib.fem_fwd_host.argtypes = sig + [vp]
+        lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
+        lib.fem_fwd_workspace_bytes.restype = sz
+        lib.fem_check_device_error.argtypes = [vp]
+        lib.fem_last_fixup_rows.argtypes = [vp]
+        lib.fem_set_kernel_events.argtypes = [vp, vp]
+        lib.fem_set_kernel_events.restype = i
+        lib.fem_status_str.argtypes = [i]
+        lib.fem_status_str.restype = ctypes.c_char_p
+        for name in ("fem_fwd", "fem_fwd_ws", "fem_fwd_f32", "fem_fwd_host", "fem_check_device_error",
+                     "fem_last_fixup_rows"):
+            getattr(lib, name).restype = i
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream, device):
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check_qkvb(q, k, v, beta, dtype, device_type):
+    if q.dim() != 4 or k.shape != q.shape or v.shape != q.shape:
+        raise ValueError("q, k, v must share the shape [B, H, T, d]")
+    B, H, T, d = q.shape
+    if beta.shape != (H, d) or beta.dtype != torch.float32:
+        raise ValueError("beta must be float32 [H, d]")
+    for name, t in (("q", q), ("k", k), ("v", v), ("beta", beta)):
+        if t.dtype != (torch.float32 if name == "beta" else dtype):
+            raise ValueError(f"{name} has dtype {t.dtype}")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+        if t.device.type != device_type:
+            raise ValueError(f"{name} must be on {device_type}")
+    return B, H, T, d
+
+
+def _outputs(q, out, lse, device):
+    B, H, T, d = q.shape
+    if out is None:
+        out = torch.empty((B, H, T, d), dtype=torch.float32, device=device)
+    if lse is None:
+        lse = torch.empty((B, H, T), dtype=torch.float32, device=device)
+    if out.shape != (B, H, T, d) or out.dtype != torch.float32 or not out.is_contiguous():
+        raise ValueError("out must be contiguous float32 [B, H, T, d]")
+    if lse is not False and (lse.shape != (B, H, T) or lse.dtype != torch.float32 or not lse.is_contiguous()):
+        raise ValueError("lse must be contiguous float32 [B, H, T]")
+    return out, lse
+
+
+def fem_fwd(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None):
+    """The read on bf16 CUDA tensors (tensor-core path).  Returns (out, lse).
+
+    Pass ``lse=False`` to skip the log-normaliser output."""
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.bfloat16, "cuda")
+    out, lse = _outputs(q, out, lse, q.device)
+    rc = load().fem_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), None if lse is False else _ptr(lse),
+                        B, H, T, d, int(bool(causal)), _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_fwd", rc)
+    return out, (None if lse is False else lse)
+
+
+def workspace_bytes(B: int, H: int, T: int, d: int, causal: bool = True) -> int:
+    return int(load().fem_fwd_workspace_bytes(B, H, T, d, int(bool(causal))))
+
+
+def fem_fwd_ws(q, k, v, beta, workspace, causal: bool = True, out=None, lse=None, stream=None):
+    """fem_fwd with a caller-owned uint8 CUDA workspace of ``workspace_bytes()`` bytes."""
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.bfloat16, "cuda")
+    out, lse = _outputs(q, out, lse, q.device)
+    rc = load().fem_fwd_ws(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), None if lse is False else _ptr(lse),
+                           B, H, T, d, int(bool(causal)), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                           _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_fwd_ws", rc)
+    return out, (None if lse is False else lse)
+
+
+def fem_fwd_f32(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None):
+    """The read on fp32 CUDA tensors (CUDA-core path).  Returns (out, lse)."""
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.float32, "cuda")
+    out, lse = _outputs(q, out, lse, q.device)
+    rc = load().fem_fwd_f32(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), None if lse is False else _ptr(lse),
+                            B, H, T, d, int(bool(causal)), _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_fwd_f32", rc)
+    return out, (None if lse is False else lse)
+
+
+def fem_fwd_host(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None, device=None):
+    """The read on HOST (ideally pinned) bf16 tensors: copies in, computes, copies out."""
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.bfloat16, "cpu")
+    out, lse = _outputs(q, out, lse, "cpu")
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    rc = load().fem_fwd_host(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), None if lse is False else _ptr(lse),
+                             B, H, T, d, int(bool(causal)), _stream(stream, dev))
+    if rc != 0:
+        raise FemError("fem_fwd_host", rc)
+    return out, (None if lse is False else lse)
+
+
+def check_device_error(stream=None, device=None):
+    """Synchronise and raise FemError if a kernel gave up on a bounded wait."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    rc = load().fem_check_device_error(_stream(stream, dev))
+    if rc != 0:
+        raise FemError("fem_check_device_error", rc)
+
+
+def set_kernel_events(start, stop):
+    """Have the next bf16 read of this thread record torch CUDA events around its tensor-core kernel."""
+    load().fem_set_kernel_events(ctypes.c_void_p(start.cuda_event), ctypes.c_void_p(stop.cuda_event))
+
+
+def last_fixup_rows(stream=None, device=None) -> int:
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    return int(load().fem_last_fixup_rows(_stream(stream, dev)))

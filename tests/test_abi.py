@@ -1,0 +1,76 @@
+"""The C ABI library builds, loads and exports what include/fem.h declares (CPU only)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2602_07160_gb300 import build, fem
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "fem.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(fem_[a-z0-9_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return fem.load()
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    assert names == sorted(fem.EXPORTS), names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    raw = ctypes.CDLL(fem.library_path())
+    for name in _declared():
+        assert hasattr(raw, name), f"{name} missing from libfem.so"
+
+
+def test_status_strings(lib):
+    for code, name in fem.STATUS.items():
+        assert lib.fem_status_str(code).decode() == name
+    assert lib.fem_status_str(99).decode() == "FEM_ERR_UNKNOWN"
+
+
+def test_workspace_bytes(lib):
+    assert lib.fem_fwd_workspace_bytes(0, 1, 1, 64, 1) == 0
+    assert lib.fem_fwd_workspace_bytes(1, 1, -3, 64, 1) == 0
+    a = lib.fem_fwd_workspace_bytes(4, 16, 8192, 128, 1)
+    b = lib.fem_fwd_workspace_bytes(4, 16, 8192, 128, 0)
+    assert a > b > 0 and a % 256 == 0 and b % 256 == 0
+
+
+def _call(lib, fn, q=16, k=16, v=16, beta=16, out=16, lse=0, B=1, H=1, T=8, d=64, causal=1):
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    return getattr(lib, fn)(p(q), p(k), p(v), p(beta), p(out), p(lse), B, H, T, d, causal, None)
+
+
+@pytest.mark.parametrize("fn", ["fem_fwd", "fem_fwd_f32", "fem_fwd_host"])
+def test_argument_errors_are_synchronous(lib, fn):
+    """Invalid arguments are rejected on the host before any CUDA call."""
+    assert _call(lib, fn, q=0) == 1
+    assert _call(lib, fn, beta=0) == 1
+    assert _call(lib, fn, out=0) == 1
+    assert _call(lib, fn, B=0) == 1
+    assert _call(lib, fn, T=-1) == 1
+    assert _call(lib, fn, causal=2) == 1
+    if fn != "fem_fwd_host":
+        assert _call(lib, fn, q=24) == 1  # not 16-byte aligned
+
+
+def test_unsupported_head_dim(lib):
+    assert _call(lib, "fem_fwd", d=96) == 2
+    assert _call(lib, "fem_fwd_host", d=32) == 2
+    assert _call(lib, "fem_fwd_f32", d=300) == 2
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    with pytest.raises(RuntimeError):
+        fem.load(str(tmp_path / "missing.so"))

@@ -1,0 +1,198 @@
+"""GPU read against the float64 oracle, element by element (needs a GB300).
+
+Tolerances are the target's: bf16 inputs -> fp32 output within max abs 2e-2
+and mean abs 2e-3 of the oracle evaluated on the same bf16-rounded inputs
+upcast to double; fp32 inputs within 1e-4.  Small cases span several key
+tiles with ragged tails; the five workloads run at full size and are
+compared on sampled rows (the oracle's row entry point) that always include
+the first rows of a head (the causal rows with the fewest keys, where the
+exact fix-up applies) and the last tile.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2602_07160_gb300 import build, fem
+from paper_2602_07160_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+BF16_MAX, BF16_MEAN = 2e-2, 2e-3
+F32_MAX = 1e-4
+LSE_MAX = 2e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    return fem.load()
+
+
+def _gpu_bf16(q, k, v, beta, causal):
+    dev = torch.device("cuda", 0)
+    qd, kd, vd, bd = (x.to(dev) for x in (q, k, v, beta))
+    out = torch.full(q.shape, float("nan"), dtype=torch.float32, device=dev)  # poisoned: every element must be written
+    out, lse = fem.fem_fwd(qd, kd, vd, bd, causal=causal, out=out)
+    fem.check_device_error()
+    return out.cpu().double().numpy(), lse.cpu().double().numpy()
+
+
+def _assert_close(out, ref, max_tol=BF16_MAX, mean_tol=BF16_MEAN, what=""):
+    assert np.isfinite(out).all(), f"{what}: non-finite output"
+    err = np.abs(out - ref)
+    mx, mn = float(err.max()), float(err.mean())
+    where = np.unravel_index(int(err.argmax()), err.shape)
+    assert mx <= max_tol and mn <= mean_tol, f"{what}: max {mx:.3e} at {where}, mean {mn:.3e}"
+    return mx, mn
+
+
+SMALL = [
+    # B, H, T, d, causal
+    (1, 2, 1, 64, True),
+    (1, 2, 2, 128, True),
+    (2, 2, 127, 64, True),
+    (2, 3, 129, 128, True),
+    (1, 2, 300, 128, True),
+    (2, 2, 384, 64, True),
+    (1, 2, 1, 128, False),
+    (2, 2, 129, 64, False),
+    (2, 3, 197, 64, False),
+    (1, 2, 300, 128, False),
+]
+
+
+@pytest.mark.parametrize("B,H,T,d,causal", SMALL)
+def test_small_cases_full_compare(B, H, T, d, causal):
+    q, k, v, beta = W.make_custom(B, H, T, d, seed=T + d)
+    out, lse = _gpu_bf16(q, k, v, beta, causal)
+    ref, ref_lse = oracle.fem_read(q, k, v, beta, causal)
+    _assert_close(out, ref, what=f"B{B} H{H} T{T} d{d} causal={causal}")
+    assert np.abs(lse - ref_lse).max() <= LSE_MAX
+
+
+BETA_SWEEP = [0.0, 1e-4, 1e-3, 1e-2, 0.1, 0.5, 1.0, 5.0, 20.0, 100.0, 1e3]
+
+
+@pytest.mark.parametrize("d,causal", [(64, True), (128, True), (128, False)])
+def test_beta_sweep(d, causal):
+    B, H, T = 1, 2, 320
+    q, k, v, _ = W.make_custom(B, H, T, d, seed=7)
+    beta = W.beta_grid(H, d, BETA_SWEEP)
+    out, _ = _gpu_bf16(q, k, v, beta, causal)
+    ref, _ = oracle.fem_read(q, k, v, beta, causal)
+    _assert_close(out, ref, what=f"beta sweep d{d} causal={causal}")
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_student_t_values_wide_beta(d):
+    q, k, v, beta = W.make_custom(1, 3, 520, d, beta_lo=1e-3, beta_hi=100.0, v_dist="student_t3",
+                                  const_channels=4, seed=11)
+    out, _ = _gpu_bf16(q, k, v, beta, True)
+    ref, _ = oracle.fem_read(q, k, v, beta, True)
+    _assert_close(out, ref, what="student-t")
+
+
+def test_first_row_is_first_value_and_constant_channels():
+    """P1 and P2 on the device: row 0 reads v_0; constant channels read the constant."""
+    q, k, v, beta = W.make_custom(2, 2, 260, 128, beta_lo=1e-3, beta_hi=100.0, const_channels=4, seed=3)
+    out, _ = _gpu_bf16(q, k, v, beta, True)
+    vf = v.double().numpy()
+    assert np.abs(out[:, :, 0, :] - vf[:, :, 0, :]).max() <= BF16_MAX
+    assert np.abs(out[..., :4] - vf[:, :, :1, :4]).max() <= 1e-5
+
+
+def test_beta_zero_is_softmax_attention():
+    """beta = 0 gives the prior mean, i.e. softmax attention (checked against torch SDPA in fp32)."""
+    q, k, v, _ = W.make_custom(2, 2, 300, 128, seed=5)
+    beta = torch.zeros(2, 128)
+    out, _ = _gpu_bf16(q, k, v, beta, True)
+    ref = torch.nn.functional.scaled_dot_product_attention(q.double(), k.double(), v.double(), is_causal=True)
+    _assert_close(out, ref.numpy(), what="beta=0 vs sdpa")
+
+
+def test_deterministic():
+    q, k, v, beta = W.make_custom(1, 2, 300, 128, seed=9)
+    a, la = _gpu_bf16(q, k, v, beta, True)
+    b, lb = _gpu_bf16(q, k, v, beta, True)
+    assert np.array_equal(a, b) and np.array_equal(la, lb)
+
+
+def test_workspace_variant_matches():
+    q, k, v, beta = W.make_custom(1, 2, 300, 64, seed=4)
+    dev = torch.device("cuda", 0)
+    qd, kd, vd, bd = (x.to(dev) for x in (q, k, v, beta))
+    o1, l1 = fem.fem_fwd(qd, kd, vd, bd, causal=True)
+    ws = torch.empty(fem.workspace_bytes(1, 2, 300, 64, True), dtype=torch.uint8, device=dev)
+    o2, l2 = fem.fem_fwd_ws(qd, kd, vd, bd, ws, causal=True)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+
+
+def test_host_entry_point_matches():
+    q, k, v, beta = W.make_custom(1, 2, 300, 128, seed=6)
+    dev = torch.device("cuda", 0)
+    o1, l1 = fem.fem_fwd(*(x.to(dev) for x in (q, k, v, beta)), causal=True)
+    o2, l2 = fem.fem_fwd_host(q.pin_memory(), k.pin_memory(), v.pin_memory(), beta.pin_memory(), causal=True)
+    assert torch.equal(o1.cpu(), o2) and torch.equal(l1.cpu(), l2)
+
+
+# ---------------------------------------------------------------------------
+# fp32-input path
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("B,H,T,d,causal", [(1, 1, 64, 16, True), (1, 2, 300, 64, True), (2, 1, 130, 128, False),
+                                            (1, 1, 5, 256, True), (1, 1, 33, 7, False)])
+def test_f32_path(B, H, T, d, causal):
+    q, k, v, beta = W.make_custom(B, H, T, d, dtype="f32", beta_lo=1e-3, beta_hi=100.0, seed=B + T)
+    beta[0, 0] = 0.0
+    dev = torch.device("cuda", 0)
+    out, lse = fem.fem_fwd_f32(*(x.to(dev) for x in (q, k, v, beta)), causal=causal)
+    ref, ref_lse = oracle.fem_read(q, k, v, beta, causal)
+    _assert_close(out.cpu().double().numpy(), ref, max_tol=F32_MAX, mean_tol=F32_MAX, what="f32")
+    assert np.abs(lse.cpu().double().numpy() - ref_lse).max() <= 1e-5
+
+
+# ---------------------------------------------------------------------------
+# The five workloads at full size
+# ---------------------------------------------------------------------------
+def test_workload_tiny_f32_full():
+    w = W.WORKLOADS["tiny_f32_causal"]
+    q, k, v, beta = W.make_inputs(w)
+    dev = torch.device("cuda", 0)
+    out, _ = fem.fem_fwd_f32(*(x.to(dev) for x in (q, k, v, beta)), causal=w.causal)
+    ref, _ = oracle.fem_read(q, k, v, beta, w.causal)
+    _assert_close(out.cpu().double().numpy(), ref, max_tol=F32_MAX, mean_tol=F32_MAX, what=w.name)
+
+
+def test_workload_vit_full():
+    w = W.WORKLOADS["vit_s_full_prior"]
+    q, k, v, beta = W.make_inputs(w)
+    out, _ = _gpu_bf16(q, k, v, beta, w.causal)
+    ref, _ = oracle.fem_read(q, k, v, beta, w.causal)
+    _assert_close(out, ref, what=w.name)
+
+
+def _sample_rows(w, n_random, seed=0):
+    rows_per_bh = w.T
+    r = np.random.default_rng(seed)
+    first = np.arange(min(384, w.T))                     # head (0, 0): the first three tiles
+    last_bh = w.B * w.H - 1
+    last = last_bh * rows_per_bh + np.arange(max(0, w.T - 128), w.T)  # last tile of the last head
+    rand = r.choice(w.B * w.H * w.T, size=n_random, replace=False)
+    return np.unique(np.concatenate([first, last, rand]))
+
+
+@pytest.mark.parametrize("name,n_random", [("lm_causal_d64", 3000), ("lm_causal_d128", 1500),
+                                           ("long_causal_student_t", 600)])
+def test_workload_full_size_sampled(name, n_random):
+    w = W.WORKLOADS[name]
+    q, k, v, beta = W.make_inputs(w)
+    out, lse = _gpu_bf16(q, k, v, beta, w.causal)
+    rows = _sample_rows(w, n_random)
+    ref, ref_lse = oracle.fem_read_rows(q, k, v, beta, w.causal, rows)
+    got = out.reshape(-1, w.d)[rows]
+    _assert_close(got, ref, what=name)
+    assert np.abs(lse.reshape(-1)[rows] - ref_lse).max() <= LSE_MAX
+    if name == "long_causal_student_t":
+        vf = v.double().numpy()
+        assert np.abs(out[..., :4] - vf[:, :, :1, :4]).max() <= 1e-5
