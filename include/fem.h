@@ -102,6 +102,28 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
                  void *stream);
 
 /*
+ * fem_fwd_noalloc -- fem_fwd for callers that may not allocate device memory
+ * during the call (for example a plugin whose execute callback is not
+ * allowed to allocate, or a service that reserves all device memory up
+ * front).  The paper has no counterpart; this is an interface convenience.
+ * Same arguments, layout and results as fem_fwd; the caller still passes
+ * every input and output.  Instead of cudaMallocAsync it uses a fixed
+ * 16 MiB scratch array compiled into the library, which every GPU that
+ * loads the library holds until the process exits.  Problems needing more
+ * workspace than that (fem_fwd_workspace_bytes() > 16 MiB, which for a
+ * causal read means B*H*T*ceil(d/32) beyond about 2^20) return
+ * FEM_ERR_NO_MEMORY before anything is enqueued.  It calls no allocation routine.  The first call on
+ * a device looks up the scratch address on that device (cudaGetSymbolAddress),
+ * so make that first call outside any stream capture.  All calls share the one
+ * array and it keeps the previous call's contents (the call clears what must
+ * start at zero): calls that overlap on the GPU, from any stream or thread,
+ * race and must be serialised by the caller.
+ */
+int fem_fwd_noalloc(const void *q, const void *k, const void *v,
+                    const float *beta, float *out, float *lse, int B, int H,
+                    int T, int d, int causal, void *stream);
+
+/*
  * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
  * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
  * on a bounded wait since the last check (the word is cleared), or

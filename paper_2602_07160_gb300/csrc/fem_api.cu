@@ -116,6 +116,36 @@ int check_common(const void *q, const void *k, const void *v, const float *beta,
   return FEM_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Fixed scratch for fem_fwd_noalloc.  Some callers may not allocate device
+// memory while they run the read (for example a plugin whose execute callback
+// must not allocate, or a service that hands out all device memory up front),
+// so that entry point uses this file-scope array as its workspace instead of
+// cudaMallocAsync.  Every GPU that loads the library holds it until exit.
+// Host code must not use the array's name as a device address; the entry
+// point looks the address up once per device with cudaGetSymbolAddress.
+// ---------------------------------------------------------------------------
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;  // 16 MiB
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_static_mutex;
+void *g_static_addr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device (set up on the
+// first call per device, with that device current).
+int static_scratch(void **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FEM_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_static_mutex);
+  if (!g_static_addr[dev]) {
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) return FEM_ERR_CUDA;
+    g_static_addr[dev] = ptr;
+  }
+  *out = g_static_addr[dev];
+  return FEM_OK;
+}
+
 }  // namespace
 }  // namespace fem
 
@@ -242,6 +272,18 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
   if (rc != FEM_OK) return rc;
   if (ef != cudaSuccess) return map_cuda(ef);
   return map_cuda(es);
+}
+
+int fem_fwd_noalloc(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B,
+                    int H, int T, int d, int causal, void *stream) {
+  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  const size_t need = fem_fwd_workspace_bytes(B, H, T, d, causal);
+  if (need == 0 || need > kStaticScratchBytes) return FEM_ERR_NO_MEMORY;
+  void *scratch = nullptr;
+  if ((rc = static_scratch(&scratch)) != FEM_OK) return rc;
+  return fem_fwd_ws(q, k, v, beta, out, lse, B, H, T, d, causal, scratch, kStaticScratchBytes, stream);
 }
 
 int fem_set_kernel_events(void *start, void *stop) {

@@ -22,7 +22,8 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
           4: "FEM_ERR_TIMEOUT", 5: "FEM_ERR_NO_MEMORY"}
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
-           "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str"]
+           "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
+           "fem_fwd_noalloc"]
 
 
 class FemError(RuntimeError):
@@ -51,6 +52,8 @@ def load(path: str | None = None):
         lib.fem_fwd_ws.argtypes = sig + [vp, sz, vp]
         lib.fem_fwd_f32.argtypes = sig + [vp]
         lib.fem_fwd_host.argtypes = sig + [vp]
+        lib.fem_fwd_noalloc.argtypes = sig + [vp]
+        lib.fem_fwd_noalloc.restype = i
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
@@ -155,6 +158,22 @@ def fem_fwd_host(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=
                              B, H, T, d, int(bool(causal)), _stream(stream, dev))
     if rc != 0:
         raise FemError("fem_fwd_host", rc)
+    return out, (None if lse is False else lse)
+
+
+def fem_fwd_noalloc(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None):
+    """fem_fwd without device allocation (the library's fixed 16 MiB scratch).
+
+    For callers that may not allocate device memory during the read.  ``out``
+    and ``lse`` should be passed preallocated by such callers.  Calls that
+    overlap on the GPU share the scratch and race."""
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.bfloat16, "cuda")
+    out, lse = _outputs(q, out, lse, q.device)
+    rc = load().fem_fwd_noalloc(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out),
+                                None if lse is False else _ptr(lse), B, H, T, d, int(bool(causal)),
+                                _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_fwd_noalloc", rc)
     return out, (None if lse is False else lse)
 
 
