@@ -2,9 +2,10 @@
 // layout, TMA tensor maps and the launch sequence of the FEM read.
 //
 // bf16 path, in stream order:
-//   1. value_stats  (one read of V): channel modes, shift schedule, fix-up list
-//   2. fem_tc       (tcgen05): the read for every row and channel
-//   3. fixup        (causal only): exact fp32 recompute of the listed entries
+//   1. tile_stats, plan, bank: channel modes, shift schedule, the fp16 value
+//      bank (once per key tile), the fix-up list
+//   2. fem_tc (tcgen05): the read for every row and channel
+//   3. fixup (causal only): exact fp32 recompute of the listed entries
 #include <cudaTypedefs.h>
 
 #include <mutex>
@@ -65,13 +66,14 @@ int device_state(DeviceState **out) {
   return FEM_OK;
 }
 
-// [d, T, B*H] bf16 tensor, boxes of 64 channels x 128 rows, 128-byte swizzle.
-int make_map(CUtensorMap *map, const void *base, int BH, int T, int d) {
+// [d, T, B*H] 16-bit tensor, boxes of 64 channels x 128 rows, 128-byte swizzle.
+int make_map(CUtensorMap *map, const void *base, int BH, int T, int d,
+             CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(BH)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(T) * d * 2};
   cuuint32_t box[3] = {64, 128, 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+  CUresult r = g_encode(map, dtype, 3, const_cast<void *>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? FEM_OK : FEM_ERR_CUDA;
@@ -82,7 +84,7 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-  size_t chan, cpre, fixups, count, total;
+  size_t tstat, chan, cpre, shift, colmove, bank, fixups, count, total;
 };
 
 bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
@@ -91,10 +93,18 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   const size_t n_kt = (static_cast<size_t>(T) + kBlockK - 1) / kBlockK;
   const size_t groups = (static_cast<size_t>(d) + 31) / 32;
   size_t off = 0;
+  w->bank = off;
+  off += round256(BH * static_cast<size_t>(T) * d * 2);
+  w->tstat = off;
+  off += round256(BH * n_kt * d * sizeof(float4));
   w->chan = off;
   off += round256(BH * d * sizeof(ChanInfo));
   w->cpre = off;
   off += round256(BH * n_kt * d * sizeof(float));
+  w->shift = off;
+  off += round256(BH * n_kt * d * sizeof(float));
+  w->colmove = off;
+  off += round256(BH * n_kt * sizeof(int));
   w->fixups = off;
   off += causal ? round256(BH * n_kt * kBlockQ * groups * sizeof(FixupEntry)) : 0;
   w->count = off;
@@ -184,28 +194,34 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
 
   const int BH = B * H;
-  CUtensorMap tq, tk, tv;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  BankWorkspace bw;
+  bw.tstat = reinterpret_cast<float4 *>(ws + w.tstat);
+  bw.chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
+  bw.cpre = reinterpret_cast<float *>(ws + w.cpre);
+  bw.shift = reinterpret_cast<float *>(ws + w.shift);
+  bw.colmove = reinterpret_cast<int *>(ws + w.colmove);
+  bw.bank = reinterpret_cast<__half *>(ws + w.bank);
+  bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
+  bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
+
+  CUtensorMap tq, tk, te;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&tk, k, BH, T, d)) != FEM_OK) return rc;
-  if ((rc = make_map(&tv, v, BH, T, d)) != FEM_OK) return rc;
+  if ((rc = make_map(&te, bw.bank, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT16)) != FEM_OK) return rc;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  uint8_t *ws = static_cast<uint8_t *>(workspace);
-  ChanInfo *chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
-  float *cpre = reinterpret_cast<float *>(ws + w.cpre);
-  FixupEntry *fix = reinterpret_cast<FixupEntry *>(ws + w.fixups);
-  int *count = reinterpret_cast<int *>(ws + w.count);
-
-  cudaError_t e = cudaMemsetAsync(count, 0, sizeof(int), s);
-  if (e == cudaSuccess) e = launch_value_stats(v, beta, BH, H, T, d, causal, chan, cpre, fix, count, s);
+  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = launch_value_bank(v, beta, BH, H, T, d, causal, bw, s);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
-  if (e == cudaSuccess) e = launch_tc(d, tq, tk, tv, beta, chan, cpre, out, lse, BH, H, T, causal, ds->err, s);
+  if (e == cudaSuccess)
+    e = launch_tc(d, tq, tk, te, beta, bw.chan, bw.shift, bw.colmove, out, lse, BH, H, T, causal, ds->err, s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess) {
     if (causal)
-      e = launch_fixup(q, k, v, beta, out, H, T, d, fix, count, ds->last_fixup, ds->num_sms, s);
+      e = launch_fixup(q, k, v, beta, out, H, T, d, bw.fixups, bw.fixup_count, ds->last_fixup, ds->num_sms, s);
     else
       e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
   }

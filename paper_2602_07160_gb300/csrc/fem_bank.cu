@@ -1,0 +1,285 @@
+// Value-bank pre-pass of the FEM read: statistics, shift schedule and the
+// fp16 value bank, written once per key tile for every query tile to share.
+//
+//   tile_stats  (B*H x key tiles)  max, min and sum of v_.j over each tile of
+//                                  128 keys (valid keys only)
+//   plan        (B*H)              per channel: bank mode and linear anchor
+//                                  from the whole sequence; the running maximum
+//                                  cpre[kt] = max over tiles 0..kt; the shifted
+//                                  bank's shift c[kt], raised lazily along cpre
+//                                  (only when beta*(cpre - c) > kShiftLag);
+//                                  a per-tile flag when any shift moved
+//   bank        (B*H x key tiles)  E = bank(v) in fp16 with the tile's shift;
+//                                  causal: the (row, 32-channel group) entries
+//                                  of the tile's diagonal rows whose visible
+//                                  maximum lies more than kHazardTilt/beta below
+//                                  the shift, for the exact fix-up
+//
+// The shift is the per-channel LSE stabilisation of App. E ("Numerical
+// stability"), made online over key tiles; only keys < T enter it, and a
+// query tile's last key tile is its diagonal tile, so keys beyond a tile's
+// last row never raise the shift that tile's rows use.
+#include "fem_common.cuh"
+#include "fem_launch.h"
+
+namespace fem {
+
+// Thread layout shared by tile_stats and bank: 128 threads cover a [128 x D]
+// tile with 16-byte chunks; CPR chunks per row, RG row groups of RPG rows.
+template <int D>
+struct TileMap {
+  static constexpr int CPR = D / 8;
+  static constexpr int RG = 128 / CPR;
+  static constexpr int RPG = 128 / RG;
+};
+
+template <int D>
+__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T,
+                                                          float4 *__restrict__ tstat) {
+  using M = TileMap<D>;
+  __shared__ float s_max[M::RG][D], s_min[M::RG][D], s_sum[M::RG][D];
+  const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x;
+  const int cc = threadIdx.x % M::CPR, rg = threadIdx.x / M::CPR;
+  float mx[8], mn[8], sm[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    mx[u] = -INFINITY;
+    mn[u] = INFINITY;
+    sm[u] = 0.f;
+  }
+  const __nv_bfloat16 *vb = v + static_cast<size_t>(bh) * T * D;
+#pragma unroll 4
+  for (int i = 0; i < M::RPG; ++i) {
+    const int key = kt * kBlockK + rg * M::RPG + i;
+    if (key < T) {
+      const uint4 raw = *reinterpret_cast<const uint4 *>(vb + static_cast<size_t>(key) * D + cc * 8);
+      const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float2 f = __bfloat1622float2(p2[u]);
+        mx[2 * u] = fmaxf(mx[2 * u], f.x);
+        mx[2 * u + 1] = fmaxf(mx[2 * u + 1], f.y);
+        mn[2 * u] = fminf(mn[2 * u], f.x);
+        mn[2 * u + 1] = fminf(mn[2 * u + 1], f.y);
+        sm[2 * u] += f.x;
+        sm[2 * u + 1] += f.y;
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    s_max[rg][cc * 8 + u] = mx[u];
+    s_min[rg][cc * 8 + u] = mn[u];
+    s_sum[rg][cc * 8 + u] = sm[u];
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j < D; j += 128) {
+    float a = -INFINITY, b = INFINITY, c = 0.f;
+    for (int g = 0; g < M::RG; ++g) {
+      a = fmaxf(a, s_max[g][j]);
+      b = fminf(b, s_min[g][j]);
+      c += s_sum[g][j];
+    }
+    tstat[(static_cast<size_t>(bh) * n_kt + kt) * D + j] = make_float4(a, b, c, 0.f);
+  }
+}
+
+__global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta, int H, int T, int d,
+                            int n_kt, ChanInfo *__restrict__ chan, float *__restrict__ cpre,
+                            float *__restrict__ shift, int *__restrict__ colmove) {
+  const int bh = blockIdx.x, j = threadIdx.x, h = bh % H;
+  const float b = beta[h * d + j];
+  const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * d + j;
+  float gmax = -INFINITY, gmin = INFINITY, gsum = 0.f;
+  for (int kt = 0; kt < n_kt; ++kt) {
+    const float4 s = ts[static_cast<size_t>(kt) * d];
+    gmax = fmaxf(gmax, s.x);
+    gmin = fminf(gmin, s.y);
+    gsum += s.z;
+  }
+  const float mean = gsum / static_cast<float>(T);
+  ChanInfo ci;
+  if (b > 0.f) {
+    const float hi = gmin + kLinearLowTilt / b;
+    const float lo = gmax - log1pf(kLinearBankMax * b) / b;
+    ci.linear = lo <= hi ? 1.f : 0.f;
+    ci.c_lin = fminf(fmaxf(mean, lo), hi);
+  } else {
+    ci.linear = 1.f;
+    ci.c_lin = mean;
+  }
+  chan[bh * d + j] = ci;
+  const bool lin = ci.linear != 0.f;
+  float cp = -INFINITY, cl = -INFINITY;
+  for (int kt = 0; kt < n_kt; ++kt) {
+    cp = fmaxf(cp, ts[static_cast<size_t>(kt) * d].x);
+    const float prev = cl;
+    if (lin) {
+      cl = ci.c_lin;
+    } else if (cl == -INFINITY || b * (cp - cl) > kShiftLag) {
+      cl = cp;
+    }
+    const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * d + j;
+    cpre[o] = cp;
+    shift[o] = cl;
+    const int moved = (!lin && kt > 0 && cl != prev) ? 1 : 0;
+    const int any = __syncthreads_or(moved);
+    if (j == 0) colmove[bh * n_kt + kt] = any;
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(128) bank_kernel(const __nv_bfloat16 *__restrict__ v,
+                                                    const float *__restrict__ beta, const ChanInfo *__restrict__ chan,
+                                                    const float *__restrict__ cpre, const float *__restrict__ shift,
+                                                    int H, int T, int causal, __half *__restrict__ bank,
+                                                    FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count) {
+  using M = TileMap<D>;
+  __shared__ float s_a[D], s_b[D], s_c[D], s_beta[D], s_lin[D], s_prev[D];
+  __shared__ float s_lmax[M::RG][D];
+  __shared__ int s_first[D];
+  const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x, h = bh % H;
+  const int tid = threadIdx.x;
+  const int cc = tid % M::CPR, rg = tid / M::CPR;
+  for (int j = tid; j < D; j += 128) {
+    const float b = beta[h * D + j];
+    const ChanInfo ci = chan[bh * D + j];
+    const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
+    const float c = shift[o];
+    s_beta[j] = b;
+    s_lin[j] = ci.linear;
+    s_c[j] = c;
+    s_prev[j] = kt > 0 ? cpre[o - D] : -INFINITY;
+    if (ci.linear != 0.f) {
+      s_a[j] = b > 0.f ? 1.f / b : 0.f;  // linear bank: 1/beta
+      s_b[j] = 0.f;
+    } else {
+      s_a[j] = b * kLog2e;  // shifted bank: E = ex2(a v + b)
+      s_b[j] = (kBankOffset - b * c) * kLog2e;
+    }
+    s_first[j] = kBlockK;
+  }
+  __syncthreads();
+
+  const __nv_bfloat16 *vb = v + static_cast<size_t>(bh) * T * D;
+  __half *eb = bank + static_cast<size_t>(bh) * T * D;
+  float lmax[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) lmax[u] = -INFINITY;
+#pragma unroll 2
+  for (int i = 0; i < M::RPG; ++i) {
+    const int key = kt * kBlockK + rg * M::RPG + i;
+    if (key >= T) break;
+    const uint4 raw = *reinterpret_cast<const uint4 *>(vb + static_cast<size_t>(key) * D + cc * 8);
+    const __nv_bfloat16 *vin = reinterpret_cast<const __nv_bfloat16 *>(&raw);
+    __align__(16) __half e[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int j = cc * 8 + u;
+      const float x = __bfloat162float(vin[u]);
+      lmax[u] = fmaxf(lmax[u], x);
+      float val;
+      if (s_lin[j] != 0.f) {
+        // D = expm1(y)/beta, y = beta (v - c) >= -1: Taylor series of expm1(y)/y
+        // for |y| < 1/2 (truncation < 4e-6 relative), e^y - 1 beyond
+        const float xs = x - s_c[j];
+        const float y = s_beta[j] * xs;
+        if (fabsf(y) < 0.5f) {
+          float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
+          poly = fmaf(y, poly, 1.f / 24.f);
+          poly = fmaf(y, poly, 1.f / 6.f);
+          poly = fmaf(y, poly, 0.5f);
+          poly = fmaf(y, poly, 1.f);
+          val = xs * poly;
+        } else {
+          val = (ex2_approx(y * kLog2e) - 1.f) * s_a[j];
+        }
+      } else {
+        val = ex2_approx(fmaf(s_a[j], x, s_b[j]));
+      }
+      e[u] = __float2half_rn(val);
+    }
+    *reinterpret_cast<uint4 *>(eb + static_cast<size_t>(key) * D + cc * 8) = *reinterpret_cast<const uint4 *>(e);
+  }
+  if (!causal) return;
+
+  // Diagonal-tile hazard: the first row of this tile at which the visible
+  // maximum of each shifted channel comes within kHazardTilt/beta of the
+  // tile's shift; rows before it are recomputed exactly.
+#pragma unroll
+  for (int u = 0; u < 8; ++u) s_lmax[rg][cc * 8 + u] = lmax[u];
+  __syncthreads();
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    const int j = cc * 8 + u;
+    if (s_lin[j] != 0.f) continue;
+    float run = s_prev[j];
+    for (int g = 0; g < rg; ++g) run = fmaxf(run, s_lmax[g][j]);
+    const float b = s_beta[j], c = s_c[j];
+    for (int i = 0; i < M::RPG; ++i) {
+      const int key = kt * kBlockK + rg * M::RPG + i;
+      if (key >= T) break;
+      run = fmaxf(run, __bfloat162float(vb[static_cast<size_t>(key) * D + j]));
+      if (b * (c - run) <= kHazardTilt) {
+        atomicMin(&s_first[j], rg * M::RPG + i);
+        break;
+      }
+    }
+  }
+  __syncthreads();
+  const int warp = tid >> 5, lane = tid & 31;
+  if (warp < D / 32) {
+    const int g = warp;
+    int hz = s_first[g * 32 + lane];
+    if (hz == kBlockK) hz = 0;  // linear channel, or no valid key
+    int hz_max = hz;
+    for (int off = 16; off; off >>= 1) hz_max = max(hz_max, __shfl_xor_sync(0xffffffffu, hz_max, off));
+    const int t0 = kt * kBlockQ;
+    const int n_rows = min(hz_max, T - t0);
+    if (n_rows > 0) {
+      int base = 0;
+      if (lane == 0) base = atomicAdd(fixup_count, n_rows);
+      base = __shfl_sync(0xffffffffu, base, 0);
+      for (int r = lane; r < n_rows; r += 32) {
+        unsigned mask = 0;
+        for (int c = 0; c < 32; ++c) {
+          int hc = s_first[g * 32 + c];
+          if (hc == kBlockK) hc = 0;
+          mask |= (hc > r ? 1u : 0u) << c;
+        }
+        FixupEntry e;
+        e.row = bh * T + t0 + r;
+        e.group = g;
+        e.mask = mask;
+        e.pad = 0;
+        fixups[base + r] = e;
+      }
+    }
+  }
+}
+
+cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
+                              const BankWorkspace &w, cudaStream_t stream) {
+  const int n_kt = (T + kBlockK - 1) / kBlockK;
+  const dim3 grid(n_kt, BH);
+  const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
+  if (d == 64)
+    tile_stats_kernel<64><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+  else if (d == 128)
+    tile_stats_kernel<128><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+  else
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  plan_kernel<<<BH, d, 0, stream>>>(w.tstat, beta, H, T, d, n_kt, w.chan, w.cpre, w.shift, w.colmove);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (d == 64)
+    bank_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
+                                              w.fixup_count);
+  else
+    bank_kernel<128><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
+                                               w.fixup_count);
+  return cudaGetLastError();
+}
+
+}  // namespace fem

@@ -8,15 +8,26 @@
 
 namespace fem {
 
-// Value statistics, shift schedule and exact-recompute list (one read of V).
-cudaError_t launch_value_stats(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
-                               ChanInfo *chan, float *cpre, FixupEntry *fixups, int *fixup_count,
-                               cudaStream_t stream);
+// Device workspace of the value-bank pre-pass (all arrays caller-owned).
+struct BankWorkspace {
+  float4 *tstat;            // [B*H, key tiles, d]: max, min, sum of v per tile
+  ChanInfo *chan;           // [B*H, d]
+  float *cpre;              // [B*H, key tiles, d]: running maximum of v
+  float *shift;             // [B*H, key tiles, d]: the bank's shift for each tile
+  int *colmove;             // [B*H, key tiles]: 1 when some shift moved at the tile
+  __half *bank;             // [B*H, T, d]: the value bank, fp16
+  FixupEntry *fixups;       // exact-recompute list (causal)
+  int *fixup_count;         // its length (zeroed before the pre-pass)
+};
+
+// Statistics, plan and value bank (two reads of V, one write of the bank).
+cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
+                              const BankWorkspace &w, cudaStream_t stream);
 
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
-cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, const float *beta,
-                      const ChanInfo *chan, const float *cpre, float *out, float *lse, int BH, int H, int T,
-                      int causal, unsigned *err, cudaStream_t stream);
+cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const float *beta,
+                      const ChanInfo *chan, const float *shift, const int *colmove, float *out, float *lse, int BH,
+                      int H, int T, int causal, unsigned *err, cudaStream_t stream);
 
 // Exact recompute of the listed (row, channel group) entries.
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, float *out, int H, int T,
