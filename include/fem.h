@@ -110,9 +110,9 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
  * every input and output.  Instead of cudaMallocAsync it uses a fixed
  * 16 MiB scratch array compiled into the library, which every GPU that
  * loads the library holds until the process exits.  Problems needing more
- * workspace than that (fem_fwd_workspace_bytes() > 16 MiB, which for a
- * causal read means B*H*T*ceil(d/32) beyond about 2^20) return
- * FEM_ERR_NO_MEMORY before anything is enqueued.  It calls no allocation routine.  The first call on
+ * workspace than that (fem_fwd_workspace_bytes() > 16 MiB, about 2*d + 60
+ * bytes per row (b, h, t) for a causal read) return FEM_ERR_NO_MEMORY before
+ * anything is enqueued.  It calls no allocation routine.  The first call on
  * a device looks up the scratch address on that device (cudaGetSymbolAddress),
  * so make that first call outside any stream capture.  All calls share the one
  * array and it keeps the previous call's contents (the call clears what must
@@ -132,10 +132,10 @@ int fem_fwd_noalloc(const void *q, const void *k, const void *v,
 int fem_check_device_error(void *stream);
 
 /*
- * fem_last_fixup_rows -- synchronises `stream` and returns the number of
- * (row, 32-channel group) entries the last bf16 read on the current device
- * recomputed exactly (causal rows whose visible values lie far below the
- * shared value-bank shift).  Diagnostic; -1 on error.
+ * fem_last_fixup_rows -- synchronises `stream` and returns the number of rows
+ * the last bf16 read on the current device recomputed exactly for some of
+ * their channels (causal rows whose visible values lie far below the shared
+ * value-bank shift).  Diagnostic; -1 on error.
  */
 int fem_last_fixup_rows(void *stream);
 

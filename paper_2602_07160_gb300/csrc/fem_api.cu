@@ -84,14 +84,13 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-  size_t tstat, chan, cpre, shift, colmove, bank, fixups, count, total;
+  size_t tstat, chan, cpre, shift, rfac, colmask, bank, fixups, count, total;
 };
 
 bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0) return false;
   const size_t BH = static_cast<size_t>(B) * H;
   const size_t n_kt = (static_cast<size_t>(T) + kBlockK - 1) / kBlockK;
-  const size_t groups = (static_cast<size_t>(d) + 31) / 32;
   size_t off = 0;
   w->bank = off;
   off += round256(BH * static_cast<size_t>(T) * d * 2);
@@ -103,10 +102,12 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += round256(BH * n_kt * d * sizeof(float));
   w->shift = off;
   off += round256(BH * n_kt * d * sizeof(float));
-  w->colmove = off;
-  off += round256(BH * n_kt * sizeof(int));
+  w->rfac = off;
+  off += round256(BH * n_kt * d * sizeof(float));
+  w->colmask = off;
+  off += round256(BH * n_kt * 4 * sizeof(unsigned));
   w->fixups = off;
-  off += causal ? round256(BH * n_kt * kBlockQ * groups * sizeof(FixupEntry)) : 0;
+  off += causal ? round256(BH * n_kt * kBlockQ * sizeof(FixupEntry)) : 0;
   w->count = off;
   off += 256;
   w->total = off;
@@ -200,7 +201,8 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   bw.chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
   bw.cpre = reinterpret_cast<float *>(ws + w.cpre);
   bw.shift = reinterpret_cast<float *>(ws + w.shift);
-  bw.colmove = reinterpret_cast<int *>(ws + w.colmove);
+  bw.rfac = reinterpret_cast<float *>(ws + w.rfac);
+  bw.colmask = reinterpret_cast<unsigned *>(ws + w.colmask);
   bw.bank = reinterpret_cast<__half *>(ws + w.bank);
   bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
@@ -217,7 +219,8 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
   if (e == cudaSuccess)
-    e = launch_tc(d, tq, tk, te, beta, bw.chan, bw.shift, bw.colmove, out, lse, BH, H, T, causal, ds->err, s);
+    e = launch_tc(d, tq, tk, te, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, out, lse, BH, H, T, causal, ds->err,
+                  s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess) {
     if (causal)

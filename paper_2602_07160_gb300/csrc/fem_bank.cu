@@ -8,7 +8,7 @@
 //                                  cpre[kt] = max over tiles 0..kt; the shifted
 //                                  bank's shift c[kt], raised lazily along cpre
 //                                  (only when beta*(cpre - c) > kShiftLag);
-//                                  a per-tile flag when any shift moved
+//                                  a per-tile mask of the channels whose shift moved
 //   bank        (B*H x key tiles)  E = bank(v) in fp16 with the tile's shift;
 //                                  causal: the (row, 32-channel group) entries
 //                                  of the tile's diagonal rows whose visible
@@ -86,7 +86,7 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
 
 __global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta, int H, int T, int d,
                             int n_kt, ChanInfo *__restrict__ chan, float *__restrict__ cpre,
-                            float *__restrict__ shift, int *__restrict__ colmove) {
+                            float *__restrict__ shift, float *__restrict__ rfac, unsigned *__restrict__ colmask) {
   const int bh = blockIdx.x, j = threadIdx.x, h = bh % H;
   const float b = beta[h * d + j];
   const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * d + j;
@@ -123,20 +123,20 @@ __global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__res
     cpre[o] = cp;
     shift[o] = cl;
     const int moved = (!lin && kt > 0 && cl != prev) ? 1 : 0;
-    const int any = __syncthreads_or(moved);
-    if (j == 0) colmove[bh * n_kt + kt] = any;
+    rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
+    const unsigned bits = __ballot_sync(0xffffffffu, moved);
+    if ((j & 31) == 0) colmask[(static_cast<size_t>(bh) * n_kt + kt) * 4 + (j >> 5)] = bits;
   }
 }
 
 template <int D>
-__global__ void __launch_bounds__(128) bank_kernel(const __nv_bfloat16 *__restrict__ v,
+__global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__restrict__ v,
                                                     const float *__restrict__ beta, const ChanInfo *__restrict__ chan,
                                                     const float *__restrict__ cpre, const float *__restrict__ shift,
                                                     int H, int T, int causal, __half *__restrict__ bank,
                                                     FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count) {
   using M = TileMap<D>;
-  __shared__ float s_a[D], s_b[D], s_c[D], s_beta[D], s_lin[D], s_prev[D];
-  __shared__ float s_lmax[M::RG][D];
+  __shared__ float s_a[D], s_b[D], s_c[D], s_beta[D], s_lin[D], s_thr[D];
   __shared__ int s_first[D];
   const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x, h = bh % H;
   const int tid = threadIdx.x;
@@ -149,7 +149,6 @@ __global__ void __launch_bounds__(128) bank_kernel(const __nv_bfloat16 *__restri
     s_beta[j] = b;
     s_lin[j] = ci.linear;
     s_c[j] = c;
-    s_prev[j] = kt > 0 ? cpre[o - D] : -INFINITY;
     if (ci.linear != 0.f) {
       s_a[j] = b > 0.f ? 1.f / b : 0.f;  // linear bank: 1/beta
       s_b[j] = 0.f;
@@ -157,104 +156,106 @@ __global__ void __launch_bounds__(128) bank_kernel(const __nv_bfloat16 *__restri
       s_a[j] = b * kLog2e;  // shifted bank: E = ex2(a v + b)
       s_b[j] = (kBankOffset - b * c) * kLog2e;
     }
-    s_first[j] = kBlockK;
+    // Diagonal hazard of a shifted channel: a row of this tile is safe once its
+    // visible maximum reaches c - kHazardTilt/beta, i.e. from the first key at
+    // or above that threshold on (row 0 when an earlier tile already reached it).
+    const float thr = c - kHazardTilt / b;
+    const bool haz = causal && ci.linear == 0.f;
+    s_thr[j] = haz ? thr : -INFINITY;
+    s_first[j] = (!haz || (kt > 0 && cpre[o - D] >= thr)) ? 0 : kBlockK;
   }
   __syncthreads();
 
+  // Thread: the 8 channels of chunk column cc, rows rg*RPG .. rg*RPG+RPG-1.
+  // Consecutive threads read consecutive 16-byte chunks of a row.  Both bank
+  // forms are evaluated and one is selected, so lanes never diverge.
   const __nv_bfloat16 *vb = v + static_cast<size_t>(bh) * T * D;
   __half *eb = bank + static_cast<size_t>(bh) * T * D;
-  float lmax[8];
-#pragma unroll
-  for (int u = 0; u < 8; ++u) lmax[u] = -INFINITY;
-#pragma unroll 2
-  for (int i = 0; i < M::RPG; ++i) {
-    const int key = kt * kBlockK + rg * M::RPG + i;
-    if (key >= T) break;
-    const uint4 raw = *reinterpret_cast<const uint4 *>(vb + static_cast<size_t>(key) * D + cc * 8);
-    const __nv_bfloat16 *vin = reinterpret_cast<const __nv_bfloat16 *>(&raw);
-    __align__(16) __half e[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int j = cc * 8 + u;
-      const float x = __bfloat162float(vin[u]);
-      lmax[u] = fmaxf(lmax[u], x);
-      float val;
-      if (s_lin[j] != 0.f) {
-        // D = expm1(y)/beta, y = beta (v - c) >= -1: Taylor series of expm1(y)/y
-        // for |y| < 1/2 (truncation < 4e-6 relative), e^y - 1 beyond
-        const float xs = x - s_c[j];
-        const float y = s_beta[j] * xs;
-        if (fabsf(y) < 0.5f) {
-          float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
-          poly = fmaf(y, poly, 1.f / 24.f);
-          poly = fmaf(y, poly, 1.f / 6.f);
-          poly = fmaf(y, poly, 0.5f);
-          poly = fmaf(y, poly, 1.f);
-          val = xs * poly;
-        } else {
-          val = (ex2_approx(y * kLog2e) - 1.f) * s_a[j];
-        }
-      } else {
-        val = ex2_approx(fmaf(s_a[j], x, s_b[j]));
-      }
-      e[u] = __float2half_rn(val);
-    }
-    *reinterpret_cast<uint4 *>(eb + static_cast<size_t>(key) * D + cc * 8) = *reinterpret_cast<const uint4 *>(e);
-  }
-  if (!causal) return;
-
-  // Diagonal-tile hazard: the first row of this tile at which the visible
-  // maximum of each shifted channel comes within kHazardTilt/beta of the
-  // tile's shift; rows before it are recomputed exactly.
-#pragma unroll
-  for (int u = 0; u < 8; ++u) s_lmax[rg][cc * 8 + u] = lmax[u];
-  __syncthreads();
+  float pa[8], pb[8], pc[8], pbeta[8], pthr[8];
+  bool plin[8];
+  int first[8];
 #pragma unroll
   for (int u = 0; u < 8; ++u) {
     const int j = cc * 8 + u;
-    if (s_lin[j] != 0.f) continue;
-    float run = s_prev[j];
-    for (int g = 0; g < rg; ++g) run = fmaxf(run, s_lmax[g][j]);
-    const float b = s_beta[j], c = s_c[j];
-    for (int i = 0; i < M::RPG; ++i) {
-      const int key = kt * kBlockK + rg * M::RPG + i;
+    pa[u] = s_a[j];
+    pb[u] = s_b[j];
+    pc[u] = s_c[j];
+    pbeta[u] = s_beta[j];
+    pthr[u] = s_thr[j];
+    plin[u] = s_lin[j] != 0.f;
+    first[u] = kBlockK;
+  }
+#pragma unroll 1
+  for (int i0 = 0; i0 < M::RPG; i0 += 4) {
+    uint4 raw[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int key = kt * kBlockK + rg * M::RPG + i0 + r;
+      raw[r] = key < T ? *reinterpret_cast<const uint4 *>(vb + static_cast<size_t>(key) * D + cc * 8)
+                       : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int row = rg * M::RPG + i0 + r;
+      const int key = kt * kBlockK + row;
       if (key >= T) break;
-      run = fmaxf(run, __bfloat162float(vb[static_cast<size_t>(key) * D + j]));
-      if (b * (c - run) <= kHazardTilt) {
-        atomicMin(&s_first[j], rg * M::RPG + i);
-        break;
+      const __nv_bfloat16 *vin = reinterpret_cast<const __nv_bfloat16 *>(&raw[r]);
+      __align__(16) __half e[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float x = __bfloat162float(vin[u]);
+        if (x >= pthr[u]) first[u] = min(first[u], row);
+        // linear bank: D = expm1(y)/beta, y = beta (v - c) >= -1, as a Taylor
+        // series of expm1(y)/y for |y| < 1/2 (truncation < 4e-6 relative),
+        // e^y - 1 beyond; shifted bank: E = 2^(a v + b)
+        const float xs = x - pc[u];
+        const float y = pbeta[u] * xs;
+        float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
+        poly = fmaf(y, poly, 1.f / 24.f);
+        poly = fmaf(y, poly, 1.f / 6.f);
+        poly = fmaf(y, poly, 0.5f);
+        poly = fmaf(y, poly, 1.f);
+        const float lin = fabsf(y) < 0.5f ? xs * poly : (ex2_approx(y * kLog2e) - 1.f) * pa[u];
+        const float shf = ex2_approx(fmaf(pa[u], x, pb[u]));
+        e[u] = __float2half_rn(plin[u] ? lin : shf);
       }
+      *reinterpret_cast<uint4 *>(eb + static_cast<size_t>(key) * D + cc * 8) = *reinterpret_cast<const uint4 *>(e);
     }
   }
+  if (causal) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (first[u] < kBlockK) atomicMin(&s_first[cc * 8 + u], first[u]);
+  }
+  if (!causal) return;
   __syncthreads();
-  const int warp = tid >> 5, lane = tid & 31;
-  if (warp < D / 32) {
-    const int g = warp;
-    int hz = s_first[g * 32 + lane];
-    if (hz == kBlockK) hz = 0;  // linear channel, or no valid key
-    int hz_max = hz;
-    for (int off = 16; off; off >>= 1) hz_max = max(hz_max, __shfl_xor_sync(0xffffffffu, hz_max, off));
-    const int t0 = kt * kBlockQ;
-    const int n_rows = min(hz_max, T - t0);
-    if (n_rows > 0) {
-      int base = 0;
-      if (lane == 0) base = atomicAdd(fixup_count, n_rows);
-      base = __shfl_sync(0xffffffffu, base, 0);
-      for (int r = lane; r < n_rows; r += 32) {
-        unsigned mask = 0;
-        for (int c = 0; c < 32; ++c) {
-          int hc = s_first[g * 32 + c];
-          if (hc == kBlockK) hc = 0;
-          mask |= (hc > r ? 1u : 0u) << c;
-        }
-        FixupEntry e;
-        e.row = bh * T + t0 + r;
-        e.group = g;
-        e.mask = mask;
-        e.pad = 0;
-        fixups[base + r] = e;
+  // rows r < max_j first_j of this tile get one entry with their channel masks
+  __shared__ int s_rows;
+  if (tid == 0) {
+    int hz_max = 0;
+    for (int j = 0; j < D; ++j) hz_max = max(hz_max, s_first[j]);
+    s_rows = min(hz_max, T - kt * kBlockQ);
+  }
+  __syncthreads();
+  const int n_rows = s_rows;
+  if (n_rows <= 0) return;
+  __shared__ int s_base;
+  if (tid == 0) s_base = atomicAdd(fixup_count, n_rows);
+  __syncthreads();
+  for (int r = tid; r < n_rows; r += 128) {
+    FixupEntry e;
+    e.row = bh * T + kt * kBlockQ + r;
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+      unsigned m = 0;
+      for (int c = 0; c < 32; ++c) {
+        const int j = 32 * g + c;
+        if (j < D && s_first[j] > r) m |= 1u << c;
       }
+      e.mask[g] = m;
     }
+    e.pad[0] = e.pad[1] = e.pad[2] = 0;
+    fixups[s_base + r] = e;
   }
 }
 
@@ -271,7 +272,11 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
     return cudaErrorInvalidValue;
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  plan_kernel<<<BH, d, 0, stream>>>(w.tstat, beta, H, T, d, n_kt, w.chan, w.cpre, w.shift, w.colmove);
+  if (d < 128) {  // channels beyond d have no mask bits
+    e = cudaMemsetAsync(w.colmask, 0, static_cast<size_t>(BH) * n_kt * 4 * sizeof(unsigned), stream);
+    if (e != cudaSuccess) return e;
+  }
+  plan_kernel<<<BH, d, 0, stream>>>(w.tstat, beta, H, T, d, n_kt, w.chan, w.cpre, w.shift, w.rfac, w.colmask);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (d == 64)
     bank_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,

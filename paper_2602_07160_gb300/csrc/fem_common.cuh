@@ -58,13 +58,12 @@ struct ChanInfo {
   float linear;  // 1.0f when the channel uses the linear bank, else 0.0f
 };
 
-// One exact-recompute entry: row = (b*H + h)*T + t, channels
-// 32*group + bit for every set bit of mask.
-struct FixupEntry {
+// One exact-recompute entry: row = (b*H + h)*T + t; channel 32*g + bit is
+// recomputed for every set bit of mask[g].
+struct __align__(32) FixupEntry {
   int row;
-  int group;
-  unsigned mask;
-  int pad;
+  unsigned mask[4];
+  int pad[3];
 };
 
 // ---------------------------------------------------------------------------
@@ -116,6 +115,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return done != 0;
 }
+
+// try_wait that lets the thread sleep (up to ~hint_ns) until the phase
+// completes instead of spinning.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return done != 0;
+}
+
+__device__ __forceinline__ void setmaxnreg_dec56() { asm volatile("setmaxnreg.dec.sync.aligned.u32 56;"); }
+__device__ __forceinline__ void setmaxnreg_inc224() { asm volatile("setmaxnreg.inc.sync.aligned.u32 224;"); }
 
 // Waits for the phase with the given parity to complete.  Gives up after
 // kWaitLimitNs, records `code` in the error word and returns false.
@@ -261,6 +277,16 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
       "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
       FEM_W8(0), FEM_W8(8), FEM_W8(16), FEM_W8(24)
       : "memory");
+}
+
+__device__ __forceinline__ uint32_t tmem_ld1(uint32_t taddr) {
+  uint32_t r;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr));
+  return r;
+}
+
+__device__ __forceinline__ void tmem_st1(uint32_t taddr, uint32_t r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(r) : "memory");
 }
 
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {

@@ -14,7 +14,8 @@ struct BankWorkspace {
   ChanInfo *chan;           // [B*H, d]
   float *cpre;              // [B*H, key tiles, d]: running maximum of v
   float *shift;             // [B*H, key tiles, d]: the bank's shift for each tile
-  int *colmove;             // [B*H, key tiles]: 1 when some shift moved at the tile
+  float *rfac;              // [B*H, key tiles, d]: exp(beta (shift[kt-1] - shift[kt])), 1 if unmoved
+  unsigned *colmask;        // [B*H, key tiles, 4]: bit j set when channel j's shift moved at the tile
   __half *bank;             // [B*H, T, d]: the value bank, fp16
   FixupEntry *fixups;       // exact-recompute list (causal)
   int *fixup_count;         // its length (zeroed before the pre-pass)
@@ -26,8 +27,8 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
 
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const float *beta,
-                      const ChanInfo *chan, const float *shift, const int *colmove, float *out, float *lse, int BH,
-                      int H, int T, int causal, unsigned *err, cudaStream_t stream);
+                      const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask, float *out,
+                      float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream);
 
 // Exact recompute of the listed (row, channel group) entries.
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, float *out, int H, int T,

@@ -47,9 +47,10 @@ struct TcLayout {
   static constexpr uint32_t kBar = 6 * kTile;  // 16 mbarriers
   static constexpr uint32_t kTmemSlot = kBar + 16 * 8;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
-  static constexpr uint32_t kChan = kBar + 256;
-  // beta, linear flag, anchor
-  static constexpr uint32_t kBytes = kChan + 3 * D * 4;
+  static constexpr uint32_t kChan = kBar + 256;  // beta, linear flag, anchor
+  static constexpr uint32_t kMoveBits = kChan + 3 * D * 4;  // 1 bit per key tile: a shift moved
+  static constexpr int kMaxKeyTiles = 8192;                  // T <= 1M keys
+  static constexpr uint32_t kBytes = kMoveBits + kMaxKeyTiles / 8;
   static constexpr uint32_t kAlloc = kBytes + 1024;
 };
 
@@ -71,8 +72,7 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, uns
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_timer_ns();
   while (true) {
-    for (int i = 0; i < 32; ++i)
-      if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity, 200000u)) return true;
     if (*abort_flag) return false;
     if (global_timer_ns() - t0 > kWaitLimitNs) {
       atomicOr(err, code);
@@ -92,8 +92,8 @@ __global__ void __launch_bounds__(384, 1)
     fem_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_e, const float *__restrict__ beta,
                   const ChanInfo *__restrict__ chan, const float *__restrict__ shift,
-                  const int *__restrict__ colmove, float *__restrict__ out, float *__restrict__ lse, int H, int T,
-                  int causal, unsigned *__restrict__ err) {
+                  const float *__restrict__ rfac, const unsigned *__restrict__ colmask, float *__restrict__ out,
+                  float *__restrict__ lse, int H, int T, int causal, unsigned *__restrict__ err) {
   using Lay = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -102,6 +102,7 @@ __global__ void __launch_bounds__(384, 1)
   float *c_beta = reinterpret_cast<float *>(smem + Lay::kChan);
   float *c_lin = c_beta + D;
   float *c_anchor = c_lin + D;
+  unsigned *move_bits = reinterpret_cast<unsigned *>(smem + Lay::kMoveBits);
   const uint32_t bars = sbase + Lay::kBar;
 #define FEM_BAR(i) (bars + 8u * static_cast<uint32_t>(i))
 
@@ -143,11 +144,23 @@ __global__ void __launch_bounds__(384, 1)
     c_lin[j] = ci.linear;
     c_anchor[j] = ci.c_lin;
   }
+  for (int w = tid; w < (n_kt_all + 31) / 32; w += 384) {
+    unsigned bits = 0;
+    for (int b = 0; b < 32 && 32 * w + b < n_kt_all; ++b) {
+      const uint4 m = reinterpret_cast<const uint4 *>(colmask)[static_cast<size_t>(bh) * n_kt_all + 32 * w + b];
+      bits |= ((m.x | m.y | m.z | m.w) != 0u ? 1u : 0u) << b;
+    }
+    move_bits[w] = bits;
+  }
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem + Lay::kTmemSlot);
 
+  if (warp < 4) {
+  // registers move from this warpgroup to the softmax warpgroups, which hold a
+  // 128-float score row per thread
+  setmaxnreg_dec56();
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
@@ -211,7 +224,12 @@ __global__ void __launch_bounds__(384, 1)
       }
       mma_commit(FEM_BAR(kBarAccDone + q));  // completes once everything this thread issued is done
     }
-  } else if (warp >= 4) {
+  } else if (warp == 3 && lane == 0) {
+    // make sure no MMA is still in flight before the allocation is released
+    for (int q = 0; q < n_tiles; ++q) wait_or_abort(FEM_BAR(kBarAccDone + q), 0, err, kErrWaitMma, abort_flag);
+  }
+  } else {
+    setmaxnreg_inc224();
     // ---------------------------------------------------------------- softmax + epilogue
     const int q = (warp - 4) >> 2;      // query tile of this warpgroup
     const int r = tid - 128 - 128 * q;  // row within the tile
@@ -224,69 +242,91 @@ __global__ void __launch_bounds__(384, 1)
       const uint32_t tAcc = tmem + 256 + q * D + lane_off;
       const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
       const float *shift_bh = shift + static_cast<size_t>(bh) * n_kt_all * D;
+      const float *rfac_bh = rfac + static_cast<size_t>(bh) * n_kt_all * D;
       float m_row = -INFINITY, L_row = 0.f;
       bool ok = true;
       for (int kt = 0; kt < nk; ++kt) {
-        const bool colmv = kt > 0 && colmove[bh * n_kt_all + kt] != 0;  // some channel's shift moved
+        const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
         // every lane takes the same branch: the wait's outcome is made warp-uniform
         ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSFull + q), kt & 1, err, kErrWaitMma, abort_flag));
         if (!ok) break;
         tc_fence_after_sync();
-        float s[128];
+        // the whole 128-column score row: four loads in flight, one wait
+        uint32_t sr[128];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          uint32_t v[32];
-          tmem_ld32(tS + c * 32, v);
-          tmem_ld_wait();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(v[i]) * qk_scale;
-        }
+        for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
+        tmem_ld_wait();
+        float *s = reinterpret_cast<float *>(sr);
         const int k0 = kt * kBlockK;
         if ((causal && kt == qt) || k0 + kBlockK > T) {
+          // keys k0 + n are visible for n < lim (key < T, and key <= row when causal)
+          const int lim = min(T, causal ? t_row + 1 : T) - k0;
 #pragma unroll
-          for (int n = 0; n < 128; ++n) {
-            const int key = k0 + n;
-            if (key >= T || (causal && key > t_row)) s[n] = -INFINITY;
-          }
+          for (int n = 0; n < 128; ++n) s[n] = n < lim ? s[n] : -INFINITY;
         }
-        float tmax = -INFINITY;
+        float mx[8];
 #pragma unroll
-        for (int n = 0; n < 128; ++n) tmax = fmaxf(tmax, s[n]);
+        for (int u = 0; u < 8; ++u) mx[u] = s[u];
+#pragma unroll
+        for (int n = 8; n < 128; ++n) mx[n & 7] = fmaxf(mx[n & 7], s[n]);
+        float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        tmax *= qk_scale;  // log2-domain row maximum of this tile
         float alpha = 1.f;
         if (tmax > m_row + kRowMaxLag) {
           alpha = ex2_approx(m_row - tmax);  // 0 on the first tile
           m_row = tmax;
         }
-        // P = exp2(s - m) as fp16 over the first 64 columns of S; L from the fp32 values
-        float lsum = 0.f;
+        // P = exp2(s * scale - m) as fp16 over the first 64 columns of S; L from the fp32 values
+        const float2 scale2 = make_float2(qk_scale, qk_scale), negm2 = make_float2(-m_row, -m_row);
+        float2 ls[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ls[u] = make_float2(0.f, 0.f);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           uint32_t p[16];
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
-            const float p0 = ex2_approx(s[c * 32 + 2 * i] - m_row);
-            const float p1 = ex2_approx(s[c * 32 + 2 * i + 1] - m_row);
-            lsum += p0 + p1;
-            p[i] = pack_half2(p0, p1);
+            const float2 x = __ffma2_rn(make_float2(s[c * 32 + 2 * i], s[c * 32 + 2 * i + 1]), scale2, negm2);
+            const float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+            ls[i & 3] = __fadd2_rn(ls[i & 3], e);
+            p[i] = pack_half2(e.x, e.y);
           }
           tmem_st16(tS + c * 16, p);
         }
-        // joint online rescale of acc (the previous P E has completed)
-        if (kt > 0 && (colmv || __any_sync(0xffffffffu, alpha != 1.f))) {
-          const float *c_now = shift_bh + kt * D, *c_old = c_now - D;
+        const float lsum = (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y) + (ls[2].x + ls[2].y) + (ls[3].x + ls[3].y);
+        // joint online rescale of acc (the previous P E has completed): every
+        // column when a row maximum moved, else only the moved channels
+        if (kt > 0) {
+          const float *rf = rfac_bh + kt * D;  // exp(beta_j (c_old - c_new)), 1 for unmoved channels
+          if (__any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t v[32];
-            tmem_ld32(tAcc + c * 32, v);
-            tmem_ld_wait();
+            for (int c = 0; c < D / 32; ++c) {
+              uint32_t v[32];
+              tmem_ld32(tAcc + c * 32, v);
+              tmem_ld_wait();
+              if (colmv) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int j = c * 32 + i;
-              float f = alpha;
-              if (colmv && c_lin[j] == 0.f) f *= expf(c_beta[j] * (c_old[j] - c_now[j]));
-              v[i] = __float_as_uint(__uint_as_float(v[i]) * f);
+                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha * rf[c * 32 + i]);
+              } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+              }
+              tmem_st32(tAcc + c * 32, v);
             }
-            tmem_st32(tAcc + c * 32, v);
+          } else if (colmv) {
+            const uint4 m4 = reinterpret_cast<const uint4 *>(colmask)[static_cast<size_t>(bh) * n_kt_all + kt];
+            const unsigned mw[4] = {m4.x, m4.y, m4.z, m4.w};
+#pragma unroll 1
+            for (int g = 0; g < D / 32; ++g) {
+              unsigned m = mw[g];
+              while (m) {
+                const int j = 32 * g + __ffs(m) - 1;
+                m &= m - 1;
+                const uint32_t x = tmem_ld1(tAcc + j);
+                tmem_ld_wait();
+                tmem_st1(tAcc + j, __float_as_uint(__uint_as_float(x) * rf[j]));
+              }
+            }
           }
         }
         L_row = L_row * alpha + lsum;
@@ -302,36 +342,33 @@ __global__ void __launch_bounds__(384, 1)
         const bool store = t_row < T;
         const size_t orow = static_cast<size_t>(bh) * T + t_row;
         const float invL = 1.f / L_row;
-#pragma unroll
+#pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           uint32_t v[32];
           tmem_ld32(tAcc + c * 32, v);
           tmem_ld_wait();
           if (store) {
-            __align__(16) float o[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int j = c * 32 + i;
-              const float a = __uint_as_float(v[i]) * invL;
-              const float b = c_beta[j];
-              float val;
-              if (c_lin[j] != 0.f)
-                val = b != 0.f ? c_anchor[j] + log1pf(b * a) / b : c_anchor[j] + a;
-              else
-                val = c_last[j] + (logf(a) - kBankOffset) / b;
-              o[i] = val;
-            }
             float4 *dst = reinterpret_cast<float4 *>(out + orow * D + c * 32);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) dst[i] = reinterpret_cast<const float4 *>(o)[i];
+            for (int i4 = 0; i4 < 8; ++i4) {
+              float o4[4];
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const int j = c * 32 + i4 * 4 + u;
+                const float a = __uint_as_float(v[i4 * 4 + u]) * invL;
+                const float b = c_beta[j];
+                if (c_lin[j] != 0.f)
+                  o4[u] = b != 0.f ? c_anchor[j] + log1pf(b * a) / b : c_anchor[j] + a;
+                else
+                  o4[u] = c_last[j] + (logf(a) - kBankOffset) / b;
+              }
+              dst[i4] = make_float4(o4[0], o4[1], o4[2], o4[3]);
+            }
           }
         }
         if (store && lse) lse[orow] = m_row * kLn2 + logf(L_row);
       }
     }
-  } else if (warp == 3 && lane == 0) {
-    // make sure no MMA is still in flight before the allocation is released
-    for (int q = 0; q < n_tiles; ++q) wait_or_abort(FEM_BAR(kBarAccDone + q), 0, err, kErrWaitMma, abort_flag);
   }
 
   tc_fence_before_sync();
@@ -345,23 +382,27 @@ __global__ void __launch_bounds__(384, 1)
 
 template <int D>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const float *beta,
-                               const ChanInfo *chan, const float *shift, const int *colmove, float *out, float *lse,
-                               int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream) {
+                               const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask,
+                               float *out, float *lse, int BH, int H, int T, int causal, unsigned *err,
+                               cudaStream_t stream) {
+  if ((T + kBlockK - 1) / kBlockK > TcLayout<D>::kMaxKeyTiles) return cudaErrorInvalidValue;
   const uint32_t smem = TcLayout<D>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   const dim3 grid((n_qt + 1) / 2, BH);
-  fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, beta, chan, shift, colmove, out, lse, H, T, causal, err);
+  fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, beta, chan, shift, rfac, colmask, out, lse, H, T, causal,
+                                                err);
   return cudaGetLastError();
 }
 
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const float *beta,
-                      const ChanInfo *chan, const float *shift, const int *colmove, float *out, float *lse, int BH,
-                      int H, int T, int causal, unsigned *err, cudaStream_t stream) {
-  if (d == 64) return launch_tc_d<64>(tq, tk, te, beta, chan, shift, colmove, out, lse, BH, H, T, causal, err, stream);
+                      const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask, float *out,
+                      float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream) {
+  if (d == 64)
+    return launch_tc_d<64>(tq, tk, te, beta, chan, shift, rfac, colmask, out, lse, BH, H, T, causal, err, stream);
   if (d == 128)
-    return launch_tc_d<128>(tq, tk, te, beta, chan, shift, colmove, out, lse, BH, H, T, causal, err, stream);
+    return launch_tc_d<128>(tq, tk, te, beta, chan, shift, rfac, colmask, out, lse, BH, H, T, causal, err, stream);
   return cudaErrorInvalidValue;
 }
 
