@@ -67,11 +67,13 @@ int device_state(DeviceState **out) {
 }
 
 // [d, T, B*H] 16-bit tensor, boxes of 64 channels x 128 rows, 128-byte swizzle.
+// [BH, T, d] row-major tensor; boxes of 128 rows x 128 bytes (64 16-bit or 32
+// 32-bit elements), 128-byte swizzle.
 int make_map(CUtensorMap *map, const void *base, int BH, int T, int d,
-             CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
+             CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, int elem_bytes = 2) {
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(BH)};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(T) * d * 2};
-  cuuint32_t box[3] = {64, 128, 1};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * elem_bytes, static_cast<cuuint64_t>(T) * d * elem_bytes};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(128 / elem_bytes), 128, 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = g_encode(map, dtype, 3, const_cast<void *>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -207,10 +209,11 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
 
-  CUtensorMap tq, tk, te;
+  CUtensorMap tq, tk, te, to;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&tk, k, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&te, bw.bank, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT16)) != FEM_OK) return rc;
+  if ((rc = make_map(&to, out, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4)) != FEM_OK) return rc;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, sizeof(int), s);
@@ -219,7 +222,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
   if (e == cudaSuccess)
-    e = launch_tc(d, tq, tk, te, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, out, lse, BH, H, T, causal, ds->err,
+    e = launch_tc(d, tq, tk, te, to, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, out, lse, BH, H, T, causal, ds->err,
                   s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess) {

@@ -26,7 +26,9 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
                               const BankWorkspace &w, cudaStream_t stream);
 
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
-cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const float *beta,
+// `to` maps the fp32 output [B*H, T, d] for the kernel's TMA stores.
+cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const CUtensorMap &to,
+                      const float *beta,
                       const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask, float *out,
                       float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream);
 
