@@ -5,7 +5,8 @@
 //   1. tile_stats, plan, bank: channel modes, shift schedule, the fp16 value
 //      bank (once per key tile), the fix-up list
 //   2. fem_tc (tcgen05): the read for every row and channel
-//   3. fixup (causal only): exact fp32 recompute of the listed entries
+//   3. fixup (causal only): the listed entries completed exactly over their
+//      diagonal tile, merged with the state fem_tc left for the earlier tiles
 #include <cudaTypedefs.h>
 
 #include <mutex>
@@ -86,7 +87,7 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-  size_t tstat, chan, cpre, shift, rfac, colmask, bank, fixups, count, total;
+  size_t tstat, chan, cpre, shift, rfac, colmask, bank, fixups, tilefix, count, total;
 };
 
 bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
@@ -110,6 +111,8 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += round256(BH * n_kt * 4 * sizeof(unsigned));
   w->fixups = off;
   off += causal ? round256(BH * n_kt * kBlockQ * sizeof(FixupEntry)) : 0;
+  w->tilefix = off;
+  off += causal ? round256(BH * n_kt * sizeof(int2)) : 0;
   w->count = off;
   off += 256;
   w->total = off;
@@ -208,6 +211,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   bw.bank = reinterpret_cast<__half *>(ws + w.bank);
   bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
+  bw.tilefix = causal ? reinterpret_cast<int2 *>(ws + w.tilefix) : nullptr;
 
   CUtensorMap tq, tk, te, to;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
@@ -222,12 +226,13 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
   if (e == cudaSuccess)
-    e = launch_tc(d, tq, tk, te, to, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, out, lse, BH, H, T, causal, ds->err,
-                  s);
+    e = launch_tc(d, tq, tk, te, to, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, bw.tilefix, bw.fixups, lse, BH, H, T,
+                  causal, ds->err, s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess) {
     if (causal)
-      e = launch_fixup(q, k, v, beta, out, H, T, d, bw.fixups, bw.fixup_count, ds->last_fixup, ds->num_sms, s);
+      e = launch_fixup(q, k, v, beta, bw.shift, out, H, T, d, bw.fixups, bw.fixup_count, ds->last_fixup, ds->num_sms,
+                       s);
     else
       e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
   }

@@ -134,7 +134,8 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
                                                     const float *__restrict__ beta, const ChanInfo *__restrict__ chan,
                                                     const float *__restrict__ cpre, const float *__restrict__ shift,
                                                     int H, int T, int causal, __half *__restrict__ bank,
-                                                    FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count) {
+                                                    FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count,
+                                                    int2 *__restrict__ tilefix) {
   using M = TileMap<D>;
   __shared__ float s_a[D], s_b[D], s_c[D], s_beta[D], s_lin[D], s_thr[D];
   __shared__ int s_first[D];
@@ -238,9 +239,16 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
   }
   __syncthreads();
   const int n_rows = s_rows;
-  if (n_rows <= 0) return;
+  int2 *tf = tilefix + static_cast<size_t>(bh) * n_kt + kt;
+  if (n_rows <= 0) {
+    if (tid == 0) *tf = make_int2(0, 0);
+    return;
+  }
   __shared__ int s_base;
-  if (tid == 0) s_base = atomicAdd(fixup_count, n_rows);
+  if (tid == 0) {
+    s_base = atomicAdd(fixup_count, n_rows);
+    *tf = make_int2(s_base, n_rows);
+  }
   __syncthreads();
   for (int r = tid; r < n_rows; r += 128) {
     FixupEntry e;
@@ -254,7 +262,9 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
       }
       e.mask[g] = m;
     }
-    e.pad[0] = e.pad[1] = e.pad[2] = 0;
+    e.m_pre = -INFINITY;
+    e.l_pre = 0.f;
+    e.pad = 0;
     fixups[s_base + r] = e;
   }
 }
@@ -280,10 +290,10 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (d == 64)
     bank_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
-                                              w.fixup_count);
+                                              w.fixup_count, w.tilefix);
   else
     bank_kernel<128><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
-                                               w.fixup_count);
+                                               w.fixup_count, w.tilefix);
   return cudaGetLastError();
 }
 

@@ -58,12 +58,15 @@ struct ChanInfo {
   float linear;  // 1.0f when the channel uses the linear bank, else 0.0f
 };
 
-// One exact-recompute entry: row = (b*H + h)*T + t; channel 32*g + bit is
-// recomputed for every set bit of mask[g].
+// One fix-up entry: row = (b*H + h)*T + t of a causal diagonal tile; channel
+// 32*g + bit is completed for every set bit of mask[g].  The tensor-core
+// kernel fills m_pre and l_pre: the row's running maximum (log2 units) and
+// sum of 2^(s - m_pre) over the key tiles before the diagonal one.
 struct __align__(32) FixupEntry {
   int row;
   unsigned mask[4];
-  int pad[3];
+  float m_pre, l_pre;
+  int pad;
 };
 
 // ---------------------------------------------------------------------------

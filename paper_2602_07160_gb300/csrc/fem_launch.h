@@ -19,6 +19,8 @@ struct BankWorkspace {
   __half *bank;             // [B*H, T, d]: the value bank, fp16
   FixupEntry *fixups;       // exact-recompute list (causal)
   int *fixup_count;         // its length (zeroed before the pre-pass)
+  int2 *tilefix;            // [B*H, key tiles] (causal): {first entry, number of rows} of the tile's
+                            // entries, which list the tile's rows 0 .. number-1 in order
 };
 
 // Statistics, plan and value bank (two reads of V, one write of the bank).
@@ -26,16 +28,21 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
                               const BankWorkspace &w, cudaStream_t stream);
 
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
-// `to` maps the fp32 output [B*H, T, d] for the kernel's TMA stores.
+// `to` maps the fp32 output [B*H, T, d] for the kernel's TMA stores.  For the
+// rows of a causal diagonal tile that have fix-up entries the kernel writes,
+// in place of the listed channels' outputs, their accumulator before the
+// diagonal tile, and the row's (max, sum) before it into the entry.
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const CUtensorMap &to,
-                      const float *beta,
-                      const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask, float *out,
-                      float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream);
+                      const float *beta, const ChanInfo *chan, const float *shift, const float *rfac,
+                      const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H,
+                      int T, int causal, unsigned *err, cudaStream_t stream);
 
-// Exact recompute of the listed (row, channel group) entries.
-cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, float *out, int H, int T,
-                         int d, const FixupEntry *entries, const int *count, int *last_count, int num_sms,
-                         cudaStream_t stream);
+// Completes the listed (row, channel) outputs: the diagonal tile's keys
+// exactly, merged with the state the tensor-core kernel left for the earlier
+// key tiles.
+cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
+                         float *out, int H, int T, int d, const FixupEntry *entries, const int *count, int *last_count,
+                         int num_sms, cudaStream_t stream);
 
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,

@@ -106,7 +106,8 @@ __global__ void __launch_bounds__(256, 1)
                   const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_o,
                   const float *__restrict__ beta,
                   const ChanInfo *__restrict__ chan, const float *__restrict__ shift,
-                  const float *__restrict__ rfac, const unsigned *__restrict__ colmask, float *__restrict__ lse, int H,
+                  const float *__restrict__ rfac, const unsigned *__restrict__ colmask,
+                  const int2 *__restrict__ tilefix, FixupEntry *__restrict__ fixups, float *__restrict__ lse, int H,
                   int T, int causal, unsigned *__restrict__ err) {
   using Lay = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -265,10 +266,24 @@ __global__ void __launch_bounds__(256, 1)
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;
     const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
+    // Rows 0 .. hz_rows-1 of a causal diagonal tile may have fix-up entries
+    // (entry hz_base + r): for them the accumulator before the diagonal tile is
+    // kept in a free score buffer (the stash) and written out in place of the
+    // listed channels' outputs, and (m, L) before it go into the entry.
+    int hz_base = 0, hz_rows = 0;
+    if (causal) {
+      const int2 tf = tilefix[static_cast<size_t>(bh) * n_kt_all + qt];
+      hz_base = tf.x;
+      hz_rows = tf.y;
+    }
+    const bool hz_warp = hz_rows > 32 * (warp & 3);  // warp-uniform
+    const bool hz_row = r < hz_rows;
+    const uint32_t tStash = tmem + ((qt + 1) % 3) * 128 + lane_off;
     float m_row = -INFINITY, L_row = 0.f;
     bool ok = true;
     for (int kt = 0; kt < nk; ++kt) {
       const int b = kt % 3;
+      const float m_old = m_row;
       const uint32_t tS = tmem + b * 128 + lane_off;
       const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
       // every lane takes the same branch: the wait's outcome is made warp-uniform
@@ -322,6 +337,27 @@ __global__ void __launch_bounds__(256, 1)
         tmem_st16(tS + c * 16, p);
       }
       const float lsum = (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y) + (ls[2].x + ls[2].y) + (ls[3].x + ls[3].y);
+      if (hz_warp && kt == nk - 1) {
+        // diagonal tile: keep the state before it for the fix-up
+        if (kt > 0) {
+          const int pb = (kt - 1) % 3;
+          ok = __all_sync(0xffffffffu,
+                          wait_or_abort(FEM_BAR(kBarPvDone + pb), ((kt - 1) / 3) & 1, err, kErrWaitMma, abort_flag));
+          if (!ok) break;
+          tc_fence_after_sync();
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t v[32];
+            tmem_ld32(tAcc + c * 32, v);
+            tmem_ld_wait();
+            tmem_st32(tStash + c * 32, v);
+          }
+        }
+        if (hz_row) {
+          fixups[hz_base + r].m_pre = m_old;
+          fixups[hz_base + r].l_pre = L_row;
+        }
+      }
       // joint online rescale of acc, once the previous P E has completed
       if (kt > 0) {
         const bool rowmv = __any_sync(0xffffffffu, alpha != 1.f);
@@ -412,6 +448,19 @@ __global__ void __launch_bounds__(256, 1)
           }
           *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(o4[0], o4[1], o4[2], o4[3]);
         }
+        if (hz_warp) {
+          // listed channels of fix-up rows: the accumulator before the diagonal tile
+          uint32_t w[32];
+          if (qt > 0) {
+            tmem_ld32(tStash + c * 32, w);
+            tmem_ld_wait();
+          }
+          const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if ((mc >> i) & 1u)
+              reinterpret_cast<float *>(box + sw128_offset(r, i >> 2))[i & 3] = qt > 0 ? __uint_as_float(w[i]) : 0.f;
+        }
         // the box is complete once all 128 rows are in: one thread stores it
         fence_proxy_async_smem();
         bar_sync(1, 128);
@@ -438,27 +487,29 @@ template <int D>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
                                const CUtensorMap &to, const float *beta,
                                const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask,
-                               float *out, float *lse, int BH, int H, int T, int causal, unsigned *err,
-                               cudaStream_t stream) {
+                               const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H, int T, int causal,
+                               unsigned *err, cudaStream_t stream) {
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   if (n_qt > TcLayout<D>::kMaxKeyTiles || n_qt > 65535) return cudaErrorInvalidValue;
   const uint32_t smem = TcLayout<D>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const dim3 grid(BH, n_qt);
-  fem_tc_kernel<D><<<grid, 256, smem, stream>>>(tq, tk, te, to, beta, chan, shift, rfac, colmask, lse, H, T, causal,
+  fem_tc_kernel<D><<<grid, 256, smem, stream>>>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
                                                 err);
   return cudaGetLastError();
 }
 
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const CUtensorMap &to,
-                      const float *beta,
-                      const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask, float *out,
-                      float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream) {
+                      const float *beta, const ChanInfo *chan, const float *shift, const float *rfac,
+                      const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H,
+                      int T, int causal, unsigned *err, cudaStream_t stream) {
   if (d == 64)
-    return launch_tc_d<64>(tq, tk, te, to, beta, chan, shift, rfac, colmask, out, lse, BH, H, T, causal, err, stream);
+    return launch_tc_d<64>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
+                           err, stream);
   if (d == 128)
-    return launch_tc_d<128>(tq, tk, te, to, beta, chan, shift, rfac, colmask, out, lse, BH, H, T, causal, err, stream);
+    return launch_tc_d<128>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
+                            err, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -182,6 +182,32 @@ def _sample_rows(w, n_random, seed=0):
     return np.unique(np.concatenate([first, last, rand]))
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_fixup_rows_of_late_diagonal_tiles(d):
+    """Spikes in small-valued beta=20 channels move the bank shift in the middle
+    of diagonal tiles 0, 20 and the ragged last one, so the rows before each
+    spike underflow on the bank and are completed by the fix-up from the state
+    the tensor-core kernel leaves before the diagonal tile (none for tile 0)."""
+    B, H, T = 1, 2, 3000  # 23 full key tiles and a 56-row tail
+    q, k, v, beta = W.make_custom(B, H, T, d, seed=7)
+    beta[:, :8] = 20.0
+    vf = v.float()
+    vf[..., :8] *= 0.1
+    spikes = [5, 20 * 128 + 64, 23 * 128 + 40]
+    for p in spikes:
+        vf[:, :, p, :8] = 3.0
+    v = vf.to(torch.bfloat16).contiguous()
+    out, lse = _gpu_bf16(q, k, v, beta, True)
+    n_fix = fem.last_fixup_rows()
+    assert n_fix >= 2 * (5 + 64 + 40), n_fix  # at least the rows before each spike, both heads
+    tiles = [0, 20, 23]
+    rows = np.concatenate([bh * T + np.arange(t * 128, min(T, t * 128 + 128)) for bh in range(B * H) for t in tiles])
+    ref, ref_lse = oracle.fem_read_rows(q, k, v, beta, True, rows)
+    got = out.reshape(-1, d)[rows]
+    _assert_close(got, ref, what=f"fix-up rows d={d}")
+    assert np.abs(lse.reshape(-1)[rows] - ref_lse).max() <= LSE_MAX
+
+
 @pytest.mark.parametrize("name,n_random", [("lm_causal_d64", 3000), ("lm_causal_d128", 1500),
                                            ("long_causal_student_t", 600)])
 def test_workload_full_size_sampled(name, n_random):
