@@ -152,8 +152,9 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
   return done != 0;
 }
 
+// Per-warpgroup register budget (every thread of the warpgroup executes it).
 __device__ __forceinline__ void setmaxnreg_dec56() { asm volatile("setmaxnreg.dec.sync.aligned.u32 56;"); }
-__device__ __forceinline__ void setmaxnreg_inc224() { asm volatile("setmaxnreg.inc.sync.aligned.u32 224;"); }
+__device__ __forceinline__ void setmaxnreg_inc256() { asm volatile("setmaxnreg.inc.sync.aligned.u32 256;"); }
 
 // Waits for the phase with the given parity to complete.  Gives up after
 // kWaitLimitNs, records `code` in the error word and returns false.

@@ -6,23 +6,28 @@
 // contraction of later key tiles and the value contraction of the previous
 // one run on the tensor pipe while the softmax works on the current tile:
 //
-//   warp 0      TMA producer of Q and of the K tiles (three-stage ring)
-//   warp 1      S issuer: S_k = Q K_k^T (both operands in shared memory) into
-//               score buffer k mod 3, up to two key tiles ahead of the
-//               softmax; it waits only for the P E that last read the buffer
-//   warp 2      PV issuer: acc += P_k E_k with P_k read from TMEM, as soon as
-//               the softmax has written P_k.  The two issuers are different
-//               warps, so their instruction streams overlap on the tensor pipe
-//   warp 3      TMEM allocation; TMA producer of the E tiles (two-stage ring)
-//   warps 4-7   softmax (thread = row): P = exp(s - m) with a lazily raised
-//               row maximum m, rounded to fp16 over the first 64 columns of the
-//               tile's score buffer, and the row sum L; the joint online rescale
-//               of acc by exp(m_old - m_new) * exp(beta_j (c_old - c_new)) after
-//               the previous P E completed, over every column when a row
-//               maximum moved, over the moved channels when only channel shifts
-//               moved; then the epilogue o = c + log1p(beta acc/L)/beta (linear
-//               bank) or o = c + (log(acc/L) - kappa)/beta (shifted bank),
-//               lse = m + log L.
+//   warp 0       TMA producer of Q and of the K tiles (three-stage ring)
+//   warp 1       S issuer: S_k = Q K_k^T (both operands in shared memory) into
+//                score buffer k mod 3, up to two key tiles ahead of the
+//                softmax; it waits only for the P E that last read the buffer
+//   warp 2       PV issuer: acc += P_k E_k with P_k read from TMEM, once the
+//                softmax has written P_k and the correction has rescaled acc.
+//                The two issuers are different warps, so their instruction
+//                streams overlap on the tensor pipe
+//   warp 3       TMEM allocation; TMA producer of the E tiles (two-stage ring)
+//   warps 4-7    softmax (thread = row): the tile's row maximum and the factor
+//                alpha = exp(m_old - m_new) of a lazily raised running maximum
+//                m (handed to the correction at once), then P = exp(s - m)
+//                rounded to fp16 over the first 64 columns of the tile's score
+//                buffer, and the row sum L
+//   warps 8-11   correction (thread = row): once the previous P E completed,
+//                the joint online rescale of acc by alpha * exp(beta_j (c_old -
+//                c_new)), over every column when a row maximum moved, over the
+//                moved channels when only channel shifts moved.  Off the
+//                softmax's path, it overlaps the next tile's exponentials
+//   warps 4-11   epilogue, half the columns each:
+//                o = c + log1p(beta acc/L)/beta (linear bank) or
+//                o = c + (log(acc/L) - kappa)/beta (shifted bank); lse = m + log L.
 //
 // sum_i exp(s_i - m) E_ij is the free energy's numerator up to the
 // stabilising shifts and L its normaliser (Sec. 2.3, Eq.
@@ -50,7 +55,7 @@ struct TcLayout {
   static constexpr uint32_t kK = kTile;                    // K[0..2]
   static constexpr uint32_t kE = kK + kStagesK * kTile;    // E[0..1]
   static constexpr uint32_t kBar = kE + kStagesE * kTile;  // mbarriers
-  static constexpr int kNumBars = 24;
+  static constexpr int kNumBars = 27;
   static constexpr uint32_t kTmemSlot = kBar + kNumBars * 8;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kChan = kBar + 256;               // per-channel epilogue coefficients
@@ -60,7 +65,9 @@ struct TcLayout {
   // and its moved-channel mask [4], loaded with the E tile
   static constexpr uint32_t kSide = kMoveBits + kMaxKeyTiles / 8;
   static constexpr uint32_t kSideStride = D * 4 + 128;
-  static constexpr uint32_t kBytes = kSide + kStagesE * kSideStride;
+  static constexpr uint32_t kAlpha = kSide + kStagesE * kSideStride;  // alpha per row, per score buffer
+  static constexpr uint32_t kInvL = kAlpha + kBufS * 128 * 4;         // 1/L per row, for the epilogue
+  static constexpr uint32_t kBytes = kInvL + 128 * 4;
   static constexpr uint32_t kAlloc = kBytes + 1024;
   static constexpr uint32_t kAccCol = 384;
 };
@@ -73,10 +80,11 @@ enum : int {
   kBarEFull = 7,     // + E stage (2)
   kBarEEmpty = 9,    // + E stage (2)
   kBarSFull = 11,    // + score buffer (3): S_k complete
-  kBarPFull = 14,    // + score buffer (3): P_k written and acc rescaled (128 arrivals)
+  kBarPFull = 14,    // + score buffer (3): P_k written and acc rescaled (256 arrivals)
   kBarPvDone = 17,   // + score buffer (3): P_k E_k complete
   kBarAccDone = 20,  // every P E complete
-  kBarSDone = 21     // every score contraction the S issuer started is complete
+  kBarSDone = 21,    // every score contraction the S issuer started is complete
+  kBarAlpha = 22     // + score buffer (3): the softmax's alpha of tile k is in shared memory (128 arrivals)
 };
 
 // Bounded wait that also gives up as soon as another role has given up.
@@ -101,7 +109,7 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
 }
 
 template <int D>
-__global__ void __launch_bounds__(256, 1)
+__global__ void __launch_bounds__(384, 1)
     fem_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_o,
                   const float *__restrict__ beta,
@@ -122,6 +130,7 @@ __global__ void __launch_bounds__(256, 1)
 #define FEM_BAR(i) (bars + 8u * static_cast<uint32_t>(i))
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int wg = __shfl_sync(0xffffffffu, tid >> 7, 0);  // warpgroup, provably warp-uniform
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   const int n_kt_all = (T + kBlockK - 1) / kBlockK;
   // grid = (B*H, query tiles): the heaviest causal tiles are scheduled first
@@ -139,7 +148,8 @@ __global__ void __launch_bounds__(256, 1)
       mbar_init(FEM_BAR(kBarKFull + s), 1);
       mbar_init(FEM_BAR(kBarKEmpty + s), 1);
       mbar_init(FEM_BAR(kBarSFull + s), 1);
-      mbar_init(FEM_BAR(kBarPFull + s), 128);
+      mbar_init(FEM_BAR(kBarPFull + s), 256);
+      mbar_init(FEM_BAR(kBarAlpha + s), 128);
       mbar_init(FEM_BAR(kBarPvDone + s), 1);
     }
     for (int s = 0; s < 2; ++s) {
@@ -151,7 +161,7 @@ __global__ void __launch_bounds__(256, 1)
     fence_mbar_init();
     *abort_flag = 0;
   }
-  for (int j = tid; j < D; j += 256) {
+  for (int j = tid; j < D; j += 384) {
     const ChanInfo ci = chan[bh * D + j];
     const float bj = beta[h * D + j];
     const bool lin = ci.linear != 0.f;
@@ -160,7 +170,7 @@ __global__ void __launch_bounds__(256, 1)
                             lin ? 0.f : 1.f);
   }
   // one bit per key tile: set when some channel's shift moved there
-  for (int base = 0; base < nk; base += 256) {
+  for (int base = 0; base < nk; base += 384) {
     const int t = base + tid;
     bool moved = false;
     if (t < nk) {
@@ -175,6 +185,10 @@ __global__ void __launch_bounds__(256, 1)
   tc_fence_after_sync();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem + Lay::kTmemSlot);
 
+  if (wg == 0) {
+  // registers move from this warpgroup to the softmax, which holds a
+  // 128-float score row per thread
+  setmaxnreg_dec56();
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA: Q and K
     if (lane == 0) {
@@ -259,13 +273,17 @@ __global__ void __launch_bounds__(256, 1)
       }
       mma_commit(FEM_BAR(kBarAccDone));  // completes once everything this thread issued is done
     }
-  } else {
-    // ---------------------------------------------------------------- softmax + epilogue
-    const int r = tid - 128;  // row within the tile
+  }
+  } else if (wg == 1) {
+    // ---------------------------------------------------------------- softmax, then epilogue
+    setmaxnreg_inc256();
+    const bool is_sm = true;
+    const int r = (tid - 128) & 127;  // row within the tile
     const int t_row = qt * kBlockQ + r;
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;
-    const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
+    float *s_alpha = reinterpret_cast<float *>(smem + Lay::kAlpha);
+    float *s_invL = reinterpret_cast<float *>(smem + Lay::kInvL);
     // Rows 0 .. hz_rows-1 of a causal diagonal tile may have fix-up entries
     // (entry hz_base + r): for them the accumulator before the diagonal tile is
     // kept in a free score buffer (the stash) and written out in place of the
@@ -281,148 +299,90 @@ __global__ void __launch_bounds__(256, 1)
     const uint32_t tStash = tmem + ((qt + 1) % 3) * 128 + lane_off;
     float m_row = -INFINITY, L_row = 0.f;
     bool ok = true;
-    for (int kt = 0; kt < nk; ++kt) {
-      const int b = kt % 3;
-      const float m_old = m_row;
-      const uint32_t tS = tmem + b * 128 + lane_off;
-      const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
-      // every lane takes the same branch: the wait's outcome is made warp-uniform
-      ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSFull + b), (kt / 3) & 1, err, kErrWaitMma, abort_flag));
-      if (!ok) break;
-      tc_fence_after_sync();
-      // the whole 128-column score row: four loads in flight, one wait
-      uint32_t sr[128];
+    {
+      // ------------------------------------------------------------ softmax
+      const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
+      for (int kt = 0; kt < nk; ++kt) {
+        const int b = kt % 3;
+        const uint32_t tS = tmem + b * 128 + lane_off;
+        // every lane takes the same branch: the wait's outcome is made warp-uniform
+        ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSFull + b), (kt / 3) & 1, err, kErrWaitMma, abort_flag));
+        if (!ok) break;
+        tc_fence_after_sync();
+        // the whole 128-column score row: four loads in flight, one wait
+        uint32_t sr[128];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
-      tmem_ld_wait();
-      float *s = reinterpret_cast<float *>(sr);
-      const int k0 = kt * kBlockK;
-      if ((causal && kt == qt) || k0 + kBlockK > T) {
-        // keys k0 + n are visible for n < lim (key < T, and key <= row when causal)
-        const int lim = min(T, causal ? t_row + 1 : T) - k0;
+        for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
+        tmem_ld_wait();
+        float *s = reinterpret_cast<float *>(sr);
+        const int k0 = kt * kBlockK;
+        if ((causal && kt == qt) || k0 + kBlockK > T) {
+          // keys k0 + n are visible for n < lim (key < T, and key <= row when causal)
+          const int lim = min(T, causal ? t_row + 1 : T) - k0;
 #pragma unroll
-        for (int n = 0; n < 128; ++n) s[n] = n < lim ? s[n] : -INFINITY;
-      }
-      float mx[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) mx[u] = fmax3(s[u], s[u + 8], s[u + 16]);
-#pragma unroll
-      for (int n = 24; n < 120; n += 16)
-#pragma unroll
-        for (int u = 0; u < 8; ++u) mx[u] = fmax3(mx[u], s[n + u], s[n + 8 + u]);
-#pragma unroll
-      for (int u = 0; u < 8; ++u) mx[u] = fmaxf(mx[u], s[120 + u]);
-      float tmax = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
-      tmax *= qk_scale;  // log2-domain row maximum of this tile
-      float alpha = 1.f;
-      if (tmax > m_row + kRowMaxLag) {
-        alpha = ex2_approx(m_row - tmax);  // 0 on the first tile
-        m_row = tmax;
-      }
-      // P = exp2(s * scale - m) as fp16 over the first 64 columns of the buffer; L from the fp32 values
-      const float2 scale2 = make_float2(qk_scale, qk_scale), negm2 = make_float2(-m_row, -m_row);
-      float2 ls[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) ls[u] = make_float2(0.f, 0.f);
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t p[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float2 x = __ffma2_rn(make_float2(s[c * 32 + 2 * i], s[c * 32 + 2 * i + 1]), scale2, negm2);
-          const float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
-          ls[i & 3] = __fadd2_rn(ls[i & 3], e);
-          p[i] = pack_half2(e.x, e.y);
+          for (int n = 0; n < 128; ++n) s[n] = n < lim ? s[n] : -INFINITY;
         }
-        tmem_st16(tS + c * 16, p);
-      }
-      const float lsum = (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y) + (ls[2].x + ls[2].y) + (ls[3].x + ls[3].y);
-      if (hz_warp && kt == nk - 1) {
-        // diagonal tile: keep the state before it for the fix-up
-        if (kt > 0) {
-          const int pb = (kt - 1) % 3;
-          ok = __all_sync(0xffffffffu,
-                          wait_or_abort(FEM_BAR(kBarPvDone + pb), ((kt - 1) / 3) & 1, err, kErrWaitMma, abort_flag));
-          if (!ok) break;
-          tc_fence_after_sync();
-#pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t v[32];
-            tmem_ld32(tAcc + c * 32, v);
-            tmem_ld_wait();
-            tmem_st32(tStash + c * 32, v);
-          }
+        float mx[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mx[u] = fmax3(s[u], s[u + 8], s[u + 16]);
+#pragma unroll
+        for (int n = 24; n < 120; n += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mx[u] = fmax3(mx[u], s[n + u], s[n + 8 + u]);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mx[u] = fmaxf(mx[u], s[120 + u]);
+        float tmax = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
+        tmax *= qk_scale;  // log2-domain row maximum of this tile
+        float alpha = 1.f;
+        const float m_old = m_row;
+        if (tmax > m_row + kRowMaxLag) {
+          alpha = ex2_approx(m_row - tmax);  // 0 on the first tile
+          m_row = tmax;
         }
-        if (hz_row) {
+        s_alpha[b * 128 + r] = alpha;
+        mbar_arrive(FEM_BAR(kBarAlpha + b));
+        if (hz_row && kt == nk - 1) {
+          // diagonal tile: the row's state before it, for the fix-up
           fixups[hz_base + r].m_pre = m_old;
           fixups[hz_base + r].l_pre = L_row;
         }
-      }
-      // joint online rescale of acc, once the previous P E has completed
-      if (kt > 0) {
-        const bool rowmv = __any_sync(0xffffffffu, alpha != 1.f);
-        if (rowmv || colmv) {
-          const int pb = (kt - 1) % 3;
-          ok = __all_sync(0xffffffffu,
-                          wait_or_abort(FEM_BAR(kBarPvDone + pb), ((kt - 1) / 3) & 1, err, kErrWaitMma, abort_flag));
-          if (!ok) break;
-          tc_fence_after_sync();
-          // this tile's rescale factors arrive with its E tile
-          const float *rf = reinterpret_cast<const float *>(smem + Lay::kSide + (kt & 1) * Lay::kSideStride);
-          if (colmv) {
-            ok = __all_sync(0xffffffffu,
-                            wait_or_abort(FEM_BAR(kBarEFull + (kt & 1)), (kt >> 1) & 1, err, kErrWaitTma, abort_flag));
-            if (!ok) break;
+        // P = exp2(s * scale - m) as fp16 over the first 64 columns of the buffer; L from the fp32 values
+        const float2 scale2 = make_float2(qk_scale, qk_scale), negm2 = make_float2(-m_row, -m_row);
+        float2 ls[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ls[u] = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t p[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float2 x = __ffma2_rn(make_float2(s[c * 32 + 2 * i], s[c * 32 + 2 * i + 1]), scale2, negm2);
+            const float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+            ls[i & 3] = __fadd2_rn(ls[i & 3], e);
+            p[i] = pack_half2(e.x, e.y);
           }
-          if (rowmv) {
-#pragma unroll 1
-            for (int c = 0; c < D / 32; ++c) {
-              uint32_t v[32];
-              tmem_ld32(tAcc + c * 32, v);
-              tmem_ld_wait();
-              if (colmv) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha * rf[c * 32 + i]);
-              } else {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-              }
-              tmem_st32(tAcc + c * 32, v);
-            }
-          } else {
-            // 32-column groups holding a moved channel (rf = 1 elsewhere)
-            const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + D);
-            const unsigned gm = (m4.x ? 1u : 0u) | (m4.y ? 2u : 0u) | (m4.z ? 4u : 0u) | (m4.w ? 8u : 0u);
-#pragma unroll 1
-            for (int c = 0; c < D / 32; ++c) {
-              if (!((gm >> c) & 1u)) continue;
-              uint32_t v[32];
-              tmem_ld32(tAcc + c * 32, v);
-              float f[32];
-#pragma unroll
-              for (int i = 0; i < 32; ++i) f[i] = rf[c * 32 + i];
-              tmem_ld_wait();
-#pragma unroll
-              for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * f[i]);
-              tmem_st32(tAcc + c * 32, v);
-            }
-          }
+          tmem_st16(tS + c * 16, p);
         }
+        const float lsum = (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y) + (ls[2].x + ls[2].y) + (ls[3].x + ls[3].y);
+        L_row = L_row * alpha + lsum;
+        tmem_st_wait();
+        tc_fence_before_sync();
+        mbar_arrive(FEM_BAR(kBarPFull + b));
       }
-      L_row = L_row * alpha + lsum;
-      tmem_st_wait();
-      tc_fence_before_sync();
-      mbar_arrive(FEM_BAR(kBarPFull + b));
+      s_invL[r] = 1.f / L_row;
+      if (ok && lse && t_row < T) lse[static_cast<size_t>(bh) * T + t_row] = (m_row + lg2_approx(L_row)) * kLn2;
     }
-    // ---- epilogue: o staged in shared memory (the K ring is idle once every
-    // contraction completed) in the output map's swizzled boxes, then TMA stores
+    // ---- epilogue, half the columns per warpgroup: o staged in shared memory
+    // (the K ring is idle once every contraction completed) in the output
+    // map's swizzled boxes, then TMA stores
     if (ok) ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAccDone), 0, err, kErrWaitMma, abort_flag));
-    ok = bar_and(1, 128, ok);  // every softmax warp read all its key tiles
+    ok = bar_and(1, 256, ok);  // both warpgroups went through every key tile
     if (ok) {
       tc_fence_after_sync();
-      const float invL = 1.f / L_row;
+      const float invL = s_invL[r];
+      const int c_lo = is_sm ? 0 : D / 64;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; ++c) {
+      for (int c = c_lo; c < c_lo + D / 64; ++c) {
         uint32_t v[32];
         tmem_ld32(tAcc + c * 32, v);
         tmem_ld_wait();
@@ -463,13 +423,162 @@ __global__ void __launch_bounds__(256, 1)
         }
         // the box is complete once all 128 rows are in: one thread stores it
         fence_proxy_async_smem();
-        bar_sync(1, 128);
+        bar_sync(is_sm ? 2 : 3, 128);
         if (r == 0) {
           tma_store_3d(&tmap_o, sbase + Lay::kK + c * 16384, c * 32, qt * kBlockQ, bh);
           bulk_commit_group();
         }
       }
-      if (lse && t_row < T) lse[static_cast<size_t>(bh) * T + t_row] = (m_row + lg2_approx(L_row)) * kLn2;
+      if (r == 0) bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
+    }
+  } else {
+    // ---------------------------------------------------------------- correction, then epilogue
+    const bool is_sm = false;
+    const int r = (tid - 128) & 127;  // row within the tile
+    const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;
+    const float *s_alpha = reinterpret_cast<const float *>(smem + Lay::kAlpha);
+    const float *s_invL = reinterpret_cast<float *>(smem + Lay::kInvL);
+    // fix-up rows of the diagonal tile, as in the softmax warpgroup
+    int hz_base = 0, hz_rows = 0;
+    if (causal) {
+      const int2 tf = tilefix[static_cast<size_t>(bh) * n_kt_all + qt];
+      hz_base = tf.x;
+      hz_rows = tf.y;
+    }
+    const bool hz_warp = hz_rows > 32 * (warp & 3);  // warp-uniform
+    const bool hz_row = r < hz_rows;
+    const uint32_t tStash = tmem + ((qt + 1) % 3) * 128 + lane_off;
+    bool ok = true;
+    {
+      // ------------------------------------------------------------ correction
+      for (int kt = 0; kt < nk; ++kt) {
+        const int b = kt % 3;
+        ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAlpha + b), (kt / 3) & 1, err, kErrWaitMma, abort_flag));
+        if (!ok) break;
+        const float alpha = s_alpha[b * 128 + r];
+        const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
+        const bool rowmv = __any_sync(0xffffffffu, alpha != 1.f);
+        const bool stash = hz_warp && kt == nk - 1;  // diagonal tile of rows with fix-up entries
+        if (kt > 0 && (rowmv || colmv || stash)) {
+          // acc is final for tile kt-1 once its P E completed
+          const int pb = (kt - 1) % 3;
+          ok = __all_sync(0xffffffffu,
+                          wait_or_abort(FEM_BAR(kBarPvDone + pb), ((kt - 1) / 3) & 1, err, kErrWaitMma, abort_flag));
+          if (!ok) break;
+          tc_fence_after_sync();
+          if (stash) {
+#pragma unroll 1
+            for (int c = 0; c < D / 32; ++c) {
+              uint32_t v[32];
+              tmem_ld32(tAcc + c * 32, v);
+              tmem_ld_wait();
+              tmem_st32(tStash + c * 32, v);
+            }
+          }
+          // this tile's rescale factors exp(beta_j (c_old - c_new)) arrive with its E tile
+          const float *rf = reinterpret_cast<const float *>(smem + Lay::kSide + (kt & 1) * Lay::kSideStride);
+          if (colmv) {
+            ok = __all_sync(0xffffffffu,
+                            wait_or_abort(FEM_BAR(kBarEFull + (kt & 1)), (kt >> 1) & 1, err, kErrWaitTma, abort_flag));
+            if (!ok) break;
+          }
+          if (rowmv) {
+#pragma unroll 1
+            for (int c = 0; c < D / 32; ++c) {
+              uint32_t v[32];
+              tmem_ld32(tAcc + c * 32, v);
+              tmem_ld_wait();
+              if (colmv) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha * rf[c * 32 + i]);
+              } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+              }
+              tmem_st32(tAcc + c * 32, v);
+            }
+          } else if (colmv) {
+            // 32-column groups holding a moved channel (rf = 1 elsewhere)
+            const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + D);
+            const unsigned gm = (m4.x ? 1u : 0u) | (m4.y ? 2u : 0u) | (m4.z ? 4u : 0u) | (m4.w ? 8u : 0u);
+#pragma unroll 1
+            for (int c = 0; c < D / 32; ++c) {
+              if (!((gm >> c) & 1u)) continue;
+              uint32_t v[32];
+              tmem_ld32(tAcc + c * 32, v);
+              float f[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) f[i] = rf[c * 32 + i];
+              tmem_ld_wait();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * f[i]);
+              tmem_st32(tAcc + c * 32, v);
+            }
+          }
+          tmem_st_wait();
+        }
+        tc_fence_before_sync();
+        mbar_arrive(FEM_BAR(kBarPFull + b));
+      }
+    }
+    // ---- epilogue, half the columns per warpgroup: o staged in shared memory
+    // (the K ring is idle once every contraction completed) in the output
+    // map's swizzled boxes, then TMA stores
+    if (ok) ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAccDone), 0, err, kErrWaitMma, abort_flag));
+    ok = bar_and(1, 256, ok);  // both warpgroups went through every key tile
+    if (ok) {
+      tc_fence_after_sync();
+      const float invL = s_invL[r];
+      const int c_lo = is_sm ? 0 : D / 64;
+#pragma unroll 1
+      for (int c = c_lo; c < c_lo + D / 64; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tAcc + c * 32, v);
+        tmem_ld_wait();
+        uint8_t *box = smem + Lay::kK + c * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
+#pragma unroll
+        for (int i4 = 0; i4 < 8; ++i4) {
+          float o4[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float4 cf = c_coef[c * 32 + i4 * 4 + u];
+            const float a = __uint_as_float(v[i4 * 4 + u]) * invL;
+            // shifted bank: (log a - kappa) / beta.  Linear bank: log1p(x)/beta with
+            // x = beta a, as a times the series of log1p(x)/x for |x| < 2^-6 (also
+            // beta = 0), else log(1 + x) plus the rounding error of 1 + x over 1 + x
+            const float x = cf.x * a;
+            const float u1 = 1.f + x;
+            const float l = lg2_approx(cf.w != 0.f ? a : u1) * kLn2;
+            const float o_sh = (l - kBankOffset) * cf.y;
+            const float o_lg = fmaf((x - (u1 - 1.f)), rcp_approx(u1), l) * cf.y;
+            const float o_se = a * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f);
+            const float o = cf.w != 0.f ? o_sh : (fabsf(x) < 0.015625f ? o_se : o_lg);
+            o4[u] = cf.z + o;
+          }
+          *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(o4[0], o4[1], o4[2], o4[3]);
+        }
+        if (hz_warp) {
+          // listed channels of fix-up rows: the accumulator before the diagonal tile
+          uint32_t w[32];
+          if (qt > 0) {
+            tmem_ld32(tStash + c * 32, w);
+            tmem_ld_wait();
+          }
+          const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if ((mc >> i) & 1u)
+              reinterpret_cast<float *>(box + sw128_offset(r, i >> 2))[i & 3] = qt > 0 ? __uint_as_float(w[i]) : 0.f;
+        }
+        // the box is complete once all 128 rows are in: one thread stores it
+        fence_proxy_async_smem();
+        bar_sync(is_sm ? 2 : 3, 128);
+        if (r == 0) {
+          tma_store_3d(&tmap_o, sbase + Lay::kK + c * 16384, c * 32, qt * kBlockQ, bh);
+          bulk_commit_group();
+        }
+      }
       if (r == 0) bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
     }
   }
@@ -494,8 +603,15 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
   const uint32_t smem = TcLayout<D>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
+  // The producer warpgroup gives registers down to 56 and the softmax takes
+  // them up to 256 from the block's launch allocation (384 threads x numRegs);
+  // the correction keeps numRegs.  An increase the allocation cannot cover
+  // would wait forever, so the split is checked before any launch.
+  cudaFuncAttributes fa;
+  if ((e = cudaFuncGetAttributes(&fa, fem_tc_kernel<D>)) != cudaSuccess) return e;
+  if (128 * (56 + 256 + fa.numRegs) > 384 * fa.numRegs) return cudaErrorInvalidConfiguration;
   const dim3 grid(BH, n_qt);
-  fem_tc_kernel<D><<<grid, 256, smem, stream>>>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
+  fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
                                                 err);
   return cudaGetLastError();
 }
