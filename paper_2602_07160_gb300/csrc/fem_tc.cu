@@ -55,17 +55,18 @@ struct TcLayout {
   static constexpr uint32_t kK = kTile;                    // K[0..2]
   static constexpr uint32_t kE = kK + kStagesK * kTile;    // E[0..1]
   static constexpr uint32_t kBar = kE + kStagesE * kTile;  // mbarriers
-  static constexpr int kNumBars = 27;
+  static constexpr int kNumBars = 35;
   static constexpr uint32_t kTmemSlot = kBar + kNumBars * 8;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
-  static constexpr uint32_t kChan = kBar + 256;               // per-channel epilogue coefficients
+  static constexpr uint32_t kChan = kBar + 512;               // per-channel epilogue coefficients
   static constexpr uint32_t kMoveBits = kChan + 4 * D * 4;   // 1 bit per key tile: a shift moved
   static constexpr int kMaxKeyTiles = 8192;                  // T <= 1M keys
-  // per E stage: the tile's rescale factors exp(beta_j (c_old - c_new)) [D]
-  // and its moved-channel mask [4], loaded with the E tile
+  // side ring: per key tile its rescale factors exp(beta_j (c_old - c_new)) [D]
+  // and moved-channel mask [4], loaded with the K tile, kSideStages tiles deep
+  static constexpr int kSideStages = 8;
   static constexpr uint32_t kSide = kMoveBits + kMaxKeyTiles / 8;
   static constexpr uint32_t kSideStride = D * 4 + 128;
-  static constexpr uint32_t kAlpha = kSide + kStagesE * kSideStride;  // alpha per row, per score buffer
+  static constexpr uint32_t kAlpha = kSide + kSideStages * kSideStride;  // alpha per row, per score buffer
   static constexpr uint32_t kInvL = kAlpha + kBufS * 128 * 4;         // 1/L per row, for the epilogue
   static constexpr uint32_t kBytes = kInvL + 128 * 4;
   static constexpr uint32_t kAlloc = kBytes + 1024;
@@ -84,7 +85,8 @@ enum : int {
   kBarPvDone = 17,   // + score buffer (3): P_k E_k complete
   kBarAccDone = 20,  // every P E complete
   kBarSDone = 21,    // every score contraction the S issuer started is complete
-  kBarAlpha = 22     // + score buffer (3): the softmax's alpha of tile k is in shared memory (128 arrivals)
+  kBarAlpha = 22,    // + score buffer (3): the softmax's alpha of tile k is in shared memory (128 arrivals)
+  kBarSide = 25      // + side slot (8): tile k's rescale factors and moved-channel mask are in shared memory
 };
 
 // Bounded wait that also gives up as soon as another role has given up.
@@ -156,6 +158,7 @@ __global__ void __launch_bounds__(384, 1)
       mbar_init(FEM_BAR(kBarEFull + s), 1);
       mbar_init(FEM_BAR(kBarEEmpty + s), 1);
     }
+    for (int s = 0; s < Lay::kSideStages; ++s) mbar_init(FEM_BAR(kBarSide + s), 1);
     mbar_init(FEM_BAR(kBarAccDone), 1);
     mbar_init(FEM_BAR(kBarSDone), 1);
     fence_mbar_init();
@@ -205,6 +208,13 @@ __global__ void __launch_bounds__(384, 1)
         for (int b = 0; b < D / 64; ++b)
           tma_load_3d(sbase + Lay::kK + st * Lay::kTile + b * 16384, &tmap_k, FEM_BAR(kBarKFull + st), b * 64,
                       kt * kBlockK, bh);
+        // Side slot kt % 8 was last read by the correction of tile kt - 8, which
+        // finished before PV(kt - 6), hence before S(kt - 3) released this K stage.
+        const int ss = kt % Lay::kSideStages;
+        const size_t row = static_cast<size_t>(bh) * n_kt_all + kt;
+        mbar_arrive_expect_tx(FEM_BAR(kBarSide + ss), D * 4 + 16);
+        bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride, rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
+        bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride + D * 4, colmask + row * 4, 16, FEM_BAR(kBarSide + ss));
       }
     }
   } else if (warp == 3) {
@@ -215,13 +225,10 @@ __global__ void __launch_bounds__(384, 1)
         const int st = kt & 1;
         const uint32_t use = static_cast<uint32_t>(kt >> 1);
         if (use > 0 && !wait_or_abort(FEM_BAR(kBarEEmpty + st), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
-        const size_t row = static_cast<size_t>(bh) * n_kt_all + kt;
-        mbar_arrive_expect_tx(FEM_BAR(kBarEFull + st), Lay::kTile + D * 4 + 16);
+        mbar_arrive_expect_tx(FEM_BAR(kBarEFull + st), Lay::kTile);
         for (int b = 0; b < D / 64; ++b)
           tma_load_3d(sbase + Lay::kE + st * Lay::kTile + b * 16384, &tmap_e, FEM_BAR(kBarEFull + st), b * 64,
                       kt * kBlockK, bh);
-        bulk_load(sbase + Lay::kSide + st * Lay::kSideStride, rfac + row * D, D * 4, FEM_BAR(kBarEFull + st));
-        bulk_load(sbase + Lay::kSide + st * Lay::kSideStride + D * 4, colmask + row * 4, 16, FEM_BAR(kBarEFull + st));
       }
       // no contraction may be in flight when the TMEM allocation is released:
       // both issuers commit these barriers on every exit path
@@ -461,6 +468,23 @@ __global__ void __launch_bounds__(384, 1)
         const bool rowmv = __any_sync(0xffffffffu, alpha != 1.f);
         const bool stash = hz_warp && kt == nk - 1;  // diagonal tile of rows with fix-up entries
         if (kt > 0 && (rowmv || colmv || stash)) {
+          // this tile's rescale factors exp(beta_j (c_old - c_new)), 1 for unmoved
+          // channels, and its moved-channel mask, loaded tiles ahead with K
+          const float *rf =
+              reinterpret_cast<const float *>(smem + Lay::kSide + (kt % Lay::kSideStages) * Lay::kSideStride);
+          unsigned gm = 0;  // 32-column groups holding a moved channel
+          int g0 = 0;
+          float f0[32];  // factors of the first such group, read before acc is ready
+          if (colmv) {
+            ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSide + kt % Lay::kSideStages),
+                                                       (kt / Lay::kSideStages) & 1, err, kErrWaitTma, abort_flag));
+            if (!ok) break;
+            const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + D);
+            gm = (m4.x ? 1u : 0u) | (m4.y ? 2u : 0u) | (m4.z ? 4u : 0u) | (m4.w ? 8u : 0u);
+            g0 = __ffs(gm) - 1;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) f0[i] = rf[g0 * 32 + i];
+          }
           // acc is final for tile kt-1 once its P E completed
           const int pb = (kt - 1) % 3;
           ok = __all_sync(0xffffffffu,
@@ -475,13 +499,6 @@ __global__ void __launch_bounds__(384, 1)
               tmem_ld_wait();
               tmem_st32(tStash + c * 32, v);
             }
-          }
-          // this tile's rescale factors exp(beta_j (c_old - c_new)) arrive with its E tile
-          const float *rf = reinterpret_cast<const float *>(smem + Lay::kSide + (kt & 1) * Lay::kSideStride);
-          if (colmv) {
-            ok = __all_sync(0xffffffffu,
-                            wait_or_abort(FEM_BAR(kBarEFull + (kt & 1)), (kt >> 1) & 1, err, kErrWaitTma, abort_flag));
-            if (!ok) break;
           }
           if (rowmv) {
 #pragma unroll 1
@@ -499,11 +516,16 @@ __global__ void __launch_bounds__(384, 1)
               tmem_st32(tAcc + c * 32, v);
             }
           } else if (colmv) {
-            // 32-column groups holding a moved channel (rf = 1 elsewhere)
-            const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + D);
-            const unsigned gm = (m4.x ? 1u : 0u) | (m4.y ? 2u : 0u) | (m4.z ? 4u : 0u) | (m4.w ? 8u : 0u);
+            {
+              uint32_t v[32];
+              tmem_ld32(tAcc + g0 * 32, v);
+              tmem_ld_wait();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * f0[i]);
+              tmem_st32(tAcc + g0 * 32, v);
+            }
 #pragma unroll 1
-            for (int c = 0; c < D / 32; ++c) {
+            for (int c = g0 + 1; c < D / 32; ++c) {
               if (!((gm >> c) & 1u)) continue;
               uint32_t v[32];
               tmem_ld32(tAcc + c * 32, v);
