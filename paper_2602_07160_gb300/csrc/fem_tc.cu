@@ -135,9 +135,10 @@ __global__ void __launch_bounds__(384, 1)
   const int wg = __shfl_sync(0xffffffffu, tid >> 7, 0);  // warpgroup, provably warp-uniform
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   const int n_kt_all = (T + kBlockK - 1) / kBlockK;
-  // grid = (B*H, query tiles): the heaviest causal tiles are scheduled first
-  const int bh = blockIdx.x, h = bh % H;
-  const int qt = causal ? n_qt - 1 - static_cast<int>(blockIdx.y) : static_cast<int>(blockIdx.y);
+  // grid = (query tiles, B*H): CTAs in flight share a few heads' K and E in L2,
+  // and within a head the heaviest causal tiles start first
+  const int bh = blockIdx.y, h = bh % H;
+  const int qt = causal ? n_qt - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x);
   const int nk = causal ? qt + 1 : n_kt_all;  // key tiles this query tile reads
 
   if (warp == 3) {
@@ -621,7 +622,7 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
                                const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H, int T, int causal,
                                unsigned *err, cudaStream_t stream) {
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
-  if (n_qt > TcLayout<D>::kMaxKeyTiles || n_qt > 65535) return cudaErrorInvalidValue;
+  if (n_qt > TcLayout<D>::kMaxKeyTiles || BH > 65535) return cudaErrorInvalidValue;
   const uint32_t smem = TcLayout<D>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
@@ -632,7 +633,7 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
   cudaFuncAttributes fa;
   if ((e = cudaFuncGetAttributes(&fa, fem_tc_kernel<D>)) != cudaSuccess) return e;
   if (128 * (56 + 256 + fa.numRegs) > 384 * fa.numRegs) return cudaErrorInvalidConfiguration;
-  const dim3 grid(BH, n_qt);
+  const dim3 grid(n_qt, BH);
   fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
                                                 err);
   return cudaGetLastError();
