@@ -48,7 +48,7 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
     sm[u] = 0.f;
   }
   const __nv_bfloat16 *vb = v + static_cast<size_t>(bh) * T * D;
-#pragma unroll 4
+#pragma unroll
   for (int i = 0; i < M::RPG; ++i) {
     const int key = kt * kBlockK + rg * M::RPG + i;
     if (key < T) {
@@ -90,12 +90,20 @@ __global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__res
   const int bh = blockIdx.x, j = threadIdx.x, h = bh % H;
   const float b = beta[h * d + j];
   const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * d + j;
+  // the tiles' statistics are read kBatch at a time, all loads in flight
+  constexpr int kBatch = 8;
   float gmax = -INFINITY, gmin = INFINITY, gsum = 0.f;
-  for (int kt = 0; kt < n_kt; ++kt) {
-    const float4 s = ts[static_cast<size_t>(kt) * d];
-    gmax = fmaxf(gmax, s.x);
-    gmin = fminf(gmin, s.y);
-    gsum += s.z;
+  for (int k0 = 0; k0 < n_kt; k0 += kBatch) {
+    float4 st[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u)
+      st[u] = k0 + u < n_kt ? ts[static_cast<size_t>(k0 + u) * d] : make_float4(-INFINITY, INFINITY, 0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      gmax = fmaxf(gmax, st[u].x);
+      gmin = fminf(gmin, st[u].y);
+      gsum += st[u].z;
+    }
   }
   const float mean = gsum / static_cast<float>(T);
   ChanInfo ci;
@@ -111,8 +119,15 @@ __global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__res
   chan[bh * d + j] = ci;
   const bool lin = ci.linear != 0.f;
   float cp = -INFINITY, cl = -INFINITY;
-  for (int kt = 0; kt < n_kt; ++kt) {
-    cp = fmaxf(cp, ts[static_cast<size_t>(kt) * d].x);
+  for (int k0 = 0; k0 < n_kt; k0 += kBatch) {
+    float tmx[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) tmx[u] = k0 + u < n_kt ? ts[static_cast<size_t>(k0 + u) * d].x : -INFINITY;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+    const int kt = k0 + u;
+    if (kt >= n_kt) break;  // uniform over the block
+    cp = fmaxf(cp, tmx[u]);
     const float prev = cl;
     if (lin) {
       cl = ci.c_lin;
@@ -126,6 +141,7 @@ __global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__res
     rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
     const unsigned bits = __ballot_sync(0xffffffffu, moved);
     if ((j & 31) == 0) colmask[(static_cast<size_t>(bh) * n_kt + kt) * 4 + (j >> 5)] = bits;
+    }
   }
 }
 

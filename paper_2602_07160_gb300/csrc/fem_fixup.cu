@@ -166,7 +166,7 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
                          int num_sms, cudaStream_t stream) {
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
-  const int grid = num_sms * 8;
+  const int grid = num_sms * 16;
   if (d == 64)
     fixup_kernel<64><<<grid, kFixThreads, 0, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, last_count);
   else if (d == 128)

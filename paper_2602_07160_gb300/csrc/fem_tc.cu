@@ -124,8 +124,9 @@ __global__ void __launch_bounds__(384, 1)
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + Lay::kAbort);
-  // per channel {beta, 1/beta (0 at beta = 0), the epilogue's offset c (the
-  // linear bank's anchor or the shifted bank's last shift), 1 if shifted}
+  // per channel, for the epilogue: shifted bank {ln2/beta, c - kappa/beta, 0, 1}
+  // with c the last shift, so o = lg2(a) * x + y; linear bank {beta, c, 1/beta
+  // (0 at beta = 0), 0} with c the anchor
   float4 *c_coef = reinterpret_cast<float4 *>(smem + Lay::kChan);
   unsigned *move_bits = reinterpret_cast<unsigned *>(smem + Lay::kMoveBits);
   const uint32_t bars = sbase + Lay::kBar;
@@ -140,6 +141,30 @@ __global__ void __launch_bounds__(384, 1)
   const int bh = blockIdx.y, h = bh % H;
   const int qt = causal ? n_qt - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x);
   const int nk = causal ? qt + 1 : n_kt_all;  // key tiles this query tile reads
+
+  // K tile kt into K stage kt % 3, with its side data into side slot kt % 8.
+  // Side slot kt % 8 was last read by the correction of tile kt - 8, which
+  // finished before PV(kt - 6), hence before S(kt - 3) released this K stage.
+  auto load_k = [&](int kt) {
+    const int st = kt % 3, ss = kt % Lay::kSideStages;
+    mbar_arrive_expect_tx(FEM_BAR(kBarKFull + st), Lay::kTile);
+    for (int b = 0; b < D / 64; ++b)
+      tma_load_3d(sbase + Lay::kK + st * Lay::kTile + b * 16384, &tmap_k, FEM_BAR(kBarKFull + st), b * 64,
+                  kt * kBlockK, bh);
+    const size_t row = static_cast<size_t>(bh) * n_kt_all + kt;
+    mbar_arrive_expect_tx(FEM_BAR(kBarSide + ss), D * 4 + 16);
+    bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride, rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
+    bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride + D * 4, colmask + row * 4, 16, FEM_BAR(kBarSide + ss));
+  };
+  // E tile kt into E stage kt % 2
+  auto load_e = [&](int kt) {
+    const int st = kt & 1;
+    mbar_arrive_expect_tx(FEM_BAR(kBarEFull + st), Lay::kTile);
+    for (int b = 0; b < D / 64; ++b)
+      tma_load_3d(sbase + Lay::kE + st * Lay::kTile + b * 16384, &tmap_e, FEM_BAR(kBarEFull + st), b * 64,
+                  kt * kBlockK, bh);
+  };
+  constexpr int kPreK = 3, kPreE = 2;  // loads the prologue issues (the rings' depths)
 
   if (warp == 3) {
     tmem_alloc(sbase + Lay::kTmemSlot, 512);
@@ -164,14 +189,24 @@ __global__ void __launch_bounds__(384, 1)
     mbar_init(FEM_BAR(kBarSDone), 1);
     fence_mbar_init();
     *abort_flag = 0;
+    // the first loads leave before the rest of the prologue: Q, the first
+    // kPreK K tiles with their side data, the first kPreE E tiles
+    mbar_arrive_expect_tx(FEM_BAR(kBarQ), Lay::kTile);
+    for (int b = 0; b < D / 64; ++b)
+      tma_load_3d(sbase + Lay::kQ + b * 16384, &tmap_q, FEM_BAR(kBarQ), b * 64, qt * kBlockQ, bh);
+    for (int kt = 0; kt < min(nk, kPreK); ++kt) load_k(kt);
+    for (int kt = 0; kt < min(nk, kPreE); ++kt) load_e(kt);
   }
   for (int j = tid; j < D; j += 384) {
     const ChanInfo ci = chan[bh * D + j];
     const float bj = beta[h * D + j];
     const bool lin = ci.linear != 0.f;
-    c_coef[j] = make_float4(bj, bj != 0.f ? 1.f / bj : 0.f,
-                            lin ? ci.c_lin : shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j],
-                            lin ? 0.f : 1.f);
+    if (lin) {
+      c_coef[j] = make_float4(bj, ci.c_lin, bj != 0.f ? 1.f / bj : 0.f, 0.f);
+    } else {
+      const float c = shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j];
+      c_coef[j] = make_float4(kLn2 / bj, c - kBankOffset / bj, 0.f, 1.f);
+    }
   }
   // one bit per key tile: set when some channel's shift moved there
   for (int base = 0; base < nk; base += 384) {
@@ -196,40 +231,19 @@ __global__ void __launch_bounds__(384, 1)
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA: Q and K
     if (lane == 0) {
-      prefetch_tensormap(&tmap_q);
-      prefetch_tensormap(&tmap_k);
-      mbar_arrive_expect_tx(FEM_BAR(kBarQ), Lay::kTile);
-      for (int b = 0; b < D / 64; ++b)
-        tma_load_3d(sbase + Lay::kQ + b * 16384, &tmap_q, FEM_BAR(kBarQ), b * 64, qt * kBlockQ, bh);
-      for (int kt = 0; kt < nk; ++kt) {
-        const int st = kt % 3;
+      for (int kt = kPreK; kt < nk; ++kt) {
         const uint32_t use = static_cast<uint32_t>(kt / 3);
-        if (use > 0 && !wait_or_abort(FEM_BAR(kBarKEmpty + st), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
-        mbar_arrive_expect_tx(FEM_BAR(kBarKFull + st), Lay::kTile);
-        for (int b = 0; b < D / 64; ++b)
-          tma_load_3d(sbase + Lay::kK + st * Lay::kTile + b * 16384, &tmap_k, FEM_BAR(kBarKFull + st), b * 64,
-                      kt * kBlockK, bh);
-        // Side slot kt % 8 was last read by the correction of tile kt - 8, which
-        // finished before PV(kt - 6), hence before S(kt - 3) released this K stage.
-        const int ss = kt % Lay::kSideStages;
-        const size_t row = static_cast<size_t>(bh) * n_kt_all + kt;
-        mbar_arrive_expect_tx(FEM_BAR(kBarSide + ss), D * 4 + 16);
-        bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride, rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
-        bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride + D * 4, colmask + row * 4, 16, FEM_BAR(kBarSide + ss));
+        if (!wait_or_abort(FEM_BAR(kBarKEmpty + kt % 3), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
+        load_k(kt);
       }
     }
   } else if (warp == 3) {
     // ---------------------------------------------------------------- TMA: E
     if (lane == 0) {
-      prefetch_tensormap(&tmap_e);
-      for (int kt = 0; kt < nk; ++kt) {
-        const int st = kt & 1;
+      for (int kt = kPreE; kt < nk; ++kt) {
         const uint32_t use = static_cast<uint32_t>(kt >> 1);
-        if (use > 0 && !wait_or_abort(FEM_BAR(kBarEEmpty + st), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
-        mbar_arrive_expect_tx(FEM_BAR(kBarEFull + st), Lay::kTile);
-        for (int b = 0; b < D / 64; ++b)
-          tma_load_3d(sbase + Lay::kE + st * Lay::kTile + b * 16384, &tmap_e, FEM_BAR(kBarEFull + st), b * 64,
-                      kt * kBlockK, bh);
+        if (!wait_or_abort(FEM_BAR(kBarEEmpty + (kt & 1)), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
+        load_e(kt);
       }
       // no contraction may be in flight when the TMEM allocation is released:
       // both issuers commit these barriers on every exit path
@@ -282,10 +296,10 @@ __global__ void __launch_bounds__(384, 1)
       mma_commit(FEM_BAR(kBarAccDone));  // completes once everything this thread issued is done
     }
   }
-  } else if (wg == 1) {
-    // ---------------------------------------------------------------- softmax, then epilogue
-    setmaxnreg_inc256();
-    const bool is_sm = true;
+  } else {
+    // ---------------------------------------------------------------- softmax (warpgroup 1) or
+    // correction (warpgroup 2), then the epilogue, which both run as one code path
+    const bool is_sm = wg == 1;
     const int r = (tid - 128) & 127;  // row within the tile
     const int t_row = qt * kBlockQ + r;
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
@@ -307,7 +321,8 @@ __global__ void __launch_bounds__(384, 1)
     const uint32_t tStash = tmem + ((qt + 1) % 3) * 128 + lane_off;
     float m_row = -INFINITY, L_row = 0.f;
     bool ok = true;
-    {
+    if (is_sm) {
+      setmaxnreg_inc256();
       // ------------------------------------------------------------ softmax
       const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
       for (int kt = 0; kt < nk; ++kt) {
@@ -380,85 +395,7 @@ __global__ void __launch_bounds__(384, 1)
       s_invL[r] = 1.f / L_row;
       if (ok && lse && t_row < T) lse[static_cast<size_t>(bh) * T + t_row] = (m_row + lg2_approx(L_row)) * kLn2;
     }
-    // ---- epilogue, half the columns per warpgroup: o staged in shared memory
-    // (the K ring is idle once every contraction completed) in the output
-    // map's swizzled boxes, then TMA stores
-    if (ok) ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAccDone), 0, err, kErrWaitMma, abort_flag));
-    ok = bar_and(1, 256, ok);  // both warpgroups went through every key tile
-    if (ok) {
-      tc_fence_after_sync();
-      const float invL = s_invL[r];
-      const int c_lo = is_sm ? 0 : D / 64;
-#pragma unroll 1
-      for (int c = c_lo; c < c_lo + D / 64; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tAcc + c * 32, v);
-        tmem_ld_wait();
-        uint8_t *box = smem + Lay::kK + c * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
-#pragma unroll
-        for (int i4 = 0; i4 < 8; ++i4) {
-          float o4[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float4 cf = c_coef[c * 32 + i4 * 4 + u];
-            const float a = __uint_as_float(v[i4 * 4 + u]) * invL;
-            // shifted bank: (log a - kappa) / beta.  Linear bank: log1p(x)/beta with
-            // x = beta a, as a times the series of log1p(x)/x for |x| < 2^-6 (also
-            // beta = 0), else log(1 + x) plus the rounding error of 1 + x over 1 + x
-            const float x = cf.x * a;
-            const float u1 = 1.f + x;
-            const float l = lg2_approx(cf.w != 0.f ? a : u1) * kLn2;
-            const float o_sh = (l - kBankOffset) * cf.y;
-            const float o_lg = fmaf((x - (u1 - 1.f)), rcp_approx(u1), l) * cf.y;
-            const float o_se = a * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f);
-            const float o = cf.w != 0.f ? o_sh : (fabsf(x) < 0.015625f ? o_se : o_lg);
-            o4[u] = cf.z + o;
-          }
-          *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(o4[0], o4[1], o4[2], o4[3]);
-        }
-        if (hz_warp) {
-          // listed channels of fix-up rows: the accumulator before the diagonal tile
-          uint32_t w[32];
-          if (qt > 0) {
-            tmem_ld32(tStash + c * 32, w);
-            tmem_ld_wait();
-          }
-          const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if ((mc >> i) & 1u)
-              reinterpret_cast<float *>(box + sw128_offset(r, i >> 2))[i & 3] = qt > 0 ? __uint_as_float(w[i]) : 0.f;
-        }
-        // the box is complete once all 128 rows are in: one thread stores it
-        fence_proxy_async_smem();
-        bar_sync(is_sm ? 2 : 3, 128);
-        if (r == 0) {
-          tma_store_3d(&tmap_o, sbase + Lay::kK + c * 16384, c * 32, qt * kBlockQ, bh);
-          bulk_commit_group();
-        }
-      }
-      if (r == 0) bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
-    }
-  } else {
-    // ---------------------------------------------------------------- correction, then epilogue
-    const bool is_sm = false;
-    const int r = (tid - 128) & 127;  // row within the tile
-    const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
-    const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;
-    const float *s_alpha = reinterpret_cast<const float *>(smem + Lay::kAlpha);
-    const float *s_invL = reinterpret_cast<float *>(smem + Lay::kInvL);
-    // fix-up rows of the diagonal tile, as in the softmax warpgroup
-    int hz_base = 0, hz_rows = 0;
-    if (causal) {
-      const int2 tf = tilefix[static_cast<size_t>(bh) * n_kt_all + qt];
-      hz_base = tf.x;
-      hz_rows = tf.y;
-    }
-    const bool hz_warp = hz_rows > 32 * (warp & 3);  // warp-uniform
-    const bool hz_row = r < hz_rows;
-    const uint32_t tStash = tmem + ((qt + 1) % 3) * 128 + lane_off;
-    bool ok = true;
-    {
+    else {
       // ------------------------------------------------------------ correction
       for (int kt = 0; kt < nk; ++kt) {
         const int b = kt % 3;
@@ -553,56 +490,76 @@ __global__ void __launch_bounds__(384, 1)
     if (ok) {
       tc_fence_after_sync();
       const float invL = s_invL[r];
-      const int c_lo = is_sm ? 0 : D / 64;
+      constexpr int NC = D / 64;  // 32-column chunks of this warpgroup
+      const int c_lo = is_sm ? 0 : NC;
+      uint32_t v[NC][32];
+#pragma unroll
+      for (int c = 0; c < NC; ++c) tmem_ld32(tAcc + (c_lo + c) * 32, v[c]);
+      tmem_ld_wait();
+      // acc/L goes to the staging boxes first; the transform then runs as a
+      // rolled loop in place (this code runs once per tile and would otherwise
+      // be fetched cold, instruction by instruction)
+#pragma unroll
+      for (int c = 0; c < NC; ++c) {
+        uint8_t *box = smem + Lay::kK + (c_lo + c) * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
+#pragma unroll
+        for (int i4 = 0; i4 < 8; ++i4)
+          *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) =
+              make_float4(__uint_as_float(v[c][4 * i4]) * invL, __uint_as_float(v[c][4 * i4 + 1]) * invL,
+                          __uint_as_float(v[c][4 * i4 + 2]) * invL, __uint_as_float(v[c][4 * i4 + 3]) * invL);
+      }
 #pragma unroll 1
-      for (int c = c_lo; c < c_lo + D / 64; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tAcc + c * 32, v);
-        tmem_ld_wait();
-        uint8_t *box = smem + Lay::kK + c * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
+      for (int ci = 0; ci < NC * 8; ++ci) {
+        const int c = c_lo + (ci >> 3), i4 = ci & 7;
+        float4 *cell = reinterpret_cast<float4 *>(smem + Lay::kK + c * 16384 + sw128_offset(r, i4));
+        const float4 a4 = *cell;
+        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+        float o4[4];
 #pragma unroll
-        for (int i4 = 0; i4 < 8; ++i4) {
-          float o4[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float4 cf = c_coef[c * 32 + i4 * 4 + u];
-            const float a = __uint_as_float(v[i4 * 4 + u]) * invL;
-            // shifted bank: (log a - kappa) / beta.  Linear bank: log1p(x)/beta with
-            // x = beta a, as a times the series of log1p(x)/x for |x| < 2^-6 (also
-            // beta = 0), else log(1 + x) plus the rounding error of 1 + x over 1 + x
+        for (int u = 0; u < 4; ++u) {
+          const float4 cf = c_coef[c * 32 + i4 * 4 + u];
+          const float a = av[u];
+          if (cf.w != 0.f) {
+            o4[u] = fmaf(lg2_approx(a), cf.x, cf.y);  // c + (log a - kappa) / beta
+          } else {
+            // c + log1p(x)/beta with x = beta a: a times the series of log1p(x)/x
+            // for |x| < 2^-6 (also beta = 0), else log(1 + x) plus the rounding
+            // error of 1 + x over 1 + x
             const float x = cf.x * a;
             const float u1 = 1.f + x;
-            const float l = lg2_approx(cf.w != 0.f ? a : u1) * kLn2;
-            const float o_sh = (l - kBankOffset) * cf.y;
-            const float o_lg = fmaf((x - (u1 - 1.f)), rcp_approx(u1), l) * cf.y;
-            const float o_se = a * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f);
-            const float o = cf.w != 0.f ? o_sh : (fabsf(x) < 0.015625f ? o_se : o_lg);
-            o4[u] = cf.z + o;
+            const float lg = fmaf(x - (u1 - 1.f), rcp_approx(u1), lg2_approx(u1) * kLn2) * cf.z;
+            const float se = a * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f);
+            o4[u] = cf.y + (fabsf(x) < 0.015625f ? se : lg);
           }
-          *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(o4[0], o4[1], o4[2], o4[3]);
         }
-        if (hz_warp) {
-          // listed channels of fix-up rows: the accumulator before the diagonal tile
+        *cell = make_float4(o4[0], o4[1], o4[2], o4[3]);
+      }
+      if (hz_warp) {
+        // listed channels of fix-up rows: the accumulator before the diagonal tile
+#pragma unroll 1
+        for (int c = c_lo; c < c_lo + NC; ++c) {
           uint32_t w[32];
           if (qt > 0) {
             tmem_ld32(tStash + c * 32, w);
             tmem_ld_wait();
           }
           const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
+          uint8_t *box = smem + Lay::kK + c * 16384;
 #pragma unroll
           for (int i = 0; i < 32; ++i)
             if ((mc >> i) & 1u)
               reinterpret_cast<float *>(box + sw128_offset(r, i >> 2))[i & 3] = qt > 0 ? __uint_as_float(w[i]) : 0.f;
         }
-        // the box is complete once all 128 rows are in: one thread stores it
-        fence_proxy_async_smem();
-        bar_sync(is_sm ? 2 : 3, 128);
-        if (r == 0) {
-          tma_store_3d(&tmap_o, sbase + Lay::kK + c * 16384, c * 32, qt * kBlockQ, bh);
-          bulk_commit_group();
-        }
       }
-      if (r == 0) bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
+      // the boxes are complete once all 128 rows are in: one thread stores them
+      fence_proxy_async_smem();
+      bar_sync(is_sm ? 2 : 3, 128);
+      if (r == 0) {
+        for (int c = c_lo; c < c_lo + NC; ++c)
+          tma_store_3d(&tmap_o, sbase + Lay::kK + c * 16384, c * 32, qt * kBlockQ, bh);
+        bulk_commit_group();
+        bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
+      }
     }
   }
 
