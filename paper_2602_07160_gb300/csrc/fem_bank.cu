@@ -2,8 +2,9 @@
 // fp16 value bank, written once per key tile for every query tile to share.
 //
 //   tile_stats  (B*H x key tiles)  max, min and sum of v_.j over each tile of
-//                                  128 keys (valid keys only)
-//   plan        (B*H)              per channel: bank mode and linear anchor
+//                                  128 keys (valid keys only); the last block of
+//                                  each (b, h) to finish then runs its plan:
+//   plan        (per b, h)         per channel: bank mode and linear anchor
 //                                  from the whole sequence; the running maximum
 //                                  cpre[kt] = max over tiles 0..kt; the shifted
 //                                  bank's shift c[kt], raised lazily along cpre
@@ -34,8 +35,11 @@ struct TileMap {
 };
 
 template <int D>
-__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T,
-                                                          float4 *__restrict__ tstat) {
+__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, const float *beta,
+                                                          int H, int T, float4 *__restrict__ tstat,
+                                                          unsigned *__restrict__ done, ChanInfo *__restrict__ chan,
+                                                          float *__restrict__ cpre, float *__restrict__ shift,
+                                                          float *__restrict__ rfac, unsigned *__restrict__ colmask) {
   using M = TileMap<D>;
   __shared__ float s_max[M::RG][D], s_min[M::RG][D], s_sum[M::RG][D];
   const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x;
@@ -82,12 +86,32 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
     }
     tstat[(static_cast<size_t>(bh) * n_kt + kt) * D + j] = make_float4(a, b, c, 0.f);
   }
+  // The last of the head's tile blocks to finish plans the head (the
+  // counter is zeroed before the launch and again here, after use).
+  __shared__ bool s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    s_last = atomicAdd(&done[bh], 1u) == static_cast<unsigned>(n_kt - 1);
+    if (s_last) done[bh] = 0u;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (threadIdx.x < D) plan_head(tstat, beta, bh, H, T, D, n_kt, chan, cpre, shift, rfac, colmask);
+  if constexpr (D < 128) {
+    // mask words of channel groups beyond d stay zero
+    constexpr int kGaps = 4 - D / 32;
+    for (int i = threadIdx.x; i < n_kt * kGaps; i += 128)
+      colmask[(static_cast<size_t>(bh) * n_kt + i / kGaps) * 4 + D / 32 + i % kGaps] = 0u;
+  }
 }
 
-__global__ void plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta, int H, int T, int d,
-                            int n_kt, ChanInfo *__restrict__ chan, float *__restrict__ cpre,
-                            float *__restrict__ shift, float *__restrict__ rfac, unsigned *__restrict__ colmask) {
-  const int bh = blockIdx.x, j = threadIdx.x, h = bh % H;
+// Plan of one (b, h), thread j = channel j (j < d).
+__device__ void plan_head(const float4 *__restrict__ tstat, const float *__restrict__ beta, int bh, int H, int T,
+                          int d, int n_kt, ChanInfo *__restrict__ chan, float *__restrict__ cpre,
+                          float *__restrict__ shift, float *__restrict__ rfac, unsigned *__restrict__ colmask) {
+  const int j = threadIdx.x, h = bh % H;
   const float b = beta[h * d + j];
   const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * d + j;
   // the tiles' statistics are read kBatch at a time, all loads in flight
@@ -291,19 +315,15 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
   const dim3 grid(n_kt, BH);
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
   if (d == 64)
-    tile_stats_kernel<64><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+    tile_stats_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, H, T, w.tstat, w.done, w.chan, w.cpre, w.shift, w.rfac,
+                                                   w.colmask);
   else if (d == 128)
-    tile_stats_kernel<128><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+    tile_stats_kernel<128><<<grid, 128, 0, stream>>>(vb, beta, H, T, w.tstat, w.done, w.chan, w.cpre, w.shift, w.rfac,
+                                                    w.colmask);
   else
     return cudaErrorInvalidValue;
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (d < 128) {  // channels beyond d have no mask bits
-    e = cudaMemsetAsync(w.colmask, 0, static_cast<size_t>(BH) * n_kt * 4 * sizeof(unsigned), stream);
-    if (e != cudaSuccess) return e;
-  }
-  plan_kernel<<<BH, d, 0, stream>>>(w.tstat, beta, H, T, d, n_kt, w.chan, w.cpre, w.shift, w.rfac, w.colmask);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (d == 64)
     bank_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
                                               w.fixup_count, w.tilefix);

@@ -19,6 +19,7 @@ struct BankWorkspace {
   __half *bank;             // [B*H, T, d]: the value bank, fp16
   FixupEntry *fixups;       // exact-recompute list (causal)
   int *fixup_count;         // its length (zeroed before the pre-pass)
+  unsigned *done;           // [B*H] tile blocks finished per head (zeroed before the pre-pass)
   int2 *tilefix;            // [B*H, key tiles] (causal): {first entry, number of rows} of the tile's
                             // entries, which list the tile's rows 0 .. number-1 in order
 };
