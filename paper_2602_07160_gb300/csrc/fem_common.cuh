@@ -32,13 +32,18 @@ namespace fem {
 // accumulation is magnified.  Every other channel uses the "shifted" bank
 //   E_ij = exp(beta_j (v_ij - c_j) + kBankOffset)
 // with a running shift c_j and reads o = c + (log(acc/L) - kBankOffset)/beta.
+// Until c_j moves, E <= exp(kShiftLag + kBankOffset) = e^11 < 65504 (fp16);
+// a larger lag means fewer tiles on which acc must be rescaled for a moved
+// shift, a smaller offset that values more than about kHazardTilt/beta below
+// c leave fp16's normal range, which only happens on causal diagonal tiles
+// and is handled by the exact fix-up.
 // ---------------------------------------------------------------------------
 constexpr float kLinearLowTilt = 1.0f;
 constexpr float kLinearBankMax = 30000.f;  // fp16 holds values up to 65504
-constexpr float kBankOffset = 8.0f;        // natural-log offset of the shifted bank
-constexpr float kShiftLag = 3.0f;          // c_j moves only when beta*(new max - c) > this
+constexpr float kBankOffset = 4.0f;        // natural-log offset of the shifted bank
+constexpr float kShiftLag = 7.0f;          // c_j moves only when beta*(new max - c) > this
 constexpr float kRowMaxLag = 8.0f;         // row max moves only when it grows by > 2^this
-constexpr float kHazardTilt = 18.0f;       // row/channel recomputed exactly when beta*(c - visible max) > this
+constexpr float kHazardTilt = 14.0f;       // row/channel recomputed exactly when beta*(c - visible max) > this
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
