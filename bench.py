@@ -376,7 +376,7 @@ def run_fem(args):
             "e2e": e2e,
             "cpu_baseline": cpu,
             "clocks": clk,
-            "gpu_launches": K * (3 if w.causal else 2),
+            "gpu_launches": K * (4 if w.causal else 3),  # stats+plan, bank, tensor-core read (+ fix-up)
         }
         print(json.dumps(line), flush=True)
     if dist is not None:
