@@ -175,7 +175,7 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
                                                     const float *__restrict__ cpre, const float *__restrict__ shift,
                                                     int H, int T, int causal, __half *__restrict__ bank,
                                                     FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count,
-                                                    int2 *__restrict__ tilefix) {
+                                                    int *__restrict__ fixup_rows, int2 *__restrict__ tilefix) {
   using M = TileMap<D>;
   __shared__ float s_a[D], s_b[D], s_c[D], s_beta[D], s_lin[D], s_thr[D];
   __shared__ int s_first[D];
@@ -284,21 +284,25 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
     if (tid == 0) *tf = make_int2(0, 0);
     return;
   }
+  // the tile's entries take a multiple of 8 slots (padding rows -1), so the
+  // fix-up's 8-entry chunks never straddle two tiles
+  const int n_slots = (n_rows + 7) & ~7;
   __shared__ int s_base;
   if (tid == 0) {
-    s_base = atomicAdd(fixup_count, n_rows);
+    s_base = atomicAdd(fixup_count, n_slots);
+    atomicAdd(fixup_rows, n_rows);
     *tf = make_int2(s_base, n_rows);
   }
   __syncthreads();
-  for (int r = tid; r < n_rows; r += 128) {
+  for (int r = tid; r < n_slots; r += 128) {
     FixupEntry e;
-    e.row = bh * T + kt * kBlockQ + r;
+    e.row = r < n_rows ? bh * T + kt * kBlockQ + r : -1;
 #pragma unroll
     for (int g = 0; g < 4; ++g) {
       unsigned m = 0;
       for (int c = 0; c < 32; ++c) {
         const int j = 32 * g + c;
-        if (j < D && s_first[j] > r) m |= 1u << c;
+        if (j < D && r < n_rows && s_first[j] > r) m |= 1u << c;
       }
       e.mask[g] = m;
     }
@@ -326,10 +330,10 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
   if (e != cudaSuccess) return e;
   if (d == 64)
     bank_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
-                                              w.fixup_count, w.tilefix);
+                                              w.fixup_count, w.fixup_rows, w.tilefix);
   else
     bank_kernel<128><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
-                                               w.fixup_count, w.tilefix);
+                                               w.fixup_count, w.fixup_rows, w.tilefix);
   return cudaGetLastError();
 }
 

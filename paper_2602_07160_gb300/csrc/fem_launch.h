@@ -18,7 +18,8 @@ struct BankWorkspace {
   unsigned *colmask;        // [B*H, key tiles, 4]: bit j set when channel j's shift moved at the tile
   __half *bank;             // [B*H, T, d]: the value bank, fp16
   FixupEntry *fixups;       // exact-recompute list (causal)
-  int *fixup_count;         // its length (zeroed before the pre-pass)
+  int *fixup_count;         // its length in slots, a multiple of 8 (zeroed before the pre-pass)
+  int *fixup_rows;          // rows listed (zeroed before the pre-pass)
   unsigned *done;           // [B*H] tile blocks finished per head (zeroed before the pre-pass)
   int2 *tilefix;            // [B*H, key tiles] (causal): {first entry, number of rows} of the tile's
                             // entries, which list the tile's rows 0 .. number-1 in order
@@ -42,8 +43,8 @@ cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const
 // exactly, merged with the state the tensor-core kernel left for the earlier
 // key tiles.
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
-                         float *out, int H, int T, int d, const FixupEntry *entries, const int *count, int *last_count,
-                         int num_sms, cudaStream_t stream);
+                         float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
+                         const int *rows, int *last_rows, int num_sms, cudaStream_t stream);
 
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
