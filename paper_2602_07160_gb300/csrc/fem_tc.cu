@@ -124,9 +124,9 @@ __global__ void __launch_bounds__(384, 1)
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + Lay::kAbort);
-  // per channel, for the epilogue: shifted bank {ln2/beta, c - kappa/beta, 0, 1}
-  // with c the last shift, so o = lg2(a) * x + y; linear bank {beta, c, 1/beta
-  // (0 at beta = 0), 0} with c the anchor
+  // per channel, for the epilogue: shifted bank {0, c - kappa/beta, ln2/beta, 1}
+  // with c the last shift; linear bank {beta, c, ln2/beta (0 at beta = 0), 0}
+  // with c the anchor
   float4 *c_coef = reinterpret_cast<float4 *>(smem + Lay::kChan);
   unsigned *move_bits = reinterpret_cast<unsigned *>(smem + Lay::kMoveBits);
   const uint32_t bars = sbase + Lay::kBar;
@@ -202,10 +202,10 @@ __global__ void __launch_bounds__(384, 1)
     const float bj = beta[h * D + j];
     const bool lin = ci.linear != 0.f;
     if (lin) {
-      c_coef[j] = make_float4(bj, ci.c_lin, bj != 0.f ? 1.f / bj : 0.f, 0.f);
+      c_coef[j] = make_float4(bj, ci.c_lin, bj != 0.f ? kLn2 / bj : 0.f, 0.f);
     } else {
       const float c = shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j];
-      c_coef[j] = make_float4(kLn2 / bj, c - kBankOffset / bj, 0.f, 1.f);
+      c_coef[j] = make_float4(0.f, c - kBankOffset / bj, kLn2 / bj, 1.f);
     }
   }
   // one bit per key tile: set when some channel's shift moved there
@@ -517,20 +517,15 @@ __global__ void __launch_bounds__(384, 1)
         float o4[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
+          // shifted bank: c + (log a - kappa)/beta = lg2(a) ln2/beta + (c - kappa/beta);
+          // linear bank: c + log1p(x)/beta with x = beta a, as lg2(1 + x) ln2/beta + c,
+          // or, for |x| < 2^-6 (also beta = 0), as c + a times the series of log1p(x)/x
           const float4 cf = c_coef[c * 32 + i4 * 4 + u];
           const float a = av[u];
-          if (cf.w != 0.f) {
-            o4[u] = fmaf(lg2_approx(a), cf.x, cf.y);  // c + (log a - kappa) / beta
-          } else {
-            // c + log1p(x)/beta with x = beta a: a times the series of log1p(x)/x
-            // for |x| < 2^-6 (also beta = 0), else log(1 + x) plus the rounding
-            // error of 1 + x over 1 + x
-            const float x = cf.x * a;
-            const float u1 = 1.f + x;
-            const float lg = fmaf(x - (u1 - 1.f), rcp_approx(u1), lg2_approx(u1) * kLn2) * cf.z;
-            const float se = a * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f);
-            o4[u] = cf.y + (fabsf(x) < 0.015625f ? se : lg);
-          }
+          const float x = cf.x * a;
+          const float lg = fmaf(lg2_approx(cf.w != 0.f ? a : 1.f + x), cf.z, cf.y);
+          const float se = fmaf(a, fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f), cf.y);
+          o4[u] = (cf.w == 0.f && fabsf(x) < 0.015625f) ? se : lg;
         }
         *cell = make_float4(o4[0], o4[1], o4[2], o4[3]);
       }
