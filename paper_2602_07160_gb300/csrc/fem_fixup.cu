@@ -21,9 +21,10 @@
 // Entries come in chunks of 8 consecutive rows of one diagonal tile (the
 // pre-pass pads each tile's entries to a multiple of 8 with rows -1).  One
 // 256-thread block takes a chunk at a time (grid-stride): it stages the tile's
-// K and V rows k0 .. k0+r_max in shared memory (rows padded by one 32-bit
-// word, so reading one column across rows is free of bank conflicts), then
-// each warp completes one entry: its lanes score four keys each and reduce
+// K and V rows k0 .. k0+r_max and the chunk's 8 query rows in shared memory,
+// scores the 8 rows against the keys with warp-level bf16 MMAs (16 keys per
+// warp, fp32 accumulation), then each warp completes one entry: its lanes
+// take four keys each and reduce
 // the row's log-sum-exp and, channel by channel, each listed channel's with
 // warp shuffles; a 32-channel group with three or more listed channels is
 // done with lane = channel instead, walking the keys in turn.
@@ -45,6 +46,23 @@ __device__ __forceinline__ float warp_sum(float x) {
   return x;
 }
 
+// Four 8x8 bf16 matrices from shared memory (lane l gives the address of row
+// l % 8 of matrix l / 8), in the mma fragment layout.
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+
+// c += A (16x16, row-major) B (16x8, column-major), bf16 in, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
 // log2(2^a + 2^b) for a, b possibly -inf
 __device__ __forceinline__ float lse2_pair(float a, float b) {
   const float mx = fmaxf(a, b);
@@ -62,12 +80,15 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
                                                             const int *__restrict__ count,
                                                             const int *__restrict__ rows_listed,
                                                             int *__restrict__ last_rows) {
-  constexpr int KS = D + 2;  // staged row stride in bf16 elements (an odd number of 32-bit words)
+  // staged row strides in bf16 elements: K and Q rows 16-byte aligned for
+  // ldmatrix with consecutive rows four banks apart; V rows an odd number of
+  // 32-bit words, so one column read across rows is free of bank conflicts
+  constexpr int KS = D + 8, VS = D + 2;
   extern __shared__ __align__(16) uint8_t fix_smem[];
   __nv_bfloat16 *sK = reinterpret_cast<__nv_bfloat16 *>(fix_smem);
   __nv_bfloat16 *sV = sK + kBlockK * KS;
-  __shared__ float sQ[kFixChunk][D];
-  __shared__ float sS[kFixChunk][kBlockK];  // each warp's row scores, for the channel-parallel form
+  __nv_bfloat16 *sQ = sV + kBlockK * VS;  // 16 rows (8 entries, 8 unused) of KS
+  __shared__ float sS[kFixChunk][kBlockK];  // the chunk's scores, log2 units
   __shared__ int s_nk;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_chunks = *count / kFixChunk;
@@ -91,19 +112,40 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
       const size_t g = (static_cast<size_t>(bh) * T + k0 + i) * D + 8 * c;
       const uint4 kr = *reinterpret_cast<const uint4 *>(k + g);
       const uint4 vr = *reinterpret_cast<const uint4 *>(v + g);
-      uint32_t *dk = reinterpret_cast<uint32_t *>(sK + i * KS + 8 * c);
-      uint32_t *dv = reinterpret_cast<uint32_t *>(sV + i * KS + 8 * c);
-      dk[0] = kr.x;
-      dk[1] = kr.y;
-      dk[2] = kr.z;
-      dk[3] = kr.w;
+      *reinterpret_cast<uint4 *>(sK + i * KS + 8 * c) = kr;
+      uint32_t *dv = reinterpret_cast<uint32_t *>(sV + i * VS + 8 * c);
       dv[0] = vr.x;
       dv[1] = vr.y;
       dv[2] = vr.z;
       dv[3] = vr.w;
     }
-    if (r >= 0)
-      for (int d = lane; d < D; d += 32) sQ[warp][d] = __bfloat162float(q[static_cast<size_t>(ent.row) * D + d]);
+    for (int idx = tid; idx < kFixChunk * (D / 8); idx += kFixThreads) {
+      const int w = idx / (D / 8), c = idx % (D / 8);
+      const int erow = entries[ch * kFixChunk + w].row;
+      *reinterpret_cast<uint4 *>(sQ + w * KS + 8 * c) =
+          erow >= 0 ? *reinterpret_cast<const uint4 *>(q + static_cast<size_t>(erow) * D + 8 * c) : make_uint4(0, 0, 0, 0);
+    }
+    __syncthreads();
+    // S[8 x nk] = Q K^T: warp w takes keys 16w .. 16w+15 (two n8 blocks) over
+    // D/16 k-steps of m16n8k16 (rows 8..15 of A are unused)
+    if (16 * warp < nk) {
+      float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int ks = 0; ks < D / 16; ++ks) {
+        uint32_t a[4], bfr[4];
+        ldmatrix_x4(a, smem_u32(sQ + (lane % 16) * KS + 16 * ks + (lane / 16) * 8));
+        const int mm = lane / 8;  // matrices: (keys lo, d lo) (keys lo, d hi) (keys hi, d lo) (keys hi, d hi)
+        ldmatrix_x4(bfr, smem_u32(sK + (16 * warp + (mm / 2) * 8 + lane % 8) * KS + 16 * ks + (mm % 2) * 8));
+        mma_bf16_16816(c0, a, bfr[0], bfr[1]);
+        mma_bf16_16816(c1, a, bfr[2], bfr[3]);
+      }
+      // fragment rows lane/4 (and lane/4 + 8, unused), columns 2 (lane % 4) + {0, 1}
+      const int rr = lane / 4, cc = 16 * warp + 2 * (lane % 4);
+      sS[rr][cc] = c0[0] * scale;
+      sS[rr][cc + 1] = c0[1] * scale;
+      sS[rr][cc + 8] = c1[0] * scale;
+      sS[rr][cc + 9] = c1[1] * scale;
+    }
     __syncthreads();
     if (r >= 0) {
       // scores of keys i = lane + 32u (log2 units), -inf past the row
@@ -111,25 +153,8 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
 #pragma unroll
       for (int u = 0; u < kBlockK / 32; ++u) {
         const int i = lane + 32 * u;
-        float acc = -INFINITY;
-        if (i <= r) {
-          acc = 0.f;
-          const __nv_bfloat162 *kr = reinterpret_cast<const __nv_bfloat162 *>(sK + i * KS);
-          const float2 *qr = reinterpret_cast<const float2 *>(sQ[warp]);
-#pragma unroll 8
-          for (int d2 = 0; d2 < D / 2; ++d2) {
-            const float2 kf = __bfloat1622float2(kr[d2]);
-            const float2 qf = qr[d2];
-            acc = fmaf(qf.x, kf.x, acc);
-            acc = fmaf(qf.y, kf.y, acc);
-          }
-          acc *= scale;
-        }
-        s[u] = acc;
+        s[u] = i <= r ? sS[warp][i] : -INFINITY;
       }
-#pragma unroll
-      for (int u = 0; u < kBlockK / 32; ++u) sS[warp][lane + 32 * u] = s[u];
-      __syncwarp();
       // the row's score log-sum-exp over all its keys
       float mx = s[0];
 #pragma unroll
@@ -160,9 +185,9 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
           const int j = 32 * gi + lane;
           const float bl = b_reg[gi] * kLog2e;
           float mj = -INFINITY;
-          for (int i = 0; i <= r; ++i) mj = fmaxf(mj, fmaf(bl, __bfloat162float(sV[i * KS + j]), sS[warp][i]));
+          for (int i = 0; i <= r; ++i) mj = fmaxf(mj, fmaf(bl, __bfloat162float(sV[i * VS + j]), sS[warp][i]));
           float sj = 0.f;
-          for (int i = 0; i <= r; ++i) sj += exp2f(fmaf(bl, __bfloat162float(sV[i * KS + j]), sS[warp][i]) - mj);
+          for (int i = 0; i <= r; ++i) sj += exp2f(fmaf(bl, __bfloat162float(sV[i * VS + j]), sS[warp][i]) - mj);
           if ((m >> lane) & 1u) {
             float pre = -INFINITY;
             if (kt > 0 && a_reg[gi] > 0.f && ent.l_pre > 0.f)
@@ -185,7 +210,7 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
 #pragma unroll
           for (int u = 0; u < kBlockK / 32; ++u) {
             const int i = lane + 32 * u;
-            x[u] = i <= r ? fmaf(bl, __bfloat162float(sV[i * KS + j]), s[u]) : -INFINITY;
+            x[u] = i <= r ? fmaf(bl, __bfloat162float(sV[i * VS + j]), s[u]) : -INFINITY;
             mj = fmaxf(mj, x[u]);
           }
           mj = warp_max(mj);
@@ -213,11 +238,11 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
                       *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = num_sms * 3;
   if (d == 64) {
-    const size_t smem = 2 * kBlockK * (64 + 2) * sizeof(__nv_bfloat16);
+    const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
     fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
                                                           last_rows);
   } else if (d == 128) {
-    const size_t smem = 2 * kBlockK * (128 + 2) * sizeof(__nv_bfloat16);
+    const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
     cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
