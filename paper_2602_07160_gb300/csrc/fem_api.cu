@@ -113,8 +113,8 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += causal ? round256(BH * n_kt * kBlockQ * sizeof(FixupEntry)) : 0;
   w->tilefix = off;
   off += causal ? round256(BH * n_kt * sizeof(int2)) : 0;
-  w->count = off;  // fix-up slots, fix-up rows, then one finished-tile counter per head
-  off += round256(sizeof(int) * (2 + BH));
+  w->count = off;  // fix-up slots, fix-up rows
+  off += 256;
   w->total = off;
   return true;
 }
@@ -212,7 +212,6 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
   bw.fixup_rows = reinterpret_cast<int *>(ws + w.count) + 1;
-  bw.done = reinterpret_cast<unsigned *>(ws + w.count) + 2;
   bw.tilefix = causal ? reinterpret_cast<int2 *>(ws + w.tilefix) : nullptr;
 
   CUtensorMap tq, tk, te, to;
@@ -222,7 +221,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   if ((rc = make_map(&to, out, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4)) != FEM_OK) return rc;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, sizeof(int) * (2 + static_cast<size_t>(BH)), s);
+  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 2 * sizeof(int), s);
   if (e == cudaSuccess) e = launch_value_bank(v, beta, BH, H, T, d, causal, bw, s);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;

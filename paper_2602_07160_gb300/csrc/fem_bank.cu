@@ -2,9 +2,8 @@
 // fp16 value bank, written once per key tile for every query tile to share.
 //
 //   tile_stats  (B*H x key tiles)  max, min and sum of v_.j over each tile of
-//                                  128 keys (valid keys only); the last block of
-//                                  each (b, h) to finish then runs its plan:
-//   plan        (per b, h)         per channel: bank mode and linear anchor
+//                                  128 keys (valid keys only)
+//   plan        (B*H)              per channel: bank mode and linear anchor
 //                                  from the whole sequence; the running maximum
 //                                  cpre[kt] = max over tiles 0..kt; the shifted
 //                                  bank's shift c[kt], raised lazily along cpre
@@ -35,11 +34,8 @@ struct TileMap {
 };
 
 template <int D>
-__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, const float *beta,
-                                                          int H, int T, float4 *__restrict__ tstat,
-                                                          unsigned *__restrict__ done, ChanInfo *__restrict__ chan,
-                                                          float *__restrict__ cpre, float *__restrict__ shift,
-                                                          float *__restrict__ rfac, unsigned *__restrict__ colmask) {
+__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T,
+                                                          float4 *__restrict__ tstat) {
   using M = TileMap<D>;
   __shared__ float s_max[M::RG][D], s_min[M::RG][D], s_sum[M::RG][D];
   const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x;
@@ -86,48 +82,45 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
     }
     tstat[(static_cast<size_t>(bh) * n_kt + kt) * D + j] = make_float4(a, b, c, 0.f);
   }
-  // The last of the head's tile blocks to finish plans the head (the
-  // counter is zeroed before the launch and again here, after use).
-  __shared__ bool s_last;
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    s_last = atomicAdd(&done[bh], 1u) == static_cast<unsigned>(n_kt - 1);
-    if (s_last) done[bh] = 0u;
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (threadIdx.x < D) plan_head(tstat, beta, bh, H, T, D, n_kt, chan, cpre, shift, rfac, colmask);
-  if constexpr (D < 128) {
-    // mask words of channel groups beyond d stay zero
-    constexpr int kGaps = 4 - D / 32;
-    for (int i = threadIdx.x; i < n_kt * kGaps; i += 128)
-      colmask[(static_cast<size_t>(bh) * n_kt + i / kGaps) * 4 + D / 32 + i % kGaps] = 0u;
-  }
 }
 
-// Plan of one (b, h), thread j = channel j (j < d).
-__device__ void plan_head(const float4 *__restrict__ tstat, const float *__restrict__ beta, int bh, int H, int T,
-                          int d, int n_kt, ChanInfo *__restrict__ chan, float *__restrict__ cpre,
-                          float *__restrict__ shift, float *__restrict__ rfac, unsigned *__restrict__ colmask) {
-  const int j = threadIdx.x, h = bh % H;
-  const float b = beta[h * d + j];
-  const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * d + j;
-  // the tiles' statistics are read kBatch at a time, all loads in flight
-  constexpr int kBatch = 8;
+// Plan of one (b, h) per block: four threads per channel, each holding a
+// quarter of a window of 64 key tiles in registers, so every load of a window
+// is in flight at once.  The lazy shift is a sequential recurrence over tiles:
+// the four quarters run it in turn, handing the running (max, shift) on by
+// warp shuffles.
+template <int D>
+__global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta,
+                                                     int H, int T, int n_kt, ChanInfo *__restrict__ chan,
+                                                     float *__restrict__ cpre, float *__restrict__ shift,
+                                                     float *__restrict__ rfac, unsigned *__restrict__ colmask) {
+  constexpr int kParts = 4, kPer = 16, kWin = kParts * kPer;
+  __shared__ unsigned s_mask[kWin][4];
+  const int tid = threadIdx.x, j = tid / kParts, part = tid % kParts, lane = tid & 31;
+  const int bh = blockIdx.x, h = bh % H;
+  const float b = beta[h * D + j];
+  const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * D + j;
+  // pass 1: the channel's max, min and sum over every key tile
   float gmax = -INFINITY, gmin = INFINITY, gsum = 0.f;
-  for (int k0 = 0; k0 < n_kt; k0 += kBatch) {
-    float4 st[kBatch];
+  for (int w0 = 0; w0 < n_kt; w0 += kWin) {
+    float4 st[kPer];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u)
-      st[u] = k0 + u < n_kt ? ts[static_cast<size_t>(k0 + u) * d] : make_float4(-INFINITY, INFINITY, 0.f, 0.f);
+    for (int u = 0; u < kPer; ++u) {
+      const int kt = w0 + part * kPer + u;
+      st[u] = kt < n_kt ? ts[static_cast<size_t>(kt) * D] : make_float4(-INFINITY, INFINITY, 0.f, 0.f);
+    }
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < kPer; ++u) {
       gmax = fmaxf(gmax, st[u].x);
       gmin = fminf(gmin, st[u].y);
       gsum += st[u].z;
     }
+  }
+#pragma unroll
+  for (int off = 1; off < kParts; off <<= 1) {
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gsum += __shfl_xor_sync(0xffffffffu, gsum, off);
   }
   const float mean = gsum / static_cast<float>(T);
   ChanInfo ci;
@@ -140,32 +133,51 @@ __device__ void plan_head(const float4 *__restrict__ tstat, const float *__restr
     ci.linear = 1.f;
     ci.c_lin = mean;
   }
-  chan[bh * d + j] = ci;
+  if (part == 0) chan[bh * D + j] = ci;
   const bool lin = ci.linear != 0.f;
+  // pass 2: running maximum, lazy shift, rescale factors, moved-channel masks
   float cp = -INFINITY, cl = -INFINITY;
-  for (int k0 = 0; k0 < n_kt; k0 += kBatch) {
-    float tmx[kBatch];
+  for (int w0 = 0; w0 < n_kt; w0 += kWin) {
+    float tmx[kPer];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) tmx[u] = k0 + u < n_kt ? ts[static_cast<size_t>(k0 + u) * d].x : -INFINITY;
+    for (int u = 0; u < kPer; ++u) {
+      const int kt = w0 + part * kPer + u;
+      tmx[u] = kt < n_kt ? ts[static_cast<size_t>(kt) * D].x : -INFINITY;
+    }
+    for (int i = tid; i < kWin * 4; i += kParts * D) s_mask[i / 4][i % 4] = 0u;
+    __syncthreads();
+    for (int stage = 0; stage < kParts; ++stage) {
+      if (part == stage) {
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-    const int kt = k0 + u;
-    if (kt >= n_kt) break;  // uniform over the block
-    cp = fmaxf(cp, tmx[u]);
-    const float prev = cl;
-    if (lin) {
-      cl = ci.c_lin;
-    } else if (cl == -INFINITY || b * (cp - cl) > kShiftLag) {
-      cl = cp;
+        for (int u = 0; u < kPer; ++u) {
+          const int kt = w0 + stage * kPer + u;
+          if (kt < n_kt) {
+            cp = fmaxf(cp, tmx[u]);
+            const float prev = cl;
+            if (lin) {
+              cl = ci.c_lin;
+            } else if (cl == -INFINITY || b * (cp - cl) > kShiftLag) {
+              cl = cp;
+            }
+            const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
+            cpre[o] = cp;
+            shift[o] = cl;
+            const bool moved = !lin && kt > 0 && cl != prev;
+            rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
+            if (moved) atomicOr(&s_mask[stage * kPer + u][j >> 5], 1u << (j & 31));
+          }
+        }
+      }
+      // the quarter that ran hands its state on to the channel's other lanes
+      cp = __shfl_sync(0xffffffffu, cp, (lane & ~(kParts - 1)) | stage);
+      cl = __shfl_sync(0xffffffffu, cl, (lane & ~(kParts - 1)) | stage);
     }
-    const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * d + j;
-    cpre[o] = cp;
-    shift[o] = cl;
-    const int moved = (!lin && kt > 0 && cl != prev) ? 1 : 0;
-    rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
-    const unsigned bits = __ballot_sync(0xffffffffu, moved);
-    if ((j & 31) == 0) colmask[(static_cast<size_t>(bh) * n_kt + kt) * 4 + (j >> 5)] = bits;
+    __syncthreads();
+    for (int i = tid; i < kWin * 4; i += kParts * D) {
+      const int kt = w0 + i / 4;
+      if (kt < n_kt) colmask[(static_cast<size_t>(bh) * n_kt + kt) * 4 + i % 4] = s_mask[i / 4][i % 4];
     }
+    __syncthreads();
   }
 }
 
@@ -318,14 +330,16 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
   const int n_kt = (T + kBlockK - 1) / kBlockK;
   const dim3 grid(n_kt, BH);
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
-  if (d == 64)
-    tile_stats_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, H, T, w.tstat, w.done, w.chan, w.cpre, w.shift, w.rfac,
-                                                   w.colmask);
-  else if (d == 128)
-    tile_stats_kernel<128><<<grid, 128, 0, stream>>>(vb, beta, H, T, w.tstat, w.done, w.chan, w.cpre, w.shift, w.rfac,
-                                                    w.colmask);
-  else
+  if (d == 64) {
+    tile_stats_kernel<64><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+    plan_kernel<64><<<BH, 4 * 64, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.cpre, w.shift, w.rfac, w.colmask);
+  } else if (d == 128) {
+    tile_stats_kernel<128><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+    plan_kernel<128><<<BH, 4 * 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.cpre, w.shift, w.rfac,
+                                                 w.colmask);
+  } else {
     return cudaErrorInvalidValue;
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (d == 64)

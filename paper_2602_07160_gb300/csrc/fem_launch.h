@@ -20,7 +20,6 @@ struct BankWorkspace {
   FixupEntry *fixups;       // exact-recompute list (causal)
   int *fixup_count;         // its length in slots, a multiple of 8 (zeroed before the pre-pass)
   int *fixup_rows;          // rows listed (zeroed before the pre-pass)
-  unsigned *done;           // [B*H] tile blocks finished per head (zeroed before the pre-pass)
   int2 *tilefix;            // [B*H, key tiles] (causal): {first entry, number of rows} of the tile's
                             // entries, which list the tile's rows 0 .. number-1 in order
 };
