@@ -222,7 +222,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 2 * sizeof(int), s);
-  if (e == cudaSuccess) e = launch_value_bank(v, beta, BH, H, T, d, causal, bw, s);
+  if (e == cudaSuccess) e = launch_value_bank(v, beta, BH, H, T, d, causal, bw, ds->err, s);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);

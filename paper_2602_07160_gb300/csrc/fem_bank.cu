@@ -33,13 +33,35 @@ struct TileMap {
   static constexpr int RPG = 128 / RG;
 };
 
+// Both kernels stream the tile's rows (contiguous in V) into shared memory
+// with one bulk copy, which keeps the HBM reads in flight independently of the
+// threads' own load slots.
+template <int D>
+__device__ __forceinline__ bool stage_tile(const __nv_bfloat16 *v, int T, int bh, int kt, uint8_t *dst,
+                                           uint64_t *bar_word, unsigned *err) {
+  const uint32_t bar = smem_u32(bar_word);
+  const int rows = min(kBlockK, T - kt * kBlockK);
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(rows * D * 2));
+    bulk_load(smem_u32(dst), v + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D,
+              static_cast<uint32_t>(rows * D * 2), bar);
+  }
+  __syncthreads();
+  return mbar_wait(bar, 0, err, kErrWaitTma);
+}
+
 template <int D>
 __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T,
-                                                          float4 *__restrict__ tstat) {
+                                                          float4 *__restrict__ tstat, unsigned *__restrict__ err) {
   using M = TileMap<D>;
+  extern __shared__ __align__(16) uint8_t tile_smem[];  // the tile's rows, [128][D] bf16
+  __shared__ __align__(8) uint64_t s_bar;
   __shared__ float s_max[M::RG][D], s_min[M::RG][D], s_sum[M::RG][D];
   const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x;
   const int cc = threadIdx.x % M::CPR, rg = threadIdx.x / M::CPR;
+  if (!stage_tile<D>(v, T, bh, kt, tile_smem, &s_bar, err)) return;
   float mx[8], mn[8], sm[8];
 #pragma unroll
   for (int u = 0; u < 8; ++u) {
@@ -47,12 +69,11 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
     mn[u] = INFINITY;
     sm[u] = 0.f;
   }
-  const __nv_bfloat16 *vb = v + static_cast<size_t>(bh) * T * D;
 #pragma unroll
   for (int i = 0; i < M::RPG; ++i) {
-    const int key = kt * kBlockK + rg * M::RPG + i;
-    if (key < T) {
-      const uint4 raw = *reinterpret_cast<const uint4 *>(vb + static_cast<size_t>(key) * D + cc * 8);
+    const int row = rg * M::RPG + i;
+    if (kt * kBlockK + row < T) {
+      const uint4 raw = *reinterpret_cast<const uint4 *>(tile_smem + (row * D + cc * 8) * 2);
       const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
@@ -182,14 +203,17 @@ __global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ 
 }
 
 template <int D>
-__global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__restrict__ v,
+__global__ void __launch_bounds__(128, 3) bank_kernel(const __nv_bfloat16 *__restrict__ v,
                                                     const float *__restrict__ beta, const ChanInfo *__restrict__ chan,
                                                     const float *__restrict__ cpre, const float *__restrict__ shift,
                                                     int H, int T, int causal, __half *__restrict__ bank,
                                                     FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count,
-                                                    int *__restrict__ fixup_rows, int2 *__restrict__ tilefix) {
+                                                    int *__restrict__ fixup_rows, int2 *__restrict__ tilefix,
+                                                    unsigned *__restrict__ err) {
   using M = TileMap<D>;
-  __shared__ float s_a[D], s_b[D], s_c[D], s_beta[D], s_lin[D], s_thr[D];
+  extern __shared__ __align__(16) uint8_t tile_smem[];  // the tile's rows of V, then of the bank, in place
+  __shared__ __align__(8) uint64_t s_bar;
+  __shared__ float s_a[D], s_b[D], s_c[D], s_lin[D], s_thr[D];
   __shared__ int s_first[D];
   const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x, h = bh % H;
   const int tid = threadIdx.x;
@@ -199,12 +223,11 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
     const ChanInfo ci = chan[bh * D + j];
     const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
     const float c = shift[o];
-    s_beta[j] = b;
     s_lin[j] = ci.linear;
     s_c[j] = c;
     if (ci.linear != 0.f) {
-      s_a[j] = b > 0.f ? 1.f / b : 0.f;  // linear bank: 1/beta
-      s_b[j] = 0.f;
+      s_a[j] = b > 0.f ? 1.f / b : 0.f;  // linear bank: 1/beta and beta
+      s_b[j] = b;
     } else {
       s_a[j] = b * kLog2e;  // shifted bank: E = ex2(a v + b)
       s_b[j] = (kBankOffset - b * c) * kLog2e;
@@ -219,12 +242,12 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
   }
   __syncthreads();
 
-  // Thread: the 8 channels of chunk column cc, rows rg*RPG .. rg*RPG+RPG-1.
-  // Consecutive threads read consecutive 16-byte chunks of a row.  Both bank
+  if (!stage_tile<D>(v, T, bh, kt, tile_smem, &s_bar, err)) return;
+  // Thread: the 8 channels of chunk column cc, rows rg*RPG .. rg*RPG+RPG-1,
+  // each 16-byte chunk of V replaced by the chunk of the bank.  Both bank
   // forms are evaluated and one is selected, so lanes never diverge.
-  const __nv_bfloat16 *vb = v + static_cast<size_t>(bh) * T * D;
-  __half *eb = bank + static_cast<size_t>(bh) * T * D;
-  float pa[8], pb[8], pc[8], pbeta[8], pthr[8];
+  const int rows = min(kBlockK, T - kt * kBlockK);
+  float pa[8], pb[8], pc[8], pthr[8];
   bool plin[8];
   int first[8];
 #pragma unroll
@@ -233,26 +256,18 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
     pa[u] = s_a[j];
     pb[u] = s_b[j];
     pc[u] = s_c[j];
-    pbeta[u] = s_beta[j];
     pthr[u] = s_thr[j];
     plin[u] = s_lin[j] != 0.f;
     first[u] = kBlockK;
   }
-#pragma unroll 1
-  for (int i0 = 0; i0 < M::RPG; i0 += 4) {
-    uint4 raw[4];
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const int key = kt * kBlockK + rg * M::RPG + i0 + r;
-      raw[r] = key < T ? *reinterpret_cast<const uint4 *>(vb + static_cast<size_t>(key) * D + cc * 8)
-                       : make_uint4(0, 0, 0, 0);
-    }
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const int row = rg * M::RPG + i0 + r;
-      const int key = kt * kBlockK + row;
-      if (key >= T) break;
-      const __nv_bfloat16 *vin = reinterpret_cast<const __nv_bfloat16 *>(&raw[r]);
+#pragma unroll 2
+  for (int i = 0; i < M::RPG; ++i) {
+    {
+      const int row = rg * M::RPG + i;
+      if (row >= rows) break;
+      uint4 *cell = reinterpret_cast<uint4 *>(tile_smem + (row * D + cc * 8) * 2);
+      const uint4 raw = *cell;
+      const __nv_bfloat16 *vin = reinterpret_cast<const __nv_bfloat16 *>(&raw);
       __align__(16) __half e[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
@@ -262,7 +277,7 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
         // series of expm1(y)/y for |y| < 1/2 (truncation < 4e-6 relative),
         // e^y - 1 beyond; shifted bank: E = 2^(a v + b)
         const float xs = x - pc[u];
-        const float y = pbeta[u] * xs;
+        const float y = pb[u] * xs;
         float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
         poly = fmaf(y, poly, 1.f / 24.f);
         poly = fmaf(y, poly, 1.f / 6.f);
@@ -272,15 +287,26 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
         const float shf = ex2_approx(fmaf(pa[u], x, pb[u]));
         e[u] = __float2half_rn(plin[u] ? lin : shf);
       }
-      *reinterpret_cast<uint4 *>(eb + static_cast<size_t>(key) * D + cc * 8) = *reinterpret_cast<const uint4 *>(e);
+      *cell = *reinterpret_cast<const uint4 *>(e);
     }
+  }
+  // the tile of the bank leaves with one bulk store
+  fence_proxy_async_smem();
+  __syncthreads();
+  if (tid == 0) {
+    bulk_store(bank + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D, smem_u32(tile_smem),
+               static_cast<uint32_t>(rows * D * 2));
+    bulk_commit_group();
   }
   if (causal) {
 #pragma unroll
     for (int u = 0; u < 8; ++u)
       if (first[u] < kBlockK) atomicMin(&s_first[cc * 8 + u], first[u]);
   }
-  if (!causal) return;
+  if (!causal) {
+    if (tid == 0) bulk_wait_group_read0();
+    return;
+  }
   __syncthreads();
   // rows r < max_j first_j of this tile get one entry with their channel masks
   __shared__ int s_rows;
@@ -293,7 +319,10 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
   const int n_rows = s_rows;
   int2 *tf = tilefix + static_cast<size_t>(bh) * n_kt + kt;
   if (n_rows <= 0) {
-    if (tid == 0) *tf = make_int2(0, 0);
+    if (tid == 0) {
+      *tf = make_int2(0, 0);
+      bulk_wait_group_read0();
+    }
     return;
   }
   // the tile's entries take a multiple of 8 slots (padding rows -1), so the
@@ -323,18 +352,19 @@ __global__ void __launch_bounds__(128, 4) bank_kernel(const __nv_bfloat16 *__res
     e.pad = 0;
     fixups[s_base + r] = e;
   }
+  if (tid == 0) bulk_wait_group_read0();
 }
 
 cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
-                              const BankWorkspace &w, cudaStream_t stream) {
+                              const BankWorkspace &w, unsigned *err, cudaStream_t stream) {
   const int n_kt = (T + kBlockK - 1) / kBlockK;
   const dim3 grid(n_kt, BH);
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
   if (d == 64) {
-    tile_stats_kernel<64><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+    tile_stats_kernel<64><<<grid, 128, kBlockK * 64 * 2, stream>>>(vb, T, w.tstat, err);
     plan_kernel<64><<<BH, 4 * 64, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.cpre, w.shift, w.rfac, w.colmask);
   } else if (d == 128) {
-    tile_stats_kernel<128><<<grid, 128, 0, stream>>>(vb, T, w.tstat);
+    tile_stats_kernel<128><<<grid, 128, kBlockK * 128 * 2, stream>>>(vb, T, w.tstat, err);
     plan_kernel<128><<<BH, 4 * 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.cpre, w.shift, w.rfac,
                                                  w.colmask);
   } else {
@@ -343,11 +373,12 @@ cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, i
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (d == 64)
-    bank_kernel<64><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
-                                              w.fixup_count, w.fixup_rows, w.tilefix);
+    bank_kernel<64><<<grid, 128, kBlockK * 64 * 2, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank,
+                                                             w.fixups, w.fixup_count, w.fixup_rows, w.tilefix, err);
   else
-    bank_kernel<128><<<grid, 128, 0, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank, w.fixups,
-                                               w.fixup_count, w.fixup_rows, w.tilefix);
+    bank_kernel<128><<<grid, 128, kBlockK * 128 * 2, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal,
+                                                               w.bank, w.fixups, w.fixup_count, w.fixup_rows,
+                                                               w.tilefix, err);
   return cudaGetLastError();
 }
 

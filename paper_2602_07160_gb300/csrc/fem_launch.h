@@ -26,7 +26,7 @@ struct BankWorkspace {
 
 // Statistics, plan and value bank (two reads of V, one write of the bank).
 cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
-                              const BankWorkspace &w, cudaStream_t stream);
+                              const BankWorkspace &w, unsigned *err, cudaStream_t stream);
 
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
 // `to` maps the fp32 output [B*H, T, d] for the kernel's TMA stores.  For the
