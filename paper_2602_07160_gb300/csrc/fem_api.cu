@@ -87,7 +87,7 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-  size_t tstat, chan, cpre, shift, rfac, colmask, bank, fixups, tilefix, count, total;
+  size_t tstat, chan, bcoef, shift, rfac, colmask, bank, fixups, tilefix, count, total;
 };
 
 bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
@@ -101,8 +101,8 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += round256(BH * n_kt * d * sizeof(float4));
   w->chan = off;
   off += round256(BH * d * sizeof(ChanInfo));
-  w->cpre = off;
-  off += round256(BH * n_kt * d * sizeof(float));
+  w->bcoef = off;
+  off += round256(BH * n_kt * d * sizeof(float4));
   w->shift = off;
   off += round256(BH * n_kt * d * sizeof(float));
   w->rfac = off;
@@ -204,7 +204,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   BankWorkspace bw;
   bw.tstat = reinterpret_cast<float4 *>(ws + w.tstat);
   bw.chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
-  bw.cpre = reinterpret_cast<float *>(ws + w.cpre);
+  bw.bcoef = reinterpret_cast<float4 *>(ws + w.bcoef);
   bw.shift = reinterpret_cast<float *>(ws + w.shift);
   bw.rfac = reinterpret_cast<float *>(ws + w.rfac);
   bw.colmask = reinterpret_cast<unsigned *>(ws + w.colmask);
@@ -214,20 +214,20 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   bw.fixup_rows = reinterpret_cast<int *>(ws + w.count) + 1;
   bw.tilefix = causal ? reinterpret_cast<int2 *>(ws + w.tilefix) : nullptr;
 
-  CUtensorMap tq, tk, te, to;
+  CUtensorMap tq, tk, tv, te;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&tk, k, BH, T, d)) != FEM_OK) return rc;
+  if ((rc = make_map(&tv, v, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&te, bw.bank, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT16)) != FEM_OK) return rc;
-  if ((rc = make_map(&to, out, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4)) != FEM_OK) return rc;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 2 * sizeof(int), s);
-  if (e == cudaSuccess) e = launch_value_bank(v, beta, BH, H, T, d, causal, bw, ds->err, s);
+  if (e == cudaSuccess) e = launch_value_bank(v, tv, te, beta, BH, H, T, d, causal, bw, ds->err, ds->num_sms, s);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
   if (e == cudaSuccess)
-    e = launch_tc(d, tq, tk, te, to, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, bw.tilefix, bw.fixups, lse, BH, H, T,
+    e = launch_tc(d, tq, tk, te, out, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, bw.tilefix, bw.fixups, lse, BH, H, T,
                   causal, ds->err, s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess) {

@@ -1,15 +1,16 @@
 // Value-bank pre-pass of the FEM read: statistics, shift schedule and the
 // fp16 value bank, written once per key tile for every query tile to share.
 //
-//   tile_stats  (B*H x key tiles)  max, min and sum of v_.j over each tile of
+//   tile_stats  (persistent)       max, min and sum of v_.j over each tile of
 //                                  128 keys (valid keys only)
-//   plan        (B*H)              per channel: bank mode and linear anchor
-//                                  from the whole sequence; the running maximum
-//                                  cpre[kt] = max over tiles 0..kt; the shifted
-//                                  bank's shift c[kt], raised lazily along cpre
-//                                  (only when beta*(cpre - c) > kShiftLag);
-//                                  a per-tile mask of the channels whose shift moved
-//   bank        (B*H x key tiles)  E = bank(v) in fp16 with the tile's shift;
+//   plan        (B*H x 32-channel  per channel: bank mode and linear anchor
+//                groups)           from the whole sequence; the running maximum
+//                                  over tiles 0..kt; the shifted bank's shift
+//                                  c[kt], raised lazily along it (only when
+//                                  beta*(max - c) > kShiftLag); a per-tile mask
+//                                  of the channels whose shift moved; the
+//                                  bank's coefficients for every tile
+//   bank        (persistent)       E = bank(v) in fp16 with the tile's shift;
 //                                  causal: the (row, 32-channel group) entries
 //                                  of the tile's diagonal rows whose visible
 //                                  maximum lies more than kHazardTilt/beta below
@@ -24,100 +25,141 @@
 
 namespace fem {
 
-// Thread layout shared by tile_stats and bank: 128 threads cover a [128 x D]
-// tile with 16-byte chunks; CPR chunks per row, RG row groups of RPG rows.
+// Ring of key tiles a persistent pre-pass block streams through shared
+// memory: kStages slots, one mbarrier each, filled by bulk copies that thread 0
+// issues kStages - 1 tiles ahead.  A block takes the tiles blockIdx.x,
+// blockIdx.x + gridDim.x, ... of the (b, h, key tile) list, key tile fastest.
+constexpr int kStages = 3;
+
+__device__ __forceinline__ int tiles_of_block(int n_tiles) {
+  return blockIdx.x < n_tiles ? (n_tiles - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1 : 0;
+}
+
+// ---------------------------------------------------------------------------
+// tile_stats: 128 threads; thread (cc, rg) reads 16-byte chunk cc of rows
+// rg*RPG .. rg*RPG + RPG - 1 of the tile (consecutive lanes read consecutive
+// chunks of a row), lanes holding the same chunk combine by shuffles, the four
+// warps through shared memory.  Tiles arrive as plain bulk copies of their
+// rows, which are contiguous in V.
+// ---------------------------------------------------------------------------
 template <int D>
-struct TileMap {
-  static constexpr int CPR = D / 8;
-  static constexpr int RG = 128 / CPR;
-  static constexpr int RPG = 128 / RG;
+struct StatsMap {
+  static constexpr int CPR = D / 8;        // chunks per row
+  static constexpr int RG = 128 / CPR;     // row groups
+  static constexpr int RPG = 128 / RG;     // rows per group
+  static constexpr int kTileBytes = kBlockK * D * 2;
 };
 
-// Both kernels stream the tile's rows (contiguous in V) into shared memory
-// with one bulk copy, which keeps the HBM reads in flight independently of the
-// threads' own load slots.
 template <int D>
-__device__ __forceinline__ bool stage_tile(const __nv_bfloat16 *v, int T, int bh, int kt, uint8_t *dst,
-                                           uint64_t *bar_word, unsigned *err) {
-  const uint32_t bar = smem_u32(bar_word);
-  const int rows = min(kBlockK, T - kt * kBlockK);
-  if (threadIdx.x == 0) {
-    mbar_init(bar, 1);
-    fence_mbar_init();
-    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(rows * D * 2));
-    bulk_load(smem_u32(dst), v + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D,
-              static_cast<uint32_t>(rows * D * 2), bar);
-  }
-  __syncthreads();
-  return mbar_wait(bar, 0, err, kErrWaitTma);
+__device__ __forceinline__ void stats_issue(const __nv_bfloat16 *v, int T, int n_kt, int g, uint32_t dst,
+                                            uint32_t bar) {
+  const int bh = g / n_kt, kt = g % n_kt;
+  const uint32_t bytes = static_cast<uint32_t>(min(kBlockK, T - kt * kBlockK) * D * 2);
+  mbar_arrive_expect_tx(bar, bytes);
+  bulk_load(dst, v + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D, bytes, bar);
 }
 
 template <int D>
-__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T,
-                                                          float4 *__restrict__ tstat, unsigned *__restrict__ err) {
-  using M = TileMap<D>;
-  extern __shared__ __align__(16) uint8_t tile_smem[];  // the tile's rows, [128][D] bf16
-  __shared__ __align__(8) uint64_t s_bar;
-  __shared__ float s_max[M::RG][D], s_min[M::RG][D], s_sum[M::RG][D];
-  const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x;
-  const int cc = threadIdx.x % M::CPR, rg = threadIdx.x / M::CPR;
-  if (!stage_tile<D>(v, T, bh, kt, tile_smem, &s_bar, err)) return;
-  float mx[8], mn[8], sm[8];
-#pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    mx[u] = -INFINITY;
-    mn[u] = INFINITY;
-    sm[u] = 0.f;
+__global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T, int n_kt,
+                                                          int n_tiles, float4 *__restrict__ tstat,
+                                                          unsigned *__restrict__ err) {
+  using M = StatsMap<D>;
+  extern __shared__ __align__(16) uint8_t ring[];  // kStages x [128][D] bf16
+  __shared__ __align__(8) uint64_t s_full[kStages];
+  __shared__ float s_part[2][3][4][D];  // [buffer][max, min, sum][warp][channel]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int cc = tid % M::CPR, rg = tid / M::CPR;
+  const int my_n = tiles_of_block(n_tiles);
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&s_full[s]), 1);
+    fence_mbar_init();
+    for (int i = 0; i < kStages && i < my_n; ++i)
+      stats_issue<D>(v, T, n_kt, blockIdx.x + i * gridDim.x, smem_u32(ring + i * M::kTileBytes),
+                     smem_u32(&s_full[i]));
   }
+  __syncthreads();
+  for (int i = 0; i < my_n; ++i) {
+    const int st = i % kStages, g = blockIdx.x + i * gridDim.x;
+    const int bh = g / n_kt, kt = g % n_kt, rows = min(kBlockK, T - kt * kBlockK);
+    if (!mbar_wait(smem_u32(&s_full[st]), (i / kStages) & 1, err, kErrWaitTma)) return;
+    const uint8_t *tile = ring + st * M::kTileBytes;
+    float mx[8], mn[8], sm[8];
 #pragma unroll
-  for (int i = 0; i < M::RPG; ++i) {
-    const int row = rg * M::RPG + i;
-    if (kt * kBlockK + row < T) {
-      const uint4 raw = *reinterpret_cast<const uint4 *>(tile_smem + (row * D + cc * 8) * 2);
-      const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
+    for (int u = 0; u < 8; ++u) {
+      mx[u] = -INFINITY;
+      mn[u] = INFINITY;
+      sm[u] = 0.f;
+    }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float2 f = __bfloat1622float2(p2[u]);
-        mx[2 * u] = fmaxf(mx[2 * u], f.x);
-        mx[2 * u + 1] = fmaxf(mx[2 * u + 1], f.y);
-        mn[2 * u] = fminf(mn[2 * u], f.x);
-        mn[2 * u + 1] = fminf(mn[2 * u + 1], f.y);
-        sm[2 * u] += f.x;
-        sm[2 * u + 1] += f.y;
+    for (int r = 0; r < M::RPG; ++r) {
+      const int row = rg * M::RPG + r;
+      if (row < rows) {
+        const uint4 raw = *reinterpret_cast<const uint4 *>(tile + (row * D + cc * 8) * 2);
+        const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float2 f = __bfloat1622float2(p2[u]);
+          mx[2 * u] = fmaxf(mx[2 * u], f.x);
+          mx[2 * u + 1] = fmaxf(mx[2 * u + 1], f.y);
+          mn[2 * u] = fminf(mn[2 * u], f.x);
+          mn[2 * u + 1] = fminf(mn[2 * u + 1], f.y);
+          sm[2 * u] += f.x;
+          sm[2 * u + 1] += f.y;
+        }
       }
     }
-  }
 #pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    s_max[rg][cc * 8 + u] = mx[u];
-    s_min[rg][cc * 8 + u] = mn[u];
-    s_sum[rg][cc * 8 + u] = sm[u];
-  }
-  __syncthreads();
-  for (int j = threadIdx.x; j < D; j += 128) {
-    float a = -INFINITY, b = INFINITY, c = 0.f;
-    for (int g = 0; g < M::RG; ++g) {
-      a = fmaxf(a, s_max[g][j]);
-      b = fminf(b, s_min[g][j]);
-      c += s_sum[g][j];
+    for (int off = M::CPR; off < 32; off <<= 1) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        mx[u] = fmaxf(mx[u], __shfl_xor_sync(0xffffffffu, mx[u], off));
+        mn[u] = fminf(mn[u], __shfl_xor_sync(0xffffffffu, mn[u], off));
+        sm[u] += __shfl_xor_sync(0xffffffffu, sm[u], off);
+      }
     }
-    tstat[(static_cast<size_t>(bh) * n_kt + kt) * D + j] = make_float4(a, b, c, 0.f);
+    const int buf = i & 1;
+    if (lane < M::CPR) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        s_part[buf][0][warp][cc * 8 + u] = mx[u];
+        s_part[buf][1][warp][cc * 8 + u] = mn[u];
+        s_part[buf][2][warp][cc * 8 + u] = sm[u];
+      }
+    }
+    __syncthreads();  // every read of the slot and every partial of this tile are done
+    if (tid == 0 && i + kStages < my_n)
+      stats_issue<D>(v, T, n_kt, blockIdx.x + (i + kStages) * gridDim.x, smem_u32(ring + st * M::kTileBytes),
+                     smem_u32(&s_full[st]));
+    for (int j = tid; j < D; j += 128) {
+      float a = s_part[buf][0][0][j], b = s_part[buf][1][0][j], c = s_part[buf][2][0][j];
+#pragma unroll
+      for (int w = 1; w < 4; ++w) {
+        a = fmaxf(a, s_part[buf][0][w][j]);
+        b = fminf(b, s_part[buf][1][w][j]);
+        c += s_part[buf][2][w][j];
+      }
+      tstat[(static_cast<size_t>(bh) * n_kt + kt) * D + j] = make_float4(a, b, c, 0.f);
+    }
   }
 }
 
-// Plan of one (b, h) per block: four threads per channel, each holding a
-// quarter of a window of 64 key tiles in registers, so every load of a window
-// is in flight at once.  The lazy shift is a sequential recurrence over tiles:
-// the four quarters run it in turn, handing the running (max, shift) on by
-// warp shuffles.
+// ---------------------------------------------------------------------------
+// plan: one block per (b, h) and group of 32 channels, four threads per
+// channel, each holding a quarter of a window of 64 key tiles in registers so
+// every load of a window is in flight at once.  The lazy shift is a sequential
+// recurrence over tiles: the four quarters run it in turn, handing the running
+// (max, shift) on by warp shuffles.  Besides the schedule it writes the bank's
+// per-tile coefficients (BankCoef) and the moved-channel word of its group.
+// ---------------------------------------------------------------------------
 template <int D>
-__global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta,
-                                                     int H, int T, int n_kt, ChanInfo *__restrict__ chan,
-                                                     float *__restrict__ cpre, float *__restrict__ shift,
-                                                     float *__restrict__ rfac, unsigned *__restrict__ colmask) {
+__global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta,
+                                                   int H, int T, int n_kt, int causal, ChanInfo *__restrict__ chan,
+                                                   float *__restrict__ shift, float *__restrict__ rfac,
+                                                   unsigned *__restrict__ colmask, float4 *__restrict__ bcoef) {
   constexpr int kParts = 4, kPer = 16, kWin = kParts * kPer;
-  __shared__ unsigned s_mask[kWin][4];
-  const int tid = threadIdx.x, j = tid / kParts, part = tid % kParts, lane = tid & 31;
+  __shared__ unsigned s_mask[kWin];
+  const int tid = threadIdx.x, part = tid % kParts, lane = tid & 31;
+  const int grp = blockIdx.y, j = grp * 32 + tid / kParts;
   const int bh = blockIdx.x, h = bh % H;
   const float b = beta[h * D + j];
   const float4 *ts = tstat + static_cast<size_t>(bh) * n_kt * D + j;
@@ -165,7 +207,7 @@ __global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ 
       const int kt = w0 + part * kPer + u;
       tmx[u] = kt < n_kt ? ts[static_cast<size_t>(kt) * D].x : -INFINITY;
     }
-    for (int i = tid; i < kWin * 4; i += kParts * D) s_mask[i / 4][i % 4] = 0u;
+    for (int i = tid; i < kWin; i += 128) s_mask[i] = 0u;
     __syncthreads();
     for (int stage = 0; stage < kParts; ++stage) {
       if (part == stage) {
@@ -173,6 +215,7 @@ __global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ 
         for (int u = 0; u < kPer; ++u) {
           const int kt = w0 + stage * kPer + u;
           if (kt < n_kt) {
+            const float cp_prev = cp;
             cp = fmaxf(cp, tmx[u]);
             const float prev = cl;
             if (lin) {
@@ -181,11 +224,23 @@ __global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ 
               cl = cp;
             }
             const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
-            cpre[o] = cp;
             shift[o] = cl;
             const bool moved = !lin && kt > 0 && cl != prev;
             rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
-            if (moved) atomicOr(&s_mask[stage * kPer + u][j >> 5], 1u << (j & 31));
+            if (moved) atomicOr(&s_mask[stage * kPer + u], 1u << (j & 31));
+            // Diagonal hazard of a shifted channel: a row of the tile is safe
+            // once its visible maximum reaches cl - kHazardTilt/beta, so the
+            // bank checks the tile's keys against that level unless an earlier
+            // tile already reached it.
+            float4 bc;
+            if (lin) {
+              bc = make_float4(b > 0.f ? 1.f / b : 0.f, b, cl, __int_as_float(0x7fc00000));
+            } else {
+              const float thr = cl - kHazardTilt / b;
+              const bool check = causal && !(kt > 0 && cp_prev >= thr);
+              bc = make_float4(b * kLog2e, (kBankOffset - b * cl) * kLog2e, cl, check ? thr : -INFINITY);
+            }
+            bcoef[o] = bc;
           }
         }
       }
@@ -194,191 +249,242 @@ __global__ void __launch_bounds__(4 * D) plan_kernel(const float4 *__restrict__ 
       cl = __shfl_sync(0xffffffffu, cl, (lane & ~(kParts - 1)) | stage);
     }
     __syncthreads();
-    for (int i = tid; i < kWin * 4; i += kParts * D) {
-      const int kt = w0 + i / 4;
-      if (kt < n_kt) colmask[(static_cast<size_t>(bh) * n_kt + kt) * 4 + i % 4] = s_mask[i / 4][i % 4];
+    for (int i = tid; i < kWin; i += 128) {
+      const int kt = w0 + i;
+      if (kt < n_kt) {
+        unsigned *cm = colmask + (static_cast<size_t>(bh) * n_kt + kt) * 4;
+        cm[grp] = s_mask[i];
+        if (grp == 0)
+          for (int gz = D / 32; gz < 4; ++gz) cm[gz] = 0u;
+      }
     }
     __syncthreads();
   }
 }
 
+// ---------------------------------------------------------------------------
+// bank: 256 threads.  A slot holds the tile of V as D/64 boxes of 64 channels
+// x 128 rows with the 128-byte swizzle (the layout the tensor-core kernel
+// reads the bank in) and the tile's BankCoef.  Warp w owns the 16-byte chunks
+// (8 channels) w*CPW .. w*CPW + CPW - 1; lane l handles rows l, 32 + l, 64 + l,
+// 96 + l of a chunk, so each channel's form (linear or shifted) and hazard
+// check are uniform across the warp.  The bank overwrites V in the slot and
+// leaves with one TMA store per box.
+// ---------------------------------------------------------------------------
 template <int D>
-__global__ void __launch_bounds__(128, 3) bank_kernel(const __nv_bfloat16 *__restrict__ v,
-                                                    const float *__restrict__ beta, const ChanInfo *__restrict__ chan,
-                                                    const float *__restrict__ cpre, const float *__restrict__ shift,
-                                                    int H, int T, int causal, __half *__restrict__ bank,
-                                                    FixupEntry *__restrict__ fixups, int *__restrict__ fixup_count,
-                                                    int *__restrict__ fixup_rows, int2 *__restrict__ tilefix,
-                                                    unsigned *__restrict__ err) {
-  using M = TileMap<D>;
-  extern __shared__ __align__(16) uint8_t tile_smem[];  // the tile's rows of V, then of the bank, in place
-  __shared__ __align__(8) uint64_t s_bar;
-  __shared__ float s_a[D], s_b[D], s_c[D], s_lin[D], s_thr[D];
-  __shared__ int s_first[D];
-  const int kt = blockIdx.x, bh = blockIdx.y, n_kt = gridDim.x, h = bh % H;
-  const int tid = threadIdx.x;
-  const int cc = tid % M::CPR, rg = tid / M::CPR;
-  for (int j = tid; j < D; j += 128) {
-    const float b = beta[h * D + j];
-    const ChanInfo ci = chan[bh * D + j];
-    const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
-    const float c = shift[o];
-    s_lin[j] = ci.linear;
-    s_c[j] = c;
-    if (ci.linear != 0.f) {
-      s_a[j] = b > 0.f ? 1.f / b : 0.f;  // linear bank: 1/beta and beta
-      s_b[j] = b;
-    } else {
-      s_a[j] = b * kLog2e;  // shifted bank: E = ex2(a v + b)
-      s_b[j] = (kBankOffset - b * c) * kLog2e;
-    }
-    // Diagonal hazard of a shifted channel: a row of this tile is safe once its
-    // visible maximum reaches c - kHazardTilt/beta, i.e. from the first key at
-    // or above that threshold on (row 0 when an earlier tile already reached it).
-    const float thr = c - kHazardTilt / b;
-    const bool haz = causal && ci.linear == 0.f;
-    s_thr[j] = haz ? thr : -INFINITY;
-    s_first[j] = (!haz || (kt > 0 && cpre[o - D] >= thr)) ? 0 : kBlockK;
-  }
-  __syncthreads();
+struct BankMap {
+  static constexpr int kBoxes = D / 64;
+  static constexpr int kTileBytes = kBlockK * D * 2;
+  static constexpr int kSlotBytes = kTileBytes + D * 16;  // tile, then D BankCoef
+  static constexpr int CPW = D / 64;                      // chunks per warp
+  static constexpr int kSmem = kStages * kSlotBytes + 1024;
+};
 
-  if (!stage_tile<D>(v, T, bh, kt, tile_smem, &s_bar, err)) return;
-  // Thread: the 8 channels of chunk column cc, rows rg*RPG .. rg*RPG+RPG-1,
-  // each 16-byte chunk of V replaced by the chunk of the bank.  Both bank
-  // forms are evaluated and one is selected, so lanes never diverge.
-  const int rows = min(kBlockK, T - kt * kBlockK);
-  float pa[8], pb[8], pc[8], pthr[8];
-  bool plin[8];
-  int first[8];
+template <int D>
+__device__ __forceinline__ void bank_issue(const CUtensorMap *tv, const float4 *bcoef, int n_kt, int g, uint32_t slot,
+                                           uint32_t bar) {
+  using M = BankMap<D>;
+  const int bh = g / n_kt, kt = g % n_kt;
+  mbar_arrive_expect_tx(bar, static_cast<uint32_t>(M::kSlotBytes));
 #pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    const int j = cc * 8 + u;
-    pa[u] = s_a[j];
-    pb[u] = s_b[j];
-    pc[u] = s_c[j];
-    pthr[u] = s_thr[j];
-    plin[u] = s_lin[j] != 0.f;
-    first[u] = kBlockK;
-  }
-#pragma unroll 2
-  for (int i = 0; i < M::RPG; ++i) {
-    {
-      const int row = rg * M::RPG + i;
-      if (row >= rows) break;
-      uint4 *cell = reinterpret_cast<uint4 *>(tile_smem + (row * D + cc * 8) * 2);
-      const uint4 raw = *cell;
-      const __nv_bfloat16 *vin = reinterpret_cast<const __nv_bfloat16 *>(&raw);
-      __align__(16) __half e[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float x = __bfloat162float(vin[u]);
-        if (x >= pthr[u]) first[u] = min(first[u], row);
-        // linear bank: D = expm1(y)/beta, y = beta (v - c) >= -1, as a Taylor
-        // series of expm1(y)/y for |y| < 1/2 (truncation < 4e-6 relative),
-        // e^y - 1 beyond; shifted bank: E = 2^(a v + b)
-        const float xs = x - pc[u];
-        const float y = pb[u] * xs;
-        float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
-        poly = fmaf(y, poly, 1.f / 24.f);
-        poly = fmaf(y, poly, 1.f / 6.f);
-        poly = fmaf(y, poly, 0.5f);
-        poly = fmaf(y, poly, 1.f);
-        const float lin = fabsf(y) < 0.5f ? xs * poly : (ex2_approx(y * kLog2e) - 1.f) * pa[u];
-        const float shf = ex2_approx(fmaf(pa[u], x, pb[u]));
-        e[u] = __float2half_rn(plin[u] ? lin : shf);
-      }
-      *cell = *reinterpret_cast<const uint4 *>(e);
-    }
-  }
-  // the tile of the bank leaves with one bulk store
-  fence_proxy_async_smem();
-  __syncthreads();
-  if (tid == 0) {
-    bulk_store(bank + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D, smem_u32(tile_smem),
-               static_cast<uint32_t>(rows * D * 2));
-    bulk_commit_group();
-  }
-  if (causal) {
-#pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (first[u] < kBlockK) atomicMin(&s_first[cc * 8 + u], first[u]);
-  }
-  if (!causal) {
-    if (tid == 0) bulk_wait_group_read0();
-    return;
-  }
-  __syncthreads();
-  // rows r < max_j first_j of this tile get one entry with their channel masks
-  __shared__ int s_rows;
-  if (tid == 0) {
-    int hz_max = 0;
-    for (int j = 0; j < D; ++j) hz_max = max(hz_max, s_first[j]);
-    s_rows = min(hz_max, T - kt * kBlockQ);
-  }
-  __syncthreads();
-  const int n_rows = s_rows;
-  int2 *tf = tilefix + static_cast<size_t>(bh) * n_kt + kt;
-  if (n_rows <= 0) {
-    if (tid == 0) {
-      *tf = make_int2(0, 0);
-      bulk_wait_group_read0();
-    }
-    return;
-  }
-  // the tile's entries take a multiple of 8 slots (padding rows -1), so the
-  // fix-up's 8-entry chunks never straddle two tiles
-  const int n_slots = (n_rows + 7) & ~7;
-  __shared__ int s_base;
-  if (tid == 0) {
-    s_base = atomicAdd(fixup_count, n_slots);
-    atomicAdd(fixup_rows, n_rows);
-    *tf = make_int2(s_base, n_rows);
-  }
-  __syncthreads();
-  for (int r = tid; r < n_slots; r += 128) {
-    FixupEntry e;
-    e.row = r < n_rows ? bh * T + kt * kBlockQ + r : -1;
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      unsigned m = 0;
-      for (int c = 0; c < 32; ++c) {
-        const int j = 32 * g + c;
-        if (j < D && r < n_rows && s_first[j] > r) m |= 1u << c;
-      }
-      e.mask[g] = m;
-    }
-    e.m_pre = -INFINITY;
-    e.l_pre = 0.f;
-    e.pad = 0;
-    fixups[s_base + r] = e;
-  }
-  if (tid == 0) bulk_wait_group_read0();
+  for (int bx = 0; bx < M::kBoxes; ++bx) tma_load_3d(slot + bx * 16384, tv, bar, bx * 64, kt * kBlockK, bh);
+  bulk_load(slot + M::kTileBytes, bcoef + static_cast<size_t>(g) * D, D * 16, bar);
 }
 
-cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
-                              const BankWorkspace &w, unsigned *err, cudaStream_t stream) {
-  const int n_kt = (T + kBlockK - 1) / kBlockK;
-  const dim3 grid(n_kt, BH);
+template <int D>
+__global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CUtensorMap tv,
+                                                       const __grid_constant__ CUtensorMap te,
+                                                       const float4 *__restrict__ bcoef, int T, int n_kt,
+                                                       int n_tiles, int causal, FixupEntry *__restrict__ fixups,
+                                                       int *__restrict__ fixup_count, int *__restrict__ fixup_rows,
+                                                       int2 *__restrict__ tilefix, unsigned *__restrict__ err) {
+  using M = BankMap<D>;
+  extern __shared__ uint8_t bank_smem[];
+  __shared__ __align__(8) uint64_t s_full[kStages];
+  __shared__ int s_first[2][D];  // first row of the tile at or above the channel's hazard level
+  __shared__ int s_wmax[2][8];
+  __shared__ int s_base;
+  const uint32_t base_addr = (smem_u32(bank_smem) + 1023u) & ~1023u;  // 128-byte swizzle wants 1024-B alignment
+  uint8_t *const ring = bank_smem + (base_addr - smem_u32(bank_smem));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int my_n = tiles_of_block(n_tiles);
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&s_full[s]), 1);
+    fence_mbar_init();
+    for (int i = 0; i < kStages - 1 && i < my_n; ++i)
+      bank_issue<D>(&tv, bcoef, n_kt, blockIdx.x + i * gridDim.x, base_addr + i * M::kSlotBytes,
+                    smem_u32(&s_full[i]));
+  }
+  __syncthreads();
+  for (int i = 0; i < my_n; ++i) {
+    const int st = i % kStages, g = blockIdx.x + i * gridDim.x, buf = i & 1;
+    const int bh = g / n_kt, kt = g % n_kt, rows = min(kBlockK, T - kt * kBlockK);
+    if (!mbar_wait(smem_u32(&s_full[st]), (i / kStages) & 1, err, kErrWaitTma)) {
+      if (tid == 0) bulk_wait_group_read0();
+      return;
+    }
+    uint8_t *const tile = ring + st * M::kSlotBytes;
+    const float4 *const coef = reinterpret_cast<const float4 *>(tile + M::kTileBytes);
+    int wmax = 0;
+#pragma unroll
+    for (int q = 0; q < M::CPW; ++q) {
+      const int ch = warp * M::CPW + q;  // chunk: channels 8 ch .. 8 ch + 7
+      uint8_t *cell[4];
+      uint4 raw[4];
+#pragma unroll
+      for (int rb = 0; rb < 4; ++rb) {
+        const int row = rb * 32 + lane;
+        cell[rb] = tile + (ch >> 3) * 16384 + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
+        raw[rb] = *reinterpret_cast<const uint4 *>(cell[rb]);
+      }
+      float res[4][8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float4 cf = coef[ch * 8 + u];  // {a, b, c, hazard level}; level NaN: linear bank
+        float x[4];
+#pragma unroll
+        for (int rb = 0; rb < 4; ++rb) {
+          const uint32_t w = reinterpret_cast<const uint32_t *>(&raw[rb])[u >> 1];
+          x[rb] = __uint_as_float((u & 1) ? (w & 0xffff0000u) : (w << 16));
+        }
+        if (cf.w != cf.w) {
+          // linear bank: D = expm1(y)/beta, y = beta (v - c) >= -1 (a = 1/beta,
+          // b = beta), as a Taylor series of expm1(y)/y for |y| < 1/2
+          // (truncation < 4e-6 relative), e^y - 1 beyond
+#pragma unroll
+          for (int rb = 0; rb < 4; ++rb) {
+            const float xs = x[rb] - cf.z;
+            const float y = cf.y * xs;
+            float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
+            poly = fmaf(y, poly, 1.f / 24.f);
+            poly = fmaf(y, poly, 1.f / 6.f);
+            poly = fmaf(y, poly, 0.5f);
+            poly = fmaf(y, poly, 1.f);
+            res[rb][u] = fabsf(y) < 0.5f ? xs * poly : (ex2_approx(y * kLog2e) - 1.f) * cf.x;
+          }
+        } else {
+          // shifted bank: E = 2^(a v + b)
+#pragma unroll
+          for (int rb = 0; rb < 4; ++rb) res[rb][u] = ex2_approx(fmaf(cf.x, x[rb], cf.y));
+        }
+        int first = 0;
+        if (cf.w > -INFINITY) {  // hazard check of a shifted channel
+          first = kBlockK;
+#pragma unroll
+          for (int rb = 0; rb < 4; ++rb) {
+            const unsigned hit = __ballot_sync(0xffffffffu, x[rb] >= cf.w && rb * 32 + lane < rows);
+            if (hit && first == kBlockK) first = rb * 32 + __ffs(hit) - 1;
+          }
+        }
+        if (lane == 0) s_first[buf][ch * 8 + u] = first;
+        wmax = max(wmax, first);
+      }
+#pragma unroll
+      for (int rb = 0; rb < 4; ++rb) {
+        uint4 o;
+        uint32_t *ow = reinterpret_cast<uint32_t *>(&o);
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const __half2 h2 = __floats2half2_rn(res[rb][2 * p], res[rb][2 * p + 1]);
+          ow[p] = *reinterpret_cast<const uint32_t *>(&h2);
+        }
+        *reinterpret_cast<uint4 *>(cell[rb]) = o;
+      }
+    }
+    if (lane == 0) s_wmax[buf][warp] = wmax;
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+#pragma unroll
+      for (int bx = 0; bx < M::kBoxes; ++bx) tma_store_3d(&te, base_addr + st * M::kSlotBytes + bx * 16384, bx * 64,
+                                                          kt * kBlockK, bh);
+      bulk_commit_group();
+      // the slot refilled next was last read by the previous tile's store
+      bulk_wait_group_read<1>();
+      if (i + kStages - 1 < my_n) {
+        const int sn = (i + kStages - 1) % kStages;
+        bank_issue<D>(&tv, bcoef, n_kt, blockIdx.x + (i + kStages - 1) * gridDim.x,
+                      base_addr + sn * M::kSlotBytes, smem_u32(&s_full[sn]));
+      }
+    }
+    if (!causal) continue;
+    // rows r < max_j first_j of this tile get one entry with their channel masks
+    int hz_max = 0;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) hz_max = max(hz_max, s_wmax[buf][w]);
+    const int n_rows = min(hz_max, rows);
+    int2 *tf = tilefix + g;
+    if (n_rows <= 0) {
+      if (tid == 0) *tf = make_int2(0, 0);
+      continue;
+    }
+    // the tile's entries take a multiple of 8 slots (padding rows -1), so the
+    // fix-up's 8-entry chunks never straddle two tiles
+    const int n_slots = (n_rows + 7) & ~7;
+    if (tid == 0) {
+      s_base = atomicAdd(fixup_count, n_slots);
+      atomicAdd(fixup_rows, n_rows);
+      *tf = make_int2(s_base, n_rows);
+    }
+    __syncthreads();
+    const int fbase = s_base;
+    for (int r = tid; r < n_slots; r += 256) {
+      FixupEntry e;
+      e.row = r < n_rows ? bh * T + kt * kBlockQ + r : -1;
+#pragma unroll
+      for (int gq = 0; gq < 4; ++gq) {
+        unsigned m = 0;
+        for (int c = 0; c < 32; ++c) {
+          const int j = 32 * gq + c;
+          if (j < D && r < n_rows && s_first[buf][j] > r) m |= 1u << c;
+        }
+        e.mask[gq] = m;
+      }
+      e.m_pre = -INFINITY;
+      e.l_pre = 0.f;
+      e.pad = 0;
+      fixups[fbase + r] = e;
+    }
+  }
+  if (tid == 0) bulk_wait_group_read<0>();
+}
+
+cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtensorMap &te, const float *beta, int BH,
+                              int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
+                              cudaStream_t stream) {
+  const int n_kt = (T + kBlockK - 1) / kBlockK, n_tiles = BH * n_kt;
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
+  const int grid = min(n_tiles, 2 * num_sms);
+  cudaError_t e = cudaSuccess;
   if (d == 64) {
-    tile_stats_kernel<64><<<grid, 128, kBlockK * 64 * 2, stream>>>(vb, T, w.tstat, err);
-    plan_kernel<64><<<BH, 4 * 64, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.cpre, w.shift, w.rfac, w.colmask);
+    using SM = StatsMap<64>;
+    using BM = BankMap<64>;
+    e = cudaFuncSetAttribute(tile_stats_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kStages * SM::kTileBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(bank_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
+    if (e != cudaSuccess) return e;
+    tile_stats_kernel<64><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
+    plan_kernel<64><<<dim3(BH, 2), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, causal, w.chan, w.shift, w.rfac,
+                                                     w.colmask, w.bcoef);
+    bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, causal, w.fixups,
+                                                      w.fixup_count, w.fixup_rows, w.tilefix, err);
   } else if (d == 128) {
-    tile_stats_kernel<128><<<grid, 128, kBlockK * 128 * 2, stream>>>(vb, T, w.tstat, err);
-    plan_kernel<128><<<BH, 4 * 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.cpre, w.shift, w.rfac,
-                                                 w.colmask);
+    using SM = StatsMap<128>;
+    using BM = BankMap<128>;
+    e = cudaFuncSetAttribute(tile_stats_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kStages * SM::kTileBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(bank_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
+    if (e != cudaSuccess) return e;
+    tile_stats_kernel<128><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
+    plan_kernel<128><<<dim3(BH, 4), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, causal, w.chan, w.shift, w.rfac,
+                                                      w.colmask, w.bcoef);
+    bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, causal, w.fixups,
+                                                       w.fixup_count, w.fixup_rows, w.tilefix, err);
   } else {
     return cudaErrorInvalidValue;
   }
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  if (d == 64)
-    bank_kernel<64><<<grid, 128, kBlockK * 64 * 2, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal, w.bank,
-                                                             w.fixups, w.fixup_count, w.fixup_rows, w.tilefix, err);
-  else
-    bank_kernel<128><<<grid, 128, kBlockK * 128 * 2, stream>>>(vb, beta, w.chan, w.cpre, w.shift, H, T, causal,
-                                                               w.bank, w.fixups, w.fixup_count, w.fixup_rows,
-                                                               w.tilefix, err);
   return cudaGetLastError();
 }
 

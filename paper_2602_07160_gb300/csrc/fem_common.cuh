@@ -157,9 +157,6 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
   return done != 0;
 }
 
-// Per-warpgroup register budget (every thread of the warpgroup executes it).
-__device__ __forceinline__ void setmaxnreg_dec56() { asm volatile("setmaxnreg.dec.sync.aligned.u32 56;"); }
-__device__ __forceinline__ void setmaxnreg_inc256() { asm volatile("setmaxnreg.inc.sync.aligned.u32 256;"); }
 
 // Waits for the phase with the given parity to complete.  Gives up after
 // kWaitLimitNs, records `code` in the error word and returns false.
@@ -222,6 +219,11 @@ __device__ __forceinline__ void bulk_commit_group() { asm volatile("cp.async.bul
 // Waits until every committed bulk store has finished reading shared memory.
 __device__ __forceinline__ void bulk_wait_group_read0() {
   asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// Wait until at most N committed bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_group_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
 }
 
 // Named barrier over `nthreads` threads that returns the AND of `v` over them.

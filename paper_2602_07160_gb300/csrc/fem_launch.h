@@ -12,7 +12,7 @@ namespace fem {
 struct BankWorkspace {
   float4 *tstat;            // [B*H, key tiles, d]: max, min, sum of v per tile
   ChanInfo *chan;           // [B*H, d]
-  float *cpre;              // [B*H, key tiles, d]: running maximum of v
+  float4 *bcoef;            // [B*H, key tiles, d]: the bank's coefficients for the tile (BankCoef)
   float *shift;             // [B*H, key tiles, d]: the bank's shift for each tile
   float *rfac;              // [B*H, key tiles, d]: exp(beta (shift[kt-1] - shift[kt])), 1 if unmoved
   unsigned *colmask;        // [B*H, key tiles, 4]: bit j set when channel j's shift moved at the tile
@@ -25,15 +25,25 @@ struct BankWorkspace {
 };
 
 // Statistics, plan and value bank (two reads of V, one write of the bank).
-cudaError_t launch_value_bank(const void *v, const float *beta, int BH, int H, int T, int d, int causal,
-                              const BankWorkspace &w, unsigned *err, cudaStream_t stream);
+// `tv` and `te` map V (bf16) and the bank (fp16) like the tensor-core kernel's
+// operands: boxes of 64 channels x 128 rows, 128-byte swizzle.
+//
+// BankCoef, one float4 per (b, h, key tile, channel), written by the plan:
+//   linear bank   {1/beta (0 at beta = 0), beta, c_lin, NaN}
+//   shifted bank  {beta log2 e, (kBankOffset - beta c) log2 e, c, level}
+// with level = c - kHazardTilt/beta when the tile's keys are checked for the
+// causal diagonal hazard, -inf when not (not causal, or the running maximum
+// before the tile already reached it).
+cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtensorMap &te, const float *beta, int BH,
+                              int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
+                              cudaStream_t stream);
 
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
-// `to` maps the fp32 output [B*H, T, d] for the kernel's TMA stores.  For the
+// `out` is the fp32 output [B*H, T, d], 16-byte aligned.  For the
 // rows of a causal diagonal tile that have fix-up entries the kernel writes,
 // in place of the listed channels' outputs, their accumulator before the
 // diagonal tile, and the row's (max, sum) before it into the entry.
-cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const CUtensorMap &to,
+cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, float *out,
                       const float *beta, const ChanInfo *chan, const float *shift, const float *rfac,
                       const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H,
                       int T, int causal, unsigned *err, cudaStream_t stream);

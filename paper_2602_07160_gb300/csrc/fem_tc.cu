@@ -113,7 +113,7 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
 template <int D>
 __global__ void __launch_bounds__(384, 1)
     fem_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                  const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_o,
+                  const __grid_constant__ CUtensorMap tmap_e, float *__restrict__ out,
                   const float *__restrict__ beta,
                   const ChanInfo *__restrict__ chan, const float *__restrict__ shift,
                   const float *__restrict__ rfac, const unsigned *__restrict__ colmask,
@@ -224,10 +224,10 @@ __global__ void __launch_bounds__(384, 1)
   tc_fence_after_sync();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem + Lay::kTmemSlot);
 
+  // Every warp keeps the launch's register count: moving registers from the
+  // producer warps to the softmax (setmaxnreg) made the compiled code spill
+  // more and ran slower.
   if (wg == 0) {
-  // registers move from this warpgroup to the softmax, which holds a
-  // 128-float score row per thread
-  setmaxnreg_dec56();
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA: Q and K
     if (lane == 0) {
@@ -322,7 +322,6 @@ __global__ void __launch_bounds__(384, 1)
     float m_row = -INFINITY, L_row = 0.f;
     bool ok = true;
     if (is_sm) {
-      setmaxnreg_inc256();
       // ------------------------------------------------------------ softmax
       const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
       for (int kt = 0; kt < nk; ++kt) {
@@ -482,9 +481,11 @@ __global__ void __launch_bounds__(384, 1)
         mbar_arrive(FEM_BAR(kBarPFull + b));
       }
     }
-    // ---- epilogue, half the columns per warpgroup: o staged in shared memory
-    // (the K ring is idle once every contraction completed) in the output
-    // map's swizzled boxes, then TMA stores
+    // ---- epilogue, half the columns per warpgroup.  acc/L is staged in
+    // shared memory (the K ring is idle once every contraction completed) as
+    // 32-column boxes, row r by thread r; the transform then runs
+    // column-parallel and writes each row's 32 columns of a box as one
+    // coalesced 128-byte store.
     if (ok) ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAccDone), 0, err, kErrWaitMma, abort_flag));
     ok = bar_and(1, 256, ok);  // both warpgroups went through every key tile
     if (ok) {
@@ -492,13 +493,13 @@ __global__ void __launch_bounds__(384, 1)
       const float invL = s_invL[r];
       constexpr int NC = D / 64;  // 32-column chunks of this warpgroup
       const int c_lo = is_sm ? 0 : NC;
+      // (row, chunk) masks of the channels a fix-up row lists, in the idle
+      // part of the K ring behind the staging boxes
+      unsigned *s_hzm = reinterpret_cast<unsigned *>(smem + Lay::kK + (D / 32) * 16384);
       uint32_t v[NC][32];
 #pragma unroll
       for (int c = 0; c < NC; ++c) tmem_ld32(tAcc + (c_lo + c) * 32, v[c]);
       tmem_ld_wait();
-      // acc/L goes to the staging boxes first; the transform then runs as a
-      // rolled loop in place (this code runs once per tile and would otherwise
-      // be fetched cold, instruction by instruction)
 #pragma unroll
       for (int c = 0; c < NC; ++c) {
         uint8_t *box = smem + Lay::kK + (c_lo + c) * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
@@ -508,29 +509,9 @@ __global__ void __launch_bounds__(384, 1)
               make_float4(__uint_as_float(v[c][4 * i4]) * invL, __uint_as_float(v[c][4 * i4 + 1]) * invL,
                           __uint_as_float(v[c][4 * i4 + 2]) * invL, __uint_as_float(v[c][4 * i4 + 3]) * invL);
       }
-#pragma unroll 1
-      for (int ci = 0; ci < NC * 8; ++ci) {
-        const int c = c_lo + (ci >> 3), i4 = ci & 7;
-        float4 *cell = reinterpret_cast<float4 *>(smem + Lay::kK + c * 16384 + sw128_offset(r, i4));
-        const float4 a4 = *cell;
-        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
-        float o4[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          // shifted bank: c + (log a - kappa)/beta = lg2(a) ln2/beta + (c - kappa/beta);
-          // linear bank: c + log1p(x)/beta with x = beta a, as lg2(1 + x) ln2/beta + c,
-          // or, for |x| < 2^-6 (also beta = 0), as c + a times the series of log1p(x)/x
-          const float4 cf = c_coef[c * 32 + i4 * 4 + u];
-          const float a = av[u];
-          const float x = cf.x * a;
-          const float lg = fmaf(lg2_approx(cf.w != 0.f ? a : 1.f + x), cf.z, cf.y);
-          const float se = fmaf(a, fmaf(x, fmaf(x, fmaf(x, fmaf(x, 0.2f, -0.25f), 1.f / 3.f), -0.5f), 1.f), cf.y);
-          o4[u] = (cf.w == 0.f && fabsf(x) < 0.015625f) ? se : lg;
-        }
-        *cell = make_float4(o4[0], o4[1], o4[2], o4[3]);
-      }
       if (hz_warp) {
-        // listed channels of fix-up rows: the accumulator before the diagonal tile
+        // listed channels of fix-up rows: the accumulator before the diagonal
+        // tile, staged in place of acc/L and written out untransformed
 #pragma unroll 1
         for (int c = c_lo; c < c_lo + NC; ++c) {
           uint32_t w[32];
@@ -539,6 +520,7 @@ __global__ void __launch_bounds__(384, 1)
             tmem_ld_wait();
           }
           const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
+          s_hzm[r * 4 + c] = mc;
           uint8_t *box = smem + Lay::kK + c * 16384;
 #pragma unroll
           for (int i = 0; i < 32; ++i)
@@ -546,14 +528,60 @@ __global__ void __launch_bounds__(384, 1)
               reinterpret_cast<float *>(box + sw128_offset(r, i >> 2))[i & 3] = qt > 0 ? __uint_as_float(w[i]) : 0.f;
         }
       }
-      // the boxes are complete once all 128 rows are in: one thread stores them
-      fence_proxy_async_smem();
       bar_sync(is_sm ? 2 : 3, 128);
-      if (r == 0) {
-        for (int c = c_lo; c < c_lo + NC; ++c)
-          tma_store_3d(&tmap_o, sbase + Lay::kK + c * 16384, c * 32, qt * kBlockQ, bh);
-        bulk_commit_group();
-        bulk_wait_group_read0();  // shared memory stays valid until the stores have read it
+      // Thread r takes column r % 32 of a chunk and rows r / 32 + 4k, so its
+      // channel's coefficients stay in registers, each warp access is one
+      // 128-byte row of the box, and 8 loads at a time are in flight before the math.
+      //   shifted bank: c + (log a - kappa)/beta = lg2(a) ln2/beta + (c - kappa/beta)
+      //   linear bank:  c + log1p(x)/beta with x = beta a, as lg2(1 + x) ln2/beta + c,
+      //                 or, for |x| < 2^-6 (also beta = 0), as c + a times the
+      //                 series of log1p(x)/x
+      const int col = r & 31, row0 = r >> 5;
+      const int rows_left = T - qt * kBlockQ;
+      float *out_tile = out + (static_cast<size_t>(bh) * T + static_cast<size_t>(qt) * kBlockQ) * D + col;
+#pragma unroll 1
+      for (int c = c_lo; c < c_lo + NC; ++c) {
+        const float4 cf = c_coef[c * 32 + col];
+        const bool lin = cf.w == 0.f;
+        // pairs of rows go through the packed fp32x2 pipe; the lg2 argument is
+        // a (shifted) or 1 + beta a (linear)
+        const float2 bx2 = make_float2(cf.x, cf.x), y2 = make_float2(cf.y, cf.y), z2 = make_float2(cf.z, cf.z);
+        const float2 s12 = lin ? bx2 : make_float2(1.f, 1.f), s02 = make_float2(lin ? 1.f : 0.f, lin ? 1.f : 0.f);
+        const uint8_t *box = smem + Lay::kK + c * 16384 + ((col & 3) << 2);
+#pragma unroll 1
+        for (int k0 = 0; k0 < 32; k0 += 8) {
+          float a[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            a[k] = *reinterpret_cast<const float *>(box + sw128_offset(row0 + 4 * (k0 + k), col >> 2));
+          float o[8];
+#pragma unroll
+          for (int k = 0; k < 8; k += 2) {
+            const float2 a2 = make_float2(a[k], a[k + 1]);
+            const float2 x2 = __fmul2_rn(bx2, a2);
+            const float2 g2 = __ffma2_rn(a2, s12, s02);
+            const float2 lg = __ffma2_rn(make_float2(lg2_approx(g2.x), lg2_approx(g2.y)), z2, y2);
+            float2 q = __ffma2_rn(x2, make_float2(0.2f, 0.2f), make_float2(-0.25f, -0.25f));
+            q = __ffma2_rn(x2, q, make_float2(1.f / 3.f, 1.f / 3.f));
+            q = __ffma2_rn(x2, q, make_float2(-0.5f, -0.5f));
+            q = __ffma2_rn(x2, q, make_float2(1.f, 1.f));
+            const float2 se = __ffma2_rn(a2, q, y2);
+            o[k] = (lin && fabsf(x2.x) < 0.015625f) ? se.x : lg.x;
+            o[k + 1] = (lin && fabsf(x2.y) < 0.015625f) ? se.y : lg.y;
+          }
+          if (hz_rows > 0) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const int row = row0 + 4 * (k0 + k);
+              if (row < hz_rows && ((s_hzm[row * 4 + c] >> col) & 1u)) o[k] = a[k];
+            }
+          }
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int row = row0 + 4 * (k0 + k);
+            if (row < rows_left) __stcs(out_tile + static_cast<size_t>(row) * D + c * 32, o[k]);
+          }
+        }
       }
     }
   }
@@ -569,7 +597,7 @@ __global__ void __launch_bounds__(384, 1)
 
 template <int D>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
-                               const CUtensorMap &to, const float *beta,
+                               float *out, const float *beta,
                                const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask,
                                const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H, int T, int causal,
                                unsigned *err, cudaStream_t stream) {
@@ -578,28 +606,21 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
   const uint32_t smem = TcLayout<D>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  // The producer warpgroup gives registers down to 56 and the softmax takes
-  // them up to 256 from the block's launch allocation (384 threads x numRegs);
-  // the correction keeps numRegs.  An increase the allocation cannot cover
-  // would wait forever, so the split is checked before any launch.
-  cudaFuncAttributes fa;
-  if ((e = cudaFuncGetAttributes(&fa, fem_tc_kernel<D>)) != cudaSuccess) return e;
-  if (128 * (56 + 256 + fa.numRegs) > 384 * fa.numRegs) return cudaErrorInvalidConfiguration;
   const dim3 grid(n_qt, BH);
-  fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
+  fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
                                                 err);
   return cudaGetLastError();
 }
 
-cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, const CUtensorMap &to,
+cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, float *out,
                       const float *beta, const ChanInfo *chan, const float *shift, const float *rfac,
                       const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H,
                       int T, int causal, unsigned *err, cudaStream_t stream) {
   if (d == 64)
-    return launch_tc_d<64>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
+    return launch_tc_d<64>(tq, tk, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
                            err, stream);
   if (d == 128)
-    return launch_tc_d<128>(tq, tk, te, to, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
+    return launch_tc_d<128>(tq, tk, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
                             err, stream);
   return cudaErrorInvalidValue;
 }
