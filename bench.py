@@ -52,6 +52,7 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle CPU-baseline budget")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-context", action="store_true", help="skip the torch SDPA context timing")
     ap.add_argument("--shape", default=None,
                     help="B,H,T override of the workload sizes (profiling aid; the JSON config reports them)")
     return ap.parse_args()
@@ -342,6 +343,43 @@ def run_fem(args):
     achieved = w.flops / (tc_ms * 1e-3) / 1e12
     traffic = recorded_traffic(w.name)
 
+    # ---- context: plain softmax attention (torch SDPA) on the same Q, K, V
+    context = None
+    if not args.no_context:
+        try:
+            import torch.nn.functional as F
+            for _ in range(3):
+                F.scaled_dot_product_attention(qd, kd, vd, is_causal=w.causal)
+            c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            c0.record(stream)
+            for _ in range(10):
+                F.scaled_dot_product_attention(qd, kd, vd, is_causal=w.causal)
+            c1.record(stream)
+            torch.cuda.synchronize(device)
+            sdpa_ms = c0.elapsed_time(c1) / 10
+            context = {"sdpa": {"ms": sdpa_ms, "tflops": w.flops / (sdpa_ms * 1e-3) / 1e12,
+                                "what": "torch scaled_dot_product_attention, same bf16 Q/K/V and mask "
+                                        "(plain softmax attention: no value bank, no shifts)"}}
+        except Exception as exc:  # context only; the FEM numbers stand without it
+            context = {"sdpa": {"unavailable": str(exc)[:200]}}
+        # the two-level gated read (beta = 0 and beta_max reads plus the gate kernel)
+        lam = torch.rand(q.shape, device=device)
+        gate = torch.ones(q.shape, device=device)
+        gout = torch.empty(q.shape, dtype=torch.float32, device=device)
+        for _ in range(2):
+            fem.fem_fwd_gated(qd, kd, vd, bd, lam, gate, causal=w.causal, out=gout, lse=False, stream=stream)
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(5):
+            fem.fem_fwd_gated(qd, kd, vd, bd, lam, gate, causal=w.causal, out=gout, lse=False, stream=stream)
+        g1.record(stream)
+        torch.cuda.synchronize(device)
+        fem.check_device_error(stream)
+        gated_ms = g0.elapsed_time(g1) / 5
+        context["gated_read"] = {"ms": gated_ms, "what": "fem_fwd_gated: out = g ((1 - lambda) mu + lambda Fmax), "
+                                                         "two reads (beta = 0, beta_max) and one gate kernel"}
+        del lam, gate, gout
+
     # ---- end to end through the host-buffer C ABI call
     e2e = None
     if not args.no_e2e:
@@ -383,7 +421,8 @@ def run_fem(args):
             "e2e": e2e,
             "cpu_baseline": cpu,
             "clocks": clk,
-            "gpu_launches": K * (4 if w.causal else 3),  # stats+plan, bank, tensor-core read (+ fix-up)
+            "context": context,
+            "gpu_launches": K * (5 if w.causal else 4),  # stats, plan, bank, tensor-core read (+ fix-up)
         }
         print(json.dumps(line), flush=True)
     if dist is not None:

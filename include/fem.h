@@ -124,6 +124,31 @@ int fem_fwd_noalloc(const void *q, const void *k, const void *v,
                     int T, int d, int causal, void *stream);
 
 /*
+ * fem_fwd_gated -- the two-level gated read (Sec. 3, "Two-Level Gated FEM":
+ * inner gate by linearised temperature learning, Eq. "inner-gate-main", and
+ * outer gate, Eq. "fem-two-gates-main"):
+ *
+ *   mu_{t,j}   = sum_{i in M_t} p_t(i) v_{i,j}                   (the beta = 0 read)
+ *   Fmax_{t,j} = (1/bmax_j) log sum_{i in M_t} p_t(i) exp(bmax_j v_{i,j})
+ *   out_{t,j}  = g_{t,j} ((1 - lambda_{t,j}) mu_{t,j} + lambda_{t,j} Fmax_{t,j})
+ *
+ *   q, k, v   : device, bf16 [B, H, T, d]
+ *   beta_max  : device, float32 [H, d], > 0 (the global maximum inverse temperature)
+ *   lam, gate : device, float32 [B, H, T, d]: the inner gate lambda in [0, 1]
+ *               and the outer gate g (> 0), already activated by the caller
+ *   out, lse  : as fem_fwd; lse does not depend on the gates
+ *   d in {64, 128}
+ * Runs the tensor-core read twice, at beta = 0 and at beta_max, into a
+ * workspace copy of mu and into out, then combines them elementwise in one
+ * kernel.  Allocates its workspace stream-ordered on `stream` (about
+ * 4 B*H*T*d bytes for mu plus fem_fwd's workspace).  Errors as fem_fwd; a
+ * null or misaligned lam or gate is FEM_ERR_INVALID_ARG.
+ */
+int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta_max,
+                  const float *lam, const float *gate, float *out, float *lse, int B,
+                  int H, int T, int d, int causal, void *stream);
+
+/*
  * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
  * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
  * on a bounded wait since the last check (the word is cleared), or

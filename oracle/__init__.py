@@ -13,6 +13,10 @@ Definition followed (Sec. 2.3, Eq. "fem-free-energy-main"; App. C,
 Eq. "softmax-prior"): o_{t,j} = (1/beta_j) log sum_{i in M_t} p_t(i)
 exp(beta_j v_{i,j}) with p_t = softmax(q_t . k_i / sqrt(d)) over the masked
 support M_t, beta_j = 0 meaning the prior mean; lse_t = LSE_i s_{t,i}.
+
+``gated_read`` composes it into the two-level gated read of Sec. 3
+("Two-Level Gated FEM"): out = g ((1 - lambda) mu + lambda Fmax), mu the
+beta = 0 read and Fmax the read at beta_max.
 """
 from __future__ import annotations
 
@@ -115,3 +119,22 @@ def fem_read_rows(q, k, v, beta, causal: bool, rows, nthreads: int = 0, lib=None
     if rc != 0:
         raise ValueError(f"fem_oracle_rows failed with code {rc}")
     return out, lse
+
+
+def gated_read(q, k, v, beta_max, lam, gate, causal: bool, nthreads: int = 0, lib=None):
+    """Two-level gated read (Sec. 3, "Two-Level Gated FEM").
+
+    The inner gate interpolates the prior mean mu_{t,j} = sum_i p_t(i) v_{i,j}
+    (the beta = 0 read) and the high-temperature branch Fmax_{t,j} (the read at
+    beta_max_j), Eq. "inner-gate-main"; the outer gate scales the result,
+    Eq. "fem-two-gates-main":
+
+        out = gate * ((1 - lam) * mu + lam * Fmax)
+
+    q, k, v, lam, gate: [B, H, T, d]; beta_max: [H, d] (> 0).  lam and gate
+    are taken as given (the activations that produce them are upstream).
+    Returns (out [B, H, T, d], lse [B, H, T]) as float64 numpy arrays."""
+    lam, gate, beta_max = _f64(lam), _f64(gate), _f64(beta_max)
+    mu, lse = fem_read(q, k, v, np.zeros_like(beta_max), causal, nthreads=nthreads, lib=lib)
+    fmax, _ = fem_read(q, k, v, beta_max, causal, nthreads=nthreads, lib=lib)
+    return gate * ((1.0 - lam) * mu + lam * fmax), lse

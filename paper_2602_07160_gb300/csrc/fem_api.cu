@@ -256,6 +256,36 @@ int fem_fwd(const void *q, const void *k, const void *v, const float *beta, floa
   return map_cuda(e);
 }
 
+int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta_max, const float *lam,
+                  const float *gate, float *out, float *lse, int B, int H, int T, int d, int causal, void *stream) {
+  int rc = check_common(q, k, v, beta_max, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (!lam || !gate || !aligned16(lam) || !aligned16(gate)) return FEM_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  // workspace: mu [B, H, T, d] fp32, a zero beta [H, d], then fem_fwd_ws's
+  const size_t n = static_cast<size_t>(B) * H * T * d;
+  const size_t mu_bytes = round256(n * sizeof(float)), zb_bytes = round256(static_cast<size_t>(H) * d * sizeof(float));
+  const size_t ws_bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  void *buf = nullptr;
+  cudaError_t e = cudaMallocAsync(&buf, mu_bytes + zb_bytes + ws_bytes, s);
+  if (e != cudaSuccess) return map_cuda(e);
+  float *mu = static_cast<float *>(buf);
+  float *zero_beta = reinterpret_cast<float *>(static_cast<uint8_t *>(buf) + mu_bytes);
+  void *ws = static_cast<uint8_t *>(buf) + mu_bytes + zb_bytes;
+  e = cudaMemsetAsync(zero_beta, 0, static_cast<size_t>(H) * d * sizeof(float), s);
+  rc = map_cuda(e);
+  // mu: the beta = 0 read; Fmax: the read at beta_max, into out; then the gates
+  if (rc == FEM_OK) rc = fem_fwd_ws(q, k, v, zero_beta, mu, nullptr, B, H, T, d, causal, ws, ws_bytes, stream);
+  if (rc == FEM_OK) rc = fem_fwd_ws(q, k, v, beta_max, out, lse, B, H, T, d, causal, ws, ws_bytes, stream);
+  if (rc == FEM_OK) rc = map_cuda(launch_gate(mu, lam, gate, out, n, ds->num_sms, s));
+  e = cudaFreeAsync(buf, s);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(e);
+}
+
 int fem_fwd_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse, int B,
                 int H, int T, int d, int causal, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);

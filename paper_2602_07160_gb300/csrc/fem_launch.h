@@ -55,6 +55,11 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
                          float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
                          const int *rows, int *last_rows, int num_sms, cudaStream_t stream);
 
+// out = g (lambda F + (1 - lambda) mu), elementwise over n floats (n % 4 == 0,
+// 16-byte-aligned arrays); out holds F on entry.
+cudaError_t launch_gate(const float *mu, const float *lam, const float *g, float *out, size_t n, int num_sms,
+                        cudaStream_t stream);
+
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
                        int B, int H, int T, int d, int causal, cudaStream_t stream);

@@ -23,7 +23,7 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
-           "fem_fwd_noalloc"]
+           "fem_fwd_noalloc", "fem_fwd_gated"]
 
 
 class FemError(RuntimeError):
@@ -54,6 +54,8 @@ def load(path: str | None = None):
         lib.fem_fwd_host.argtypes = sig + [vp]
         lib.fem_fwd_noalloc.argtypes = sig + [vp]
         lib.fem_fwd_noalloc.restype = i
+        lib.fem_fwd_gated.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
+        lib.fem_fwd_gated.restype = i
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
@@ -135,6 +137,24 @@ def fem_fwd_ws(q, k, v, beta, workspace, causal: bool = True, out=None, lse=None
                            _stream(stream, q.device))
     if rc != 0:
         raise FemError("fem_fwd_ws", rc)
+    return out, (None if lse is False else lse)
+
+
+def fem_fwd_gated(q, k, v, beta_max, lam, gate, causal: bool = True, out=None, lse=None, stream=None):
+    """The two-level gated read on bf16 CUDA tensors: out = gate * ((1 - lam) mu + lam Fmax).
+
+    lam and gate are float32 [B, H, T, d] (already activated); beta_max is float32 [H, d].
+    Returns (out, lse)."""
+    B, H, T, d = _check_qkvb(q, k, v, beta_max, torch.bfloat16, "cuda")
+    for name, t in (("lam", lam), ("gate", gate)):
+        if t.shape != q.shape or t.dtype != torch.float32 or not t.is_contiguous() or t.device != q.device:
+            raise ValueError(f"{name} must be a contiguous float32 tensor shaped like q on its device")
+    out, lse = _outputs(q, out, lse, q.device)
+    rc = load().fem_fwd_gated(_ptr(q), _ptr(k), _ptr(v), _ptr(beta_max), _ptr(lam), _ptr(gate), _ptr(out),
+                              None if lse is False else _ptr(lse), B, H, T, d, int(bool(causal)),
+                              _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_fwd_gated", rc)
     return out, (None if lse is False else lse)
 
 

@@ -74,3 +74,21 @@ def test_unsupported_head_dim(lib):
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError):
         fem.load(str(tmp_path / "missing.so"))
+
+
+def test_gated_argument_errors_are_synchronous(lib):
+    """fem_fwd_gated rejects bad gates and head dimensions before any CUDA call."""
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    f = lib.fem_fwd_gated
+    ok = dict(q=16, k=16, v=16, b=16, lam=16, g=16, out=16)
+
+    def call(d=64, **kw):
+        a = dict(ok, **kw)
+        return f(p(a["q"]), p(a["k"]), p(a["v"]), p(a["b"]), p(a["lam"]), p(a["g"]), p(a["out"]), None,
+                 1, 1, 8, d, 1, None)
+
+    assert call(lam=0) == 1
+    assert call(g=0) == 1
+    assert call(lam=24) == 1  # not 16-byte aligned
+    assert call(b=0) == 1
+    assert call(d=32) == 2

@@ -1,0 +1,79 @@
+"""The two-level gated read on the GPU against the float64 oracle (needs a GB300).
+
+out = g ((1 - lambda) mu + lambda Fmax) (Sec. 3, "Two-Level Gated FEM"), with
+gates drawn as the paper parameterises them (lambda a sigmoid output in
+[0, 1], g a softplus output normalised to RMS 1 over the channels).  The
+tolerance is the bf16 read's (max abs 2e-2, mean abs 2e-3) scaled by the
+largest |g|, since the outer gate multiplies the read's error.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2602_07160_gb300 import build, fem
+from paper_2602_07160_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+BF16_MAX, BF16_MEAN = 2e-2, 2e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    return fem.load()
+
+
+def _gates(seed, shape):
+    g = torch.Generator().manual_seed(seed)
+    lam = torch.sigmoid(torch.randn(shape, generator=g, dtype=torch.float32) * 2)
+    gate = torch.nn.functional.softplus(torch.randn(shape, generator=g, dtype=torch.float32))
+    gate = gate / gate.pow(2).mean(-1, keepdim=True).sqrt()
+    return lam, gate
+
+
+CASES = [
+    # B, H, T, d, causal
+    (1, 2, 300, 64, True),
+    (2, 2, 129, 128, True),
+    (1, 3, 256, 128, False),
+    (2, 2, 197, 64, False),
+]
+
+
+@pytest.mark.parametrize("B,H,T,d,causal", CASES)
+def test_gated_read_matches_oracle(B, H, T, d, causal):
+    q, k, v, bmax = W.make_custom(B, H, T, d, seed=11 * T + d)
+    lam, gate = _gates(T + d, q.shape)
+    dev = torch.device("cuda", 0)
+    args = [x.to(dev) for x in (q, k, v, bmax, lam, gate)]
+    out = torch.full(q.shape, float("nan"), dtype=torch.float32, device=dev)
+    out, lse = fem.fem_fwd_gated(*args, causal=causal, out=out)
+    fem.check_device_error()
+    ref, ref_lse = oracle.gated_read(q, k, v, bmax, lam, gate, causal)
+    o = out.cpu().double().numpy()
+    assert np.isfinite(o).all()
+    err = np.abs(o - ref)
+    scale = max(1.0, float(gate.abs().max()))
+    assert err.max() <= BF16_MAX * scale and err.mean() <= BF16_MEAN, (err.max(), err.mean())
+    assert np.abs(lse.cpu().double().numpy() - ref_lse).max() <= 2e-3
+
+
+def test_gated_read_limits_match_the_plain_reads():
+    """lambda = 0 gives g times the beta = 0 read, lambda = 1 and g = 1 the read at beta_max."""
+    B, H, T, d, causal = 1, 2, 200, 128, True
+    q, k, v, bmax = W.make_custom(B, H, T, d, seed=5)
+    dev = torch.device("cuda", 0)
+    qd, kd, vd, bd = (x.to(dev) for x in (q, k, v, bmax))
+    _, gate = _gates(3, q.shape)
+    gate = gate.to(dev)
+    zeros, ones = torch.zeros(q.shape, device=dev), torch.ones(q.shape, device=dev)
+    mu, _ = fem.fem_fwd(qd, kd, vd, torch.zeros_like(bd), causal=causal)
+    fmax, lse_f = fem.fem_fwd(qd, kd, vd, bd, causal=causal)
+    o0, lse0 = fem.fem_fwd_gated(qd, kd, vd, bd, zeros, gate, causal=causal)
+    o1, _ = fem.fem_fwd_gated(qd, kd, vd, bd, ones, ones, causal=causal)
+    fem.check_device_error()
+    assert torch.equal(o0, mu * gate)  # (1 - 0) mu + 0 (F - mu) = mu exactly, then times g
+    assert torch.allclose(o1, fmax, rtol=0, atol=1e-5)
+    assert torch.equal(lse0, lse_f)
