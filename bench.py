@@ -37,6 +37,7 @@ METRIC = "FEM fwd TFLOP/s and tensor-pipe % of GB300 peak (causal, T=8192, d=128
 UNIT = "TFLOP/s"
 L2_BYTES = 129 * 1024 * 1024
 FALLBACK_BF16_TFLOPS = 1900.0
+FALLBACK_HBM_GBS = 6800.0
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fem_tc_traffic.txt")
 TC_SOURCE = os.path.join(ROOT, "paper_2602_07160_gb300", "csrc", "fem_tc.cu")
 
@@ -165,6 +166,15 @@ def bf16_peak():
         return float(d["bf16_tflops"]), "measured (MEASURED_PEAKS.json bf16_tflops, burst)"
     except (OSError, KeyError, ValueError):
         return FALLBACK_BF16_TFLOPS, "fallback (1.9 PFLOP/s bf16 burst)"
+
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"])
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS
 
 
 def recorded_traffic(workload: str):
@@ -379,6 +389,28 @@ def run_fem(args):
         context["gated_read"] = {"ms": gated_ms, "what": "fem_fwd_gated: out = g ((1 - lambda) mu + lambda Fmax), "
                                                          "two reads (beta = 0, beta_max) and one gate kernel"}
         del lam, gate, gout
+        # the decode read: the last query row against the whole K/V cache (HBM-bound)
+        qdec = qd[:, :, -1, :].contiguous()
+        dout = torch.empty(qdec.shape, dtype=torch.float32, device=device)
+        dlse = torch.empty(qdec.shape[:2], dtype=torch.float32, device=device)
+        for _ in range(3):
+            fem.fem_decode(qdec, kd, vd, bd, out=dout, lse=dlse, stream=stream)
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        d0.record(stream)
+        for _ in range(20):
+            fem.fem_decode(qdec, kd, vd, bd, out=dout, lse=dlse, stream=stream)
+        d1.record(stream)
+        torch.cuda.synchronize(device)
+        fem.check_device_error(stream)
+        dec_ms = d0.elapsed_time(d1) / 20
+        dec_bytes = 2 * kd.numel() * kd.element_size() + qdec.numel() * 2 + dout.numel() * 4 + dlse.numel() * 4
+        hbm = hbm_peak()
+        context["decode"] = {"ms": dec_ms, "GB/s": dec_bytes / (dec_ms * 1e-3) / 1e9, "hbm_peak_GB/s": hbm,
+                             "frac": dec_bytes / (dec_ms * 1e-3) / 1e9 / hbm, "bytes": dec_bytes,
+                             "what": "fem_decode: one query per (b, h) against the K/V cache of this workload "
+                                     "(split over 128-key chunks, log-add-exp merge); algorithmic bytes K + V + q + "
+                                     "out + lse"}
+        del qdec, dout, dlse
 
     # ---- end to end through the host-buffer C ABI call
     e2e = None

@@ -149,6 +149,26 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
                   int H, int T, int d, int causal, void *stream);
 
 /*
+ * fem_decode -- the decode read: one new query per (b, h) against a cache of
+ * T keys and values that already holds the query's own key and value (the
+ * last row of a causal read; Sec. 2.3 read with the softmax prior of App. C):
+ *
+ *   s_i = q . k_i / sqrt(d),  o_j = (1/beta_j) log sum_i softmax(s)_i exp(beta_j v_{i,j}),
+ *   lse = LSE_i s_i,  i = 0 .. T-1
+ *
+ *   q        : device, bf16 [B, H, d]
+ *   k, v     : device, bf16 [B, H, T, d] (the cache)
+ *   beta     : device, float32 [H, d], beta >= 0 (0 = the prior mean)
+ *   out      : device, float32 [B, H, d];  lse: device, float32 [B, H] or NULL
+ *   d in {64, 128}
+ * Each CTA streams a range of keys in 64-key chunks; the ranges are merged
+ * with log-add-exp, all in fp32 arithmetic.  Allocates a small workspace
+ * (one partial of 3d + 2 floats per CTA) stream-ordered on `stream`.
+ */
+int fem_decode(const void *q, const void *k, const void *v, const float *beta, float *out,
+               float *lse, int B, int H, int T, int d, void *stream);
+
+/*
  * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
  * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
  * on a bounded wait since the last check (the word is cleared), or

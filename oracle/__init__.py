@@ -138,3 +138,20 @@ def gated_read(q, k, v, beta_max, lam, gate, causal: bool, nthreads: int = 0, li
     mu, lse = fem_read(q, k, v, np.zeros_like(beta_max), causal, nthreads=nthreads, lib=lib)
     fmax, _ = fem_read(q, k, v, beta_max, causal, nthreads=nthreads, lib=lib)
     return gate * ((1.0 - lam) * mu + lam * fmax), lse
+
+
+def decode_read(q, k, v, beta, nthreads: int = 0, lib=None):
+    """Decode read: one query per (b, h) against a cache of T keys and values
+    holding the query's own key and value, i.e. row T - 1 of the causal read
+    (Sec. 2.3, Eq. "fem-free-energy-main") whose query row is q.
+
+    q: [B, H, d]; k, v: [B, H, T, d]; beta: [H, d].
+    Returns (out [B, H, d], lse [B, H]) as float64 numpy arrays."""
+    q, k = _f64(q), _f64(k)
+    B, H, T, d = k.shape
+    assert q.shape == (B, H, d)
+    qf = np.zeros((B, H, T, d))
+    qf[:, :, T - 1, :] = q
+    rows = np.arange(B * H, dtype=np.int64) * T + (T - 1)
+    out, lse = fem_read_rows(qf, k, v, beta, True, rows, nthreads=nthreads, lib=lib)
+    return out.reshape(B, H, d), lse.reshape(B, H)

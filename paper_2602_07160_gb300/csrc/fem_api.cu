@@ -286,6 +286,31 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   return map_cuda(e);
 }
 
+int fem_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
+               int T, int d, void *stream) {
+  if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || T <= 0 || d <= 0) return FEM_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out)) return FEM_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(beta) & 3u) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return FEM_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * H > 65535 || static_cast<long long>(B) * H * T >= (1ll << 31))
+    return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  const int BH = B * H;
+  const size_t bytes = decode_workspace_bytes(BH, T, d, ds->num_sms);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  void *ws = nullptr;
+  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
+  if (e != cudaSuccess) return map_cuda(e);
+  rc = map_cuda(launch_decode(q, k, v, beta, out, lse, BH, H, T, d, static_cast<float *>(ws), ds->num_sms, ds->err, s));
+  e = cudaFreeAsync(ws, s);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(e);
+}
+
 int fem_fwd_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse, int B,
                 int H, int T, int d, int causal, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);

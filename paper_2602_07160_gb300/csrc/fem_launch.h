@@ -60,6 +60,12 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
 cudaError_t launch_gate(const float *mu, const float *lam, const float *g, float *out, size_t n, int num_sms,
                         cudaStream_t stream);
 
+// Decode read of one query per (b, h) against T cached keys: per-CTA key-range
+// partials into `part` (decode_workspace_bytes), then their log-add-exp merge.
+size_t decode_workspace_bytes(int BH, int T, int d, int num_sms);
+cudaError_t launch_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse,
+                          int BH, int H, int T, int d, float *part, int num_sms, unsigned *err, cudaStream_t stream);
+
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
                        int B, int H, int T, int d, int causal, cudaStream_t stream);

@@ -23,7 +23,7 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
-           "fem_fwd_noalloc", "fem_fwd_gated"]
+           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode"]
 
 
 class FemError(RuntimeError):
@@ -56,6 +56,8 @@ def load(path: str | None = None):
         lib.fem_fwd_noalloc.restype = i
         lib.fem_fwd_gated.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
         lib.fem_fwd_gated.restype = i
+        lib.fem_decode.argtypes = [vp, vp, vp, vp, vp, vp, i, i, i, i, vp]
+        lib.fem_decode.restype = i
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
@@ -155,6 +157,29 @@ def fem_fwd_gated(q, k, v, beta_max, lam, gate, causal: bool = True, out=None, l
                               _stream(stream, q.device))
     if rc != 0:
         raise FemError("fem_fwd_gated", rc)
+    return out, (None if lse is False else lse)
+
+
+def fem_decode(q, k, v, beta, out=None, lse=None, stream=None):
+    """Decode read on bf16 CUDA tensors: q [B, H, d] against the cache k, v [B, H, T, d].
+
+    Returns (out [B, H, d] float32, lse [B, H] float32)."""
+    if q.dim() != 3 or k.dim() != 4 or k.shape != v.shape or k.shape[:2] != q.shape[:2] or k.shape[3] != q.shape[2]:
+        raise ValueError("q must be [B, H, d] and k, v [B, H, T, d]")
+    B, H, T, d = k.shape
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if t.dtype != torch.bfloat16 or not t.is_contiguous() or t.device.type != "cuda":
+            raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    if beta.shape != (H, d) or beta.dtype != torch.float32 or not beta.is_contiguous() or beta.device != q.device:
+        raise ValueError("beta must be float32 [H, d] on q's device")
+    if out is None:
+        out = torch.empty((B, H, d), dtype=torch.float32, device=q.device)
+    if lse is None:
+        lse = torch.empty((B, H), dtype=torch.float32, device=q.device)
+    rc = load().fem_decode(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), None if lse is False else _ptr(lse),
+                           B, H, T, d, _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_decode", rc)
     return out, (None if lse is False else lse)
 
 

@@ -92,3 +92,13 @@ def test_gated_argument_errors_are_synchronous(lib):
     assert call(lam=24) == 1  # not 16-byte aligned
     assert call(b=0) == 1
     assert call(d=32) == 2
+
+
+def test_decode_argument_errors_are_synchronous(lib):
+    """fem_decode rejects bad pointers, sizes and head dimensions before any CUDA call."""
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    f = lib.fem_decode
+    assert f(None, p(16), p(16), p(16), p(16), None, 1, 1, 8, 64, None) == 1
+    assert f(p(16), p(16), p(16), p(16), p(24), None, 1, 1, 8, 64, None) == 1
+    assert f(p(16), p(16), p(16), p(16), p(16), None, 1, 1, 0, 64, None) == 1
+    assert f(p(16), p(16), p(16), p(16), p(16), None, 1, 1, 8, 96, None) == 2
