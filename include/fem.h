@@ -161,9 +161,9 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
  *   beta     : device, float32 [H, d], beta >= 0 (0 = the prior mean)
  *   out      : device, float32 [B, H, d];  lse: device, float32 [B, H] or NULL
  *   d in {64, 128}
- * Each CTA streams a range of keys in 64-key chunks; the ranges are merged
- * with log-add-exp, all in fp32 arithmetic.  Allocates a small workspace
- * (one partial of 3d + 2 floats per CTA) stream-ordered on `stream`.
+ * Each CTA reads a chunk of 64 keys; the chunks' partials are merged with
+ * log-add-exp in two levels, all in fp32 arithmetic.  Allocates a small
+ * workspace (3d + 2 floats per chunk) stream-ordered on `stream`.
  */
 int fem_decode(const void *q, const void *k, const void *v, const float *beta, float *out,
                float *lse, int B, int H, int T, int d, void *stream);
