@@ -411,6 +411,32 @@ def run_fem(args):
                                      "(split over 128-key chunks, log-add-exp merge); algorithmic bytes K + V + q + "
                                      "out + lse"}
         del qdec, dout, dlse
+        # the read over a GLA prior (O(T) recurrent scan), features m = 64, d = 64 on the same B, H, T
+        gen = torch.Generator(device=device).manual_seed(0)
+        Bg, Hg, Tg, mg, dg = w.B, w.H, w.T, 64, 64
+        qf = torch.relu(torch.randn((Bg, Hg, Tg, mg), device=device, generator=gen)) + 0.05
+        kf = torch.relu(torch.randn((Bg, Hg, Tg, mg), device=device, generator=gen)) + 0.05
+        vg = torch.randn((Bg, Hg, Tg, dg), device=device, generator=gen)
+        lg = -0.3 * torch.rand((Bg, Hg, Tg), device=device, generator=gen)
+        bg = torch.exp(torch.empty((Hg, dg), device=device).uniform_(-3.0, 3.0, generator=gen))
+        go = torch.empty((Bg, Hg, Tg, dg), device=device)
+        fem.fem_gla_fwd(qf, kf, vg, lg, bg, out=go, logz=False, stream=stream)
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(3):
+            fem.fem_gla_fwd(qf, kf, vg, lg, bg, out=go, logz=False, stream=stream)
+        a1.record(stream)
+        torch.cuda.synchronize(device)
+        fem.check_device_error(stream)
+        gla_ms = a0.elapsed_time(a1) / 3
+        gla_flops = 4.0 * mg * (dg + 1) * Tg * Bg * Hg  # state update and read-out, d channels + the normaliser
+        fp32_peak = 152 * 128 * 2 * 2.07e9 / 1e12  # FFMA lanes x 2 FLOP x max SM clock (nominal, derived)
+        context["gla_read"] = {"ms": gla_ms, "tflops": gla_flops / (gla_ms * 1e-3) / 1e12,
+                               "fp32_peak_tflops": fp32_peak, "frac": gla_flops / (gla_ms * 1e-3) / 1e12 / fp32_peak,
+                               "shape": {"B": Bg, "H": Hg, "T": Tg, "m": mg, "d": dg},
+                               "what": "fem_gla_fwd: FEM over a GLA prior, O(T) recurrent fp32 scan on CUDA cores; "
+                                       "FLOPs 4 m (d + 1) per step and head"}
+        del qf, kf, vg, lg, bg, go
 
     # ---- end to end through the host-buffer C ABI call
     e2e = None

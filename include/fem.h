@@ -169,6 +169,27 @@ int fem_decode(const void *q, const void *k, const void *v, const float *beta, f
                float *lse, int B, int H, int T, int d, void *stream);
 
 /*
+ * fem_gla_fwd -- the read over a gated-linear-attention prior (App. "Gated
+ * Linear Attention (GLA) Prior", Eqs. "gla-score-appendix" and "gla-assoc"):
+ *
+ *   s_t(i) = K_{t,i} <qf_t, kf_i> (i <= t),  K_{t,i} = exp(g_{i+1} + ... + g_t),
+ *   p_t = s_t / Z_t,  o_{t,j} = (1/beta_j) log sum_i p_t(i) exp(beta_j v_{i,j}),
+ *   logz_t = log Z_t
+ *
+ *   qf, kf   : device, float32 [B, H, T, m], nonnegative (the caller's
+ *              feature map, e.g. ReLU(RoPE(.)) + eps); m in {16, 32, 64}
+ *   v        : device, float32 [B, H, T, d], 1 <= d <= 155
+ *   logdecay : device, float32 [B, H, T], g_t <= 0
+ *   beta     : device, float32 [H, d], beta >= 0 (0 = the prior mean)
+ *   out      : device, float32 [B, H, T, d];  logz: device, float32 [B, H, T] or NULL
+ * An O(T) recurrent scan in fp32 on CUDA cores, one block per (b, h).  No
+ * workspace.
+ */
+int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *logdecay,
+                const float *beta, float *out, float *logz, int B, int H, int T, int m, int d,
+                void *stream);
+
+/*
  * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
  * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
  * on a bounded wait since the last check (the word is cleared), or

@@ -155,3 +155,40 @@ def decode_read(q, k, v, beta, nthreads: int = 0, lib=None):
     rows = np.arange(B * H, dtype=np.int64) * T + (T - 1)
     out, lse = fem_read_rows(qf, k, v, beta, True, rows, nthreads=nthreads, lib=lib)
     return out.reshape(B, H, d), lse.reshape(B, H)
+
+
+def gla_read(qf, kf, v, logdecay, beta):
+    """FEM read over a gated-linear-attention prior (App. "Gated Linear
+    Attention (GLA) Prior", Eq. "gla-score-appendix"), float64, O(T^2) per head.
+
+    qf, kf: [B, H, T, m] nonnegative features (the caller's ReLU(RoPE(.)) + eps);
+    v: [B, H, T, d]; logdecay: [B, H, T], g_t <= 0; beta: [H, d].
+    s_t(i) = K_{t,i} <qf_t, kf_i> for i <= t with K_{t,i} = exp(sum_{r=i+1..t} g_r),
+    p_t = s_t / Z_t, o_{t,j} = (1/beta_j) log sum_i p_t(i) exp(beta_j v_{i,j})
+    (beta_j = 0: sum_i p_t(i) v_{i,j}).
+    Returns (out [B, H, T, d], log Z [B, H, T]) as float64 numpy arrays."""
+    from scipy.special import logsumexp
+
+    qf, kf, v, g, beta = (_f64(x) for x in (qf, kf, v, logdecay, beta))
+    B, H, T, m = qf.shape
+    d = v.shape[-1]
+    out = np.empty((B, H, T, d))
+    logz = np.empty((B, H, T))
+    tri = np.tril(np.ones((T, T), dtype=bool))
+    for b in range(B):
+        for h in range(H):
+            G = np.cumsum(g[b, h])  # G_t = sum_{r <= t} g_r, so log K_{t,i} = G_t - G_i
+            with np.errstate(divide="ignore"):
+                logs = (G[:, None] - G[None, :]) + np.log(qf[b, h] @ kf[b, h].T)
+            logs = np.where(tri, logs, -np.inf)
+            lz = logsumexp(logs, axis=1)
+            logz[b, h] = lz
+            logp = logs - lz[:, None]
+            p = np.exp(logp)
+            for j in range(d):
+                bj = beta[h, j]
+                if bj == 0.0:
+                    out[b, h, :, j] = p @ v[b, h, :, j]
+                else:
+                    out[b, h, :, j] = logsumexp(logp + bj * v[b, h, None, :, j], axis=1) / bj
+    return out, logz

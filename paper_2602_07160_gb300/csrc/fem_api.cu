@@ -286,6 +286,24 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   return map_cuda(e);
 }
 
+int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta, float *out,
+                float *logz, int B, int H, int T, int m, int d, void *stream) {
+  if (!qf || !kf || !v || !logdecay || !beta || !out) return FEM_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || T <= 0 || m <= 0 || d <= 0) return FEM_ERR_INVALID_ARG;
+  if (!aligned16(qf) || !aligned16(kf)) return FEM_ERR_INVALID_ARG;
+  for (const void *p : {static_cast<const void *>(v), static_cast<const void *>(logdecay),
+                        static_cast<const void *>(beta), static_cast<const void *>(out),
+                        static_cast<const void *>(logz)})
+    if (p && (reinterpret_cast<uintptr_t>(p) & 3u)) return FEM_ERR_INVALID_ARG;
+  if ((m != 16 && m != 32 && m != 64) || d > 155) return FEM_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * H > 2147483647ll || static_cast<long long>(B) * H * T * (d > m ? d : m) >= (1ll << 40))
+    return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(launch_gla(qf, kf, v, logdecay, beta, out, logz, B * H, H, T, m, d, static_cast<cudaStream_t>(stream)));
+}
+
 int fem_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
                int T, int d, void *stream) {
   if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;

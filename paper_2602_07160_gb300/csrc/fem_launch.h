@@ -66,6 +66,10 @@ size_t decode_workspace_bytes(int BH, int T, int d, int num_sms);
 cudaError_t launch_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse,
                           int BH, int H, int T, int d, float *part, int num_sms, unsigned *err, cudaStream_t stream);
 
+// FEM read over a GLA prior (fp32, recurrent scan); m in {16, 32, 64}, d <= 155.
+cudaError_t launch_gla(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta,
+                       float *out, float *logz, int BH, int H, int T, int m, int d, cudaStream_t stream);
+
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
                        int B, int H, int T, int d, int causal, cudaStream_t stream);

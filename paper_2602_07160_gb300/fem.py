@@ -23,7 +23,7 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
-           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode"]
+           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd"]
 
 
 class FemError(RuntimeError):
@@ -58,6 +58,8 @@ def load(path: str | None = None):
         lib.fem_fwd_gated.restype = i
         lib.fem_decode.argtypes = [vp, vp, vp, vp, vp, vp, i, i, i, i, vp]
         lib.fem_decode.restype = i
+        lib.fem_gla_fwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
+        lib.fem_gla_fwd.restype = i
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
@@ -181,6 +183,31 @@ def fem_decode(q, k, v, beta, out=None, lse=None, stream=None):
     if rc != 0:
         raise FemError("fem_decode", rc)
     return out, (None if lse is False else lse)
+
+
+def fem_gla_fwd(qf, kf, v, logdecay, beta, out=None, logz=None, stream=None):
+    """The read over a GLA prior on fp32 CUDA tensors.
+
+    qf, kf: [B, H, T, m] nonnegative features; v: [B, H, T, d]; logdecay: [B, H, T] (<= 0);
+    beta: [H, d].  Returns (out [B, H, T, d], logz [B, H, T])."""
+    if qf.dim() != 4 or kf.shape != qf.shape or v.dim() != 4 or v.shape[:3] != qf.shape[:3]:
+        raise ValueError("qf, kf must be [B, H, T, m] and v [B, H, T, d]")
+    B, H, T, m = qf.shape
+    d = v.shape[3]
+    for name, t in (("qf", qf), ("kf", kf), ("v", v), ("logdecay", logdecay), ("beta", beta)):
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.device != qf.device or t.device.type != "cuda":
+            raise ValueError(f"{name} must be a contiguous float32 CUDA tensor on qf's device")
+    if logdecay.shape != (B, H, T) or beta.shape != (H, d):
+        raise ValueError("logdecay must be [B, H, T] and beta [H, d]")
+    if out is None:
+        out = torch.empty((B, H, T, d), dtype=torch.float32, device=qf.device)
+    if logz is None:
+        logz = torch.empty((B, H, T), dtype=torch.float32, device=qf.device)
+    rc = load().fem_gla_fwd(_ptr(qf), _ptr(kf), _ptr(v), _ptr(logdecay), _ptr(beta), _ptr(out),
+                            None if logz is False else _ptr(logz), B, H, T, m, d, _stream(stream, qf.device))
+    if rc != 0:
+        raise FemError("fem_gla_fwd", rc)
+    return out, (None if logz is False else logz)
 
 
 def fem_fwd_f32(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None):

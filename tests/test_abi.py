@@ -102,3 +102,18 @@ def test_decode_argument_errors_are_synchronous(lib):
     assert f(p(16), p(16), p(16), p(16), p(24), None, 1, 1, 8, 64, None) == 1
     assert f(p(16), p(16), p(16), p(16), p(16), None, 1, 1, 0, 64, None) == 1
     assert f(p(16), p(16), p(16), p(16), p(16), None, 1, 1, 8, 96, None) == 2
+
+
+def test_gla_argument_errors_are_synchronous(lib):
+    """fem_gla_fwd rejects bad pointers, sizes and feature widths before any CUDA call."""
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    f = lib.fem_gla_fwd
+
+    def call(qf=16, m=32, d=8, T=4):
+        return f(p(qf), p(16), p(16), p(16), p(16), p(16), None, 1, 1, T, m, d, None)
+
+    assert call(qf=0) == 1
+    assert call(qf=8) == 1  # not 16-byte aligned
+    assert call(T=0) == 1
+    assert call(m=48) == 2
+    assert call(d=200) == 2
