@@ -182,8 +182,9 @@ int fem_decode(const void *q, const void *k, const void *v, const float *beta, f
  *   logdecay : device, float32 [B, H, T], g_t <= 0
  *   beta     : device, float32 [H, d], beta >= 0 (0 = the prior mean)
  *   out      : device, float32 [B, H, T, d];  logz: device, float32 [B, H, T] or NULL
- * An O(T) recurrent scan in fp32 on CUDA cores, one block per (b, h).  No
- * workspace.
+ * An O(T) recurrent scan in fp32 on CUDA cores, split into time segments
+ * (segment end states, a combine over segments, then the outputs).  Allocates
+ * its workspace (the segments' start states) stream-ordered on `stream`.
  */
 int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *logdecay,
                 const float *beta, float *out, float *logz, int B, int H, int T, int m, int d,

@@ -301,7 +301,15 @@ int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *l
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
-  return map_cuda(launch_gla(qf, kf, v, logdecay, beta, out, logz, B * H, H, T, m, d, static_cast<cudaStream_t>(stream)));
+  const size_t bytes = gla_workspace_bytes(B * H, T, m, d, ds->num_sms, nullptr, nullptr);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  void *ws = nullptr;
+  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
+  if (e != cudaSuccess) return map_cuda(e);
+  rc = map_cuda(launch_gla(qf, kf, v, logdecay, beta, out, logz, B * H, H, T, m, d, ws, ds->num_sms, s));
+  e = cudaFreeAsync(ws, s);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(e);
 }
 
 int fem_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,

@@ -66,9 +66,12 @@ size_t decode_workspace_bytes(int BH, int T, int d, int num_sms);
 cudaError_t launch_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse,
                           int BH, int H, int T, int d, float *part, int num_sms, unsigned *err, cudaStream_t stream);
 
-// FEM read over a GLA prior (fp32, recurrent scan); m in {16, 32, 64}, d <= 155.
+// FEM read over a GLA prior (fp32, segmented recurrent scan); m in {16, 32, 64},
+// d <= 155; `ws` holds gla_workspace_bytes() bytes (segment states).
+size_t gla_workspace_bytes(int BH, int T, int m, int d, int num_sms, int *seg_len, int *n_seg);
 cudaError_t launch_gla(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta,
-                       float *out, float *logz, int BH, int H, int T, int m, int d, cudaStream_t stream);
+                       float *out, float *logz, int BH, int H, int T, int m, int d, void *ws, int num_sms,
+                       cudaStream_t stream);
 
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
