@@ -437,6 +437,27 @@ def run_fem(args):
                                "what": "fem_gla_fwd: FEM over a GLA prior, O(T) recurrent fp32 scan on CUDA cores; "
                                        "FLOPs 4 m (d + 1) per step and head"}
         del qf, kf, vg, lg, bg, go
+        # the time-decay conditioner's convolution, H_c = 64 channels over the same B and T (HBM-bound)
+        Hc = 64
+        ts = 0.05 * torch.nn.functional.softplus(torch.randn((w.B, w.T, Hc), device=device, generator=gen))
+        tu = torch.randn((w.B, w.T, Hc), device=device, generator=gen)
+        th = torch.empty_like(ts)
+        fem.fem_tdc_conv(ts, tu, out=th, stream=stream)
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record(stream)
+        for _ in range(20):
+            fem.fem_tdc_conv(ts, tu, out=th, stream=stream)
+        c1.record(stream)
+        torch.cuda.synchronize(device)
+        fem.check_device_error(stream)
+        tdc_ms = c0.elapsed_time(c1) / 20
+        tdc_bytes = 3 * ts.numel() * 4
+        context["tdc_conv"] = {"ms": tdc_ms, "GB/s": tdc_bytes / (tdc_ms * 1e-3) / 1e9, "hbm_peak_GB/s": hbm,
+                               "frac": tdc_bytes / (tdc_ms * 1e-3) / 1e9 / hbm,
+                               "shape": {"B": w.B, "T": w.T, "Hc": Hc},
+                               "what": "fem_tdc_conv: h_t = exp(-s_t) h_(t-1) + u_t, segmented scan; algorithmic "
+                                       "bytes s + u + h (fp32)"}
+        del ts, tu, th
 
     # ---- end to end through the host-buffer C ABI call
     e2e = None

@@ -191,6 +191,20 @@ int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *l
                 void *stream);
 
 /*
+ * fem_tdc_conv -- the time-decay conditioner's convolution (App. "Low-rank
+ * Convolution: Time-Decay Conditioner (TDC)", Eq. "tdc-conv", streaming form
+ * of Prop. "tdc-lowrank"):
+ *
+ *   h_t = sum_{i<=t} exp(-(s_{i+1} + ... + s_t)) u_i = exp(-s_t) h_{t-1} + u_t
+ *
+ *   s, u : device, float32 [B, T, Hc]; s >= 0 (the softplus rates)
+ *   h    : device, float32 [B, T, Hc]
+ * A segmented scan in fp32 (segment end states, a combine over segments, then
+ * the outputs).  Allocates its workspace stream-ordered on `stream`.
+ */
+int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc, void *stream);
+
+/*
  * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
  * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
  * on a bounded wait since the last check (the word is cleared), or

@@ -192,3 +192,19 @@ def gla_read(qf, kf, v, logdecay, beta):
                 else:
                     out[b, h, :, j] = logsumexp(logp + bj * v[b, h, None, :, j], axis=1) / bj
     return out, logz
+
+
+def tdc_conv(s, u):
+    """The time-decay conditioner's convolution (App. "Low-rank Convolution:
+    Time-Decay Conditioner (TDC)", Eq. "tdc-conv") by its definition, float64,
+    O(T^2) per channel: h_t = sum_{i<=t} exp(-(s_{i+1} + ... + s_t)) u_i.
+
+    s, u: [B, T, Hc].  Returns h [B, T, Hc] as a float64 numpy array."""
+    s, u = _f64(s), _f64(u)
+    B, T, Hc = s.shape
+    cs = np.cumsum(s, axis=1)  # cs_t = s_1 + ... + s_t, so the kernel is exp(-(cs_t - cs_i))
+    h = np.empty((B, T, Hc))
+    for t in range(T):
+        kern = np.exp(-(cs[:, t : t + 1, :] - cs[:, : t + 1, :]))
+        h[:, t, :] = (kern * u[:, : t + 1, :]).sum(axis=1)
+    return h

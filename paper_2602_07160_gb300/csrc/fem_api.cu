@@ -286,6 +286,25 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   return map_cuda(e);
 }
 
+int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc, void *stream) {
+  if (!s || !u || !h) return FEM_ERR_INVALID_ARG;
+  if (B <= 0 || T <= 0 || Hc <= 0) return FEM_ERR_INVALID_ARG;
+  for (const void *p : {static_cast<const void *>(s), static_cast<const void *>(u), static_cast<const void *>(h)})
+    if (reinterpret_cast<uintptr_t>(p) & 3u) return FEM_ERR_INVALID_ARG;
+  if (B > 65535 || static_cast<long long>(B) * T * Hc >= (1ll << 40)) return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void *ws = nullptr;
+  cudaError_t e = cudaMallocAsync(&ws, tdc_workspace_bytes(B, T, Hc), st);
+  if (e != cudaSuccess) return map_cuda(e);
+  rc = map_cuda(launch_tdc(s, u, h, B, T, Hc, ws, st));
+  e = cudaFreeAsync(ws, st);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(e);
+}
+
 int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta, float *out,
                 float *logz, int B, int H, int T, int m, int d, void *stream) {
   if (!qf || !kf || !v || !logdecay || !beta || !out) return FEM_ERR_INVALID_ARG;

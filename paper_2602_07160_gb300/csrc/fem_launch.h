@@ -73,6 +73,11 @@ cudaError_t launch_gla(const float *qf, const float *kf, const float *v, const f
                        float *out, float *logz, int BH, int H, int T, int m, int d, void *ws, int num_sms,
                        cudaStream_t stream);
 
+// Time-decay conditioner convolution h_t = exp(-s_t) h_{t-1} + u_t over [B, T, Hc]
+// (segmented scan); `ws` holds tdc_workspace_bytes() bytes.
+size_t tdc_workspace_bytes(int B, int T, int Hc);
+cudaError_t launch_tdc(const float *s, const float *u, float *h, int B, int T, int Hc, void *ws, cudaStream_t stream);
+
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
                        int B, int H, int T, int d, int causal, cudaStream_t stream);

@@ -23,7 +23,7 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
-           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd"]
+           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd", "fem_tdc_conv"]
 
 
 class FemError(RuntimeError):
@@ -60,6 +60,8 @@ def load(path: str | None = None):
         lib.fem_decode.restype = i
         lib.fem_gla_fwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
         lib.fem_gla_fwd.restype = i
+        lib.fem_tdc_conv.argtypes = [vp, vp, vp, i, i, i, vp]
+        lib.fem_tdc_conv.restype = i
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
@@ -208,6 +210,23 @@ def fem_gla_fwd(qf, kf, v, logdecay, beta, out=None, logz=None, stream=None):
     if rc != 0:
         raise FemError("fem_gla_fwd", rc)
     return out, (None if logz is False else logz)
+
+
+def fem_tdc_conv(s, u, out=None, stream=None):
+    """The time-decay conditioner's convolution h_t = exp(-s_t) h_{t-1} + u_t on fp32
+    CUDA tensors s, u of shape [B, T, Hc] (s >= 0).  Returns h."""
+    if s.dim() != 3 or u.shape != s.shape:
+        raise ValueError("s and u must share the shape [B, T, Hc]")
+    for name, t in (("s", s), ("u", u)):
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.device.type != "cuda" or t.device != s.device:
+            raise ValueError(f"{name} must be a contiguous float32 CUDA tensor on s's device")
+    B, T, Hc = s.shape
+    if out is None:
+        out = torch.empty_like(s)
+    rc = load().fem_tdc_conv(_ptr(s), _ptr(u), _ptr(out), B, T, Hc, _stream(stream, s.device))
+    if rc != 0:
+        raise FemError("fem_tdc_conv", rc)
+    return out
 
 
 def fem_fwd_f32(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None):

@@ -117,3 +117,12 @@ def test_gla_argument_errors_are_synchronous(lib):
     assert call(T=0) == 1
     assert call(m=48) == 2
     assert call(d=200) == 2
+
+
+def test_tdc_argument_errors_are_synchronous(lib):
+    """fem_tdc_conv rejects bad pointers and sizes before any CUDA call."""
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    f = lib.fem_tdc_conv
+    assert f(None, p(16), p(16), 1, 8, 4, None) == 1
+    assert f(p(16), p(16), p(18), 1, 8, 4, None) == 1
+    assert f(p(16), p(16), p(16), 1, 0, 4, None) == 1
