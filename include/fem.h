@@ -205,6 +205,27 @@ int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *l
 int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc, void *stream);
 
 /*
+ * fem_bwd_f32 -- gradients of the fp32 read (fem_fwd_f32) from its saved
+ * outputs, recomputing the scores:
+ *
+ *   dF/dv_{i,j}   = q_{t,i,j}, the posterior prop. to p_t(i) exp(beta_j v_{i,j})  (Prop. "app-geom")
+ *   dF/ds_{t,i}   = (q_{t,i,j} - p_t(i)) / beta_j                            (Prop. "app-bounds" (iv))
+ *   dF/dbeta_j    = KL(q || p) / beta_j^2                                     (Eq. "app-beta-deriv")
+ *
+ * chained through s = q k / sqrt(d).
+ *   q, k, v, out, dout : device, float32 [B, H, T, d]; out the forward's output
+ *   lse                : device, float32 [B, H, T], the forward's lse
+ *   beta               : device, float32 [H, d]
+ *   dq, dk, dv         : device, float32 [B, H, T, d]
+ *   dbeta              : device, float32 [H, d], summed over batch and time
+ *   1 <= d <= 256
+ * fp32 on CUDA cores, O(T^2 d) like the forward; no workspace.
+ */
+int fem_bwd_f32(const float *q, const float *k, const float *v, const float *beta, const float *out,
+                const float *lse, const float *dout, float *dq, float *dk, float *dv, float *dbeta,
+                int B, int H, int T, int d, int causal, void *stream);
+
+/*
  * fem_check_device_error -- synchronises `stream`, then returns FEM_OK, or
  * FEM_ERR_TIMEOUT if any kernel of this library on the current device gave up
  * on a bounded wait since the last check (the word is cleared), or

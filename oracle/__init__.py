@@ -208,3 +208,54 @@ def tdc_conv(s, u):
         kern = np.exp(-(cs[:, t : t + 1, :] - cs[:, : t + 1, :]))
         h[:, t, :] = (kern * u[:, : t + 1, :]).sum(axis=1)
     return h
+
+
+def fem_backward(q, k, v, beta, dout, causal: bool):
+    """Gradients of the read (float64 numpy), from the paper's derivatives:
+
+      dF_{t,j}/dv_{i,j}  = q_{t,i,j}                       (Prop. "app-geom", Eq. "app-grad-hess")
+      dF_{t,j}/ds_{t,i}  = (q_{t,i,j} - p_{t,i}) / beta_j  (Prop. "app-bounds" (iv), normalised logits)
+      dF_{t,j}/dbeta_j   = KL(q_{t,.,j} || p_t) / beta_j^2 (Eq. "app-beta-deriv")
+
+    with p_t = softmax(s_t), q_{t,.,j} proportional to p_t exp(beta_j v_{.,j}),
+    s_{t,i} = q_t . k_i / sqrt(d), and at beta_j = 0 the limits
+    (q - p)/beta -> p (v - mu) and KL/beta^2 -> Var_p(v)/2.  Chained through
+    the scores: dQ = dS K / sqrt(d), dK = dS^T Q / sqrt(d) with
+    dS_{t,i} = sum_j dout_{t,j} dF_{t,j}/ds_{t,i}.
+    q, k, v, dout: [B, H, T, d]; beta: [H, d].
+    Returns (dq, dk, dv [B, H, T, d], dbeta [H, d]) as float64 numpy arrays."""
+    from scipy.special import logsumexp
+
+    q, k, v, beta, dout = (_f64(x) for x in (q, k, v, beta, dout))
+    B, H, T, d = q.shape
+    dq, dk, dv = np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)
+    dbeta = np.zeros((H, d))
+    mask = np.tril(np.ones((T, T), dtype=bool)) if causal else np.ones((T, T), dtype=bool)
+    for b in range(B):
+        for h in range(H):
+            s = (q[b, h] @ k[b, h].T) / np.sqrt(d)
+            s = np.where(mask, s, -np.inf)
+            lse = logsumexp(s, axis=1)
+            p = np.exp(s - lse[:, None])
+            dS = np.zeros((T, T))
+            for j in range(d):
+                bj, vj, gj = beta[h, j], v[b, h, :, j], dout[b, h, :, j]
+                if bj == 0.0:
+                    mu = p @ vj
+                    qj = p
+                    dsj = p * (vj[None, :] - mu[:, None])
+                    kl_b2 = 0.5 * (p * (vj[None, :] - mu[:, None]) ** 2).sum(axis=1)
+                else:
+                    a = np.where(mask, s + bj * vj[None, :], -np.inf)
+                    G = logsumexp(a, axis=1)
+                    qj = np.exp(a - G[:, None])
+                    dsj = (qj - p) / bj
+                    with np.errstate(divide="ignore", invalid="ignore"):
+                        kl = np.where(qj > 0, qj * (np.log(qj) - np.log(np.where(p > 0, p, 1.0))), 0.0).sum(axis=1)
+                    kl_b2 = kl / bj**2
+                dS += gj[:, None] * dsj
+                dv[b, h, :, j] = qj.T @ gj
+                dbeta[h, j] += gj @ kl_b2
+            dq[b, h] = dS @ k[b, h] / np.sqrt(d)
+            dk[b, h] = dS.T @ q[b, h] / np.sqrt(d)
+    return dq, dk, dv, dbeta

@@ -286,6 +286,23 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   return map_cuda(e);
 }
 
+int fem_bwd_f32(const float *q, const float *k, const float *v, const float *beta, const float *out, const float *lse,
+                const float *dout, float *dq, float *dk, float *dv, float *dbeta, int B, int H, int T, int d,
+                int causal, void *stream) {
+  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (!lse || !dout || !dq || !dk || !dv || !dbeta) return FEM_ERR_INVALID_ARG;
+  for (const void *p : {static_cast<const void *>(dout), static_cast<const void *>(dq), static_cast<const void *>(dk),
+                        static_cast<const void *>(dv)})
+    if (!aligned16(p)) return FEM_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(dbeta) & 3u) return FEM_ERR_INVALID_ARG;
+  if (d > 256) return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  return map_cuda(launch_bwd_f32(q, k, v, beta, out, lse, dout, dq, dk, dv, dbeta, B, H, T, d, causal,
+                                 static_cast<cudaStream_t>(stream)));
+}
+
 int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc, void *stream) {
   if (!s || !u || !h) return FEM_ERR_INVALID_ARG;
   if (B <= 0 || T <= 0 || Hc <= 0) return FEM_ERR_INVALID_ARG;

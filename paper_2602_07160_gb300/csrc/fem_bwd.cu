@@ -1,0 +1,137 @@
+// Backward of the read for fp32 inputs on CUDA cores, from the saved out and
+// lse (flash-attention-style recomputation of the scores).  With
+// p_{t,i} = exp(s_{t,i} - lse_t) and x = beta_j (v_{i,j} - o_{t,j}), the
+// posterior is q_{t,i,j} = p_{t,i} exp(x) (since beta_j o_{t,j} + lse_t is its
+// log-normaliser), and the derivatives of the read are
+//
+//   dF_{t,j}/dv_{i,j} = q_{t,i,j}                      (Prop. "app-geom")
+//   dF_{t,j}/ds_{t,i} = (q - p)/beta = p expm1(x)/beta  (Prop. "app-bounds" (iv))
+//   dF_{t,j}/dbeta_j  = KL(q || p)/beta^2 = sum_i p phi(x)/beta^2,
+//                       phi(x) = 1 + (x - 1) e^x        (Eq. "app-beta-deriv")
+//
+// (sum_i p_i e^x = 1 turns KL = beta (E_q v - o) into the cancellation-free
+// sum of p phi(x) >= 0; at beta = 0 they become v - o and (v - o)^2 / 2).
+// Two passes, each one warp per row like the forward: rows (dq and dbeta,
+// with dS_{t,i} = sum_j dout_{t,j} dF_{t,j}/ds_{t,i}), then keys (dk and dv,
+// summing over the rows that see the key).
+#include "fem_common.cuh"
+#include "fem_launch.h"
+
+namespace fem {
+
+constexpr int kBwdMaxPerLane = 8;  // d <= 256
+
+// For y = v - o, x = b y and the log prior weight lp = s - lse, the
+// p-weighted terms q = p e^x, p expm1(x)/b and p phi(x)/b^2, formed without
+// e^x alone (which can overflow where p is tiny) and continuous at b = 0.
+__device__ __forceinline__ void bwd_terms(float b, float y, float lp, float &qv, float &ds, float &dbt) {
+  const float x = b * y, p = expf(lp);
+  qv = expf(lp + x);
+  if (fabsf(x) < 0.5f) {
+    ds = p * (b != 0.f ? expm1f(x) / b : y);
+  } else {
+    ds = (qv - p) / b;
+  }
+  if (fabsf(x) < 0.1f) {
+    // phi(x) = x^2/2 + x^3/3 + x^4/8 + x^5/30 + x^6/144 + ..., divided by b^2
+    dbt = p * y * y * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 1.f / 144.f, 1.f / 30.f), 0.125f), 1.f / 3.f), 0.5f);
+  } else {
+    dbt = fmaf(x - 1.f, qv, p) / (b * b);  // p phi(x) = p + (x - 1) q
+  }
+}
+
+// MODE 0: one warp per query row t -> dq_t and the row's dbeta terms.
+// MODE 1: one warp per key row i  -> dk_i and dv_i.
+template <int MODE>
+__global__ void __launch_bounds__(128) fem_bwd_kernel(const float *__restrict__ q, const float *__restrict__ k,
+                                                       const float *__restrict__ v, const float *__restrict__ beta,
+                                                       const float *__restrict__ out, const float *__restrict__ lse,
+                                                       const float *__restrict__ dout, float *__restrict__ da,
+                                                       float *__restrict__ db, float *__restrict__ dbeta, int H,
+                                                       int T, int d, int causal, long long n_rows) {
+  const int lane = threadIdx.x & 31;
+  const long long row = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (row >= n_rows) return;
+  const long long bh = row / T;
+  const int r = static_cast<int>(row % T);
+  const int h = static_cast<int>(bh % H);
+  const int per = (d + 31) / 32;
+  const float inv_sqrt_d = rsqrtf(static_cast<float>(d));
+  const size_t base = static_cast<size_t>(bh) * T * d;
+  float bj[kBwdMaxPerLane], own[kBwdMaxPerLane], own2[kBwdMaxPerLane], own3[kBwdMaxPerLane];
+  float acc1[kBwdMaxPerLane], acc2[kBwdMaxPerLane];
+#pragma unroll
+  for (int u = 0; u < kBwdMaxPerLane; ++u) {
+    const int j = lane + 32 * u;
+    const bool ok = u < per && j < d;
+    bj[u] = ok ? beta[h * d + j] : 0.f;
+    // MODE 0: own = q_t, own2 = o_t, own3 = dout_t;  MODE 1: own = k_i, own2 = v_i
+    own[u] = ok ? (MODE == 0 ? q : k)[base + static_cast<size_t>(r) * d + j] : 0.f;
+    own2[u] = ok ? (MODE == 0 ? out : v)[base + static_cast<size_t>(r) * d + j] : 0.f;
+    own3[u] = ok && MODE == 0 ? dout[base + static_cast<size_t>(r) * d + j] : 0.f;
+    acc1[u] = 0.f;
+    acc2[u] = 0.f;
+  }
+  const float lse_t = MODE == 0 ? lse[bh * T + r] : 0.f;
+  // the other side of the score: keys 0 .. (causal ? t : T-1) for a row,
+  // rows (causal ? i : 0) .. T-1 for a key
+  const int lo = MODE == 0 ? 0 : (causal ? r : 0);
+  const int hi = MODE == 0 ? (causal ? r + 1 : T) : T;
+  for (int o = lo; o < hi; ++o) {
+    const size_t ob = base + static_cast<size_t>(o) * d;
+    float part = 0.f;
+#pragma unroll
+    for (int u = 0; u < kBwdMaxPerLane; ++u) {
+      const int j = lane + 32 * u;
+      if (u < per && j < d) part = fmaf(own[u], (MODE == 0 ? k : q)[ob + j], part);
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+    const float lp = part * inv_sqrt_d - (MODE == 0 ? lse_t : lse[bh * T + o]);  // log p_{t,i}
+    float dS = 0.f;
+#pragma unroll
+    for (int u = 0; u < kBwdMaxPerLane; ++u) {
+      const int j = lane + 32 * u;
+      if (!(u < per && j < d)) continue;
+      // y = v_{i,j} - o_{t,j} with (i, t) = (o, r) for rows and (r, o) for keys
+      const float y = MODE == 0 ? v[ob + j] - own2[u] : own2[u] - out[ob + j];
+      const float g = MODE == 0 ? own3[u] : dout[ob + j];
+      float qv, ds, dbt;
+      bwd_terms(bj[u], y, lp, qv, ds, dbt);
+      dS = fmaf(g, ds, dS);
+      if (MODE == 0) acc2[u] = fmaf(g, dbt, acc2[u]);  // dbeta terms of this row
+      else acc2[u] = fmaf(g, qv, acc2[u]);             // dv_i: sum_t dout_{t,j} q_{t,i,j}
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) dS += __shfl_xor_sync(0xffffffffu, dS, off);
+#pragma unroll
+    for (int u = 0; u < kBwdMaxPerLane; ++u) {
+      const int j = lane + 32 * u;
+      if (u < per && j < d) acc1[u] = fmaf(dS, (MODE == 0 ? k : q)[ob + j], acc1[u]);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < kBwdMaxPerLane; ++u) {
+    const int j = lane + 32 * u;
+    if (!(u < per && j < d)) continue;
+    da[base + static_cast<size_t>(r) * d + j] = acc1[u] * inv_sqrt_d;
+    if (MODE == 0) atomicAdd(&dbeta[h * d + j], acc2[u]);
+    else db[base + static_cast<size_t>(r) * d + j] = acc2[u];
+  }
+}
+
+cudaError_t launch_bwd_f32(const float *q, const float *k, const float *v, const float *beta, const float *out,
+                           const float *lse, const float *dout, float *dq, float *dk, float *dv, float *dbeta, int B,
+                           int H, int T, int d, int causal, cudaStream_t stream) {
+  const long long n_rows = static_cast<long long>(B) * H * T;
+  const unsigned blocks = static_cast<unsigned>((n_rows + 3) / 4);
+  cudaError_t e = cudaMemsetAsync(dbeta, 0, static_cast<size_t>(H) * d * sizeof(float), stream);
+  if (e != cudaSuccess) return e;
+  fem_bwd_kernel<0><<<blocks, 128, 0, stream>>>(q, k, v, beta, out, lse, dout, dq, nullptr, dbeta, H, T, d, causal,
+                                                n_rows);
+  fem_bwd_kernel<1><<<blocks, 128, 0, stream>>>(q, k, v, beta, out, lse, dout, dk, dv, nullptr, H, T, d, causal,
+                                                n_rows);
+  return cudaGetLastError();
+}
+
+}  // namespace fem

@@ -78,6 +78,11 @@ cudaError_t launch_gla(const float *qf, const float *kf, const float *v, const f
 size_t tdc_workspace_bytes(int B, int T, int Hc);
 cudaError_t launch_tdc(const float *s, const float *u, float *h, int B, int T, int Hc, void *ws, cudaStream_t stream);
 
+// Backward of the fp32 read (dq, dk, dv, and dbeta summed over batch and time).
+cudaError_t launch_bwd_f32(const float *q, const float *k, const float *v, const float *beta, const float *out,
+                           const float *lse, const float *dout, float *dq, float *dk, float *dv, float *dbeta, int B,
+                           int H, int T, int d, int causal, cudaStream_t stream);
+
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
                        int B, int H, int T, int d, int causal, cudaStream_t stream);

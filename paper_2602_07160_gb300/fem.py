@@ -23,7 +23,7 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
-           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd", "fem_tdc_conv"]
+           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd", "fem_tdc_conv", "fem_bwd_f32"]
 
 
 class FemError(RuntimeError):
@@ -62,6 +62,8 @@ def load(path: str | None = None):
         lib.fem_gla_fwd.restype = i
         lib.fem_tdc_conv.argtypes = [vp, vp, vp, i, i, i, vp]
         lib.fem_tdc_conv.restype = i
+        lib.fem_bwd_f32.argtypes = [vp] * 11 + [i, i, i, i, i, vp]
+        lib.fem_bwd_f32.restype = i
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
@@ -227,6 +229,23 @@ def fem_tdc_conv(s, u, out=None, stream=None):
     if rc != 0:
         raise FemError("fem_tdc_conv", rc)
     return out
+
+
+def fem_bwd_f32(q, k, v, beta, out, lse, dout, causal: bool = True, stream=None):
+    """Gradients of the fp32 read from its saved (out, lse) and the output cotangent dout.
+
+    Returns (dq, dk, dv [B, H, T, d], dbeta [H, d] summed over batch and time)."""
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.float32, "cuda")
+    for name, t, shape in (("out", out, q.shape), ("dout", dout, q.shape), ("lse", lse, q.shape[:3])):
+        if t.shape != shape or t.dtype != torch.float32 or not t.is_contiguous() or t.device != q.device:
+            raise ValueError(f"{name} must be a contiguous float32 tensor of shape {tuple(shape)} on q's device")
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    dbeta = torch.empty_like(beta)
+    rc = load().fem_bwd_f32(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), _ptr(lse), _ptr(dout), _ptr(dq),
+                            _ptr(dk), _ptr(dv), _ptr(dbeta), B, H, T, d, int(bool(causal)), _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_bwd_f32", rc)
+    return dq, dk, dv, dbeta
 
 
 def fem_fwd_f32(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None):

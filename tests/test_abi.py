@@ -126,3 +126,17 @@ def test_tdc_argument_errors_are_synchronous(lib):
     assert f(None, p(16), p(16), 1, 8, 4, None) == 1
     assert f(p(16), p(16), p(18), 1, 8, 4, None) == 1
     assert f(p(16), p(16), p(16), 1, 0, 4, None) == 1
+
+
+def test_backward_argument_errors_are_synchronous(lib):
+    """fem_bwd_f32 rejects missing buffers and head dimensions before any CUDA call."""
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    f = lib.fem_bwd_f32
+
+    def call(lse=16, dq=16, d=64):
+        return f(p(16), p(16), p(16), p(16), p(16), p(lse), p(16), p(dq), p(16), p(16), p(16), 1, 1, 8, d, 1, None)
+
+    assert call(lse=0) == 1
+    assert call(dq=0) == 1
+    assert call(dq=8) == 1
+    assert call(d=300) == 2
