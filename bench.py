@@ -408,7 +408,7 @@ def run_fem(args):
         context["decode"] = {"ms": dec_ms, "GB/s": dec_bytes / (dec_ms * 1e-3) / 1e9, "hbm_peak_GB/s": hbm,
                              "frac": dec_bytes / (dec_ms * 1e-3) / 1e9 / hbm, "bytes": dec_bytes,
                              "what": "fem_decode: one query per (b, h) against the K/V cache of this workload "
-                                     "(split over 128-key chunks, log-add-exp merge); algorithmic bytes K + V + q + "
+                                     "(64-key chunk partials, log-add-exp merge); algorithmic bytes K + V + q + "
                                      "out + lse"}
         del qdec, dout, dlse
         # the read over a GLA prior (O(T) recurrent scan), features m = 64, d = 64 on the same B, H, T

@@ -67,14 +67,13 @@ int device_state(DeviceState **out) {
   return FEM_OK;
 }
 
-// [d, T, B*H] 16-bit tensor, boxes of 64 channels x 128 rows, 128-byte swizzle.
-// [BH, T, d] row-major tensor; boxes of 128 rows x 128 bytes (64 16-bit or 32
-// 32-bit elements), 128-byte swizzle.
+// [BH, T, d] row-major tensor; boxes of box_rows rows x 128 bytes (64 16-bit
+// or 32 32-bit elements), 128-byte swizzle.
 int make_map(CUtensorMap *map, const void *base, int BH, int T, int d,
-             CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, int elem_bytes = 2) {
+             CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, int elem_bytes = 2, int box_rows = 128) {
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(BH)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * elem_bytes, static_cast<cuuint64_t>(T) * d * elem_bytes};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(128 / elem_bytes), 128, 1};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(128 / elem_bytes), static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = g_encode(map, dtype, 3, const_cast<void *>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -367,7 +366,12 @@ int fem_decode(const void *q, const void *k, const void *v, const float *beta, f
   void *ws = nullptr;
   cudaError_t e = cudaMallocAsync(&ws, bytes, s);
   if (e != cudaSuccess) return map_cuda(e);
-  rc = map_cuda(launch_decode(q, k, v, beta, out, lse, BH, H, T, d, static_cast<float *>(ws), ds->num_sms, ds->err, s));
+  CUtensorMap tk;
+  if ((rc = make_map(&tk, k, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kDecodeKeysPerCta)) != FEM_OK) {
+    cudaFreeAsync(ws, s);
+    return rc;
+  }
+  rc = map_cuda(launch_decode(tk, q, v, beta, out, lse, BH, H, T, d, static_cast<float *>(ws), ds->err, s));
   e = cudaFreeAsync(ws, s);
   if (rc != FEM_OK) return rc;
   return map_cuda(e);

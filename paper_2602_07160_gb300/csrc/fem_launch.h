@@ -60,11 +60,14 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
 cudaError_t launch_gate(const float *mu, const float *lam, const float *g, float *out, size_t n, int num_sms,
                         cudaStream_t stream);
 
-// Decode read of one query per (b, h) against T cached keys: per-CTA key-range
+// Decode read of one query per (b, h) against T cached keys: per-CTA key-chunk
 // partials into `part` (decode_workspace_bytes), then their log-add-exp merge.
+// tk maps K as [BH, T, d] bf16 in boxes of kDecodeKeysPerCta rows x 64
+// channels with the 128-byte swizzle.
+constexpr int kDecodeKeysPerCta = 64;
 size_t decode_workspace_bytes(int BH, int T, int d, int num_sms);
-cudaError_t launch_decode(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse,
-                          int BH, int H, int T, int d, float *part, int num_sms, unsigned *err, cudaStream_t stream);
+cudaError_t launch_decode(const CUtensorMap &tk, const void *q, const void *v, const float *beta, float *out,
+                          float *lse, int BH, int H, int T, int d, float *part, unsigned *err, cudaStream_t stream);
 
 // FEM read over a GLA prior (fp32, segmented recurrent scan); m in {16, 32, 64},
 // d <= 155; `ws` holds gla_workspace_bytes() bytes (segment states).
