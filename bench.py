@@ -372,7 +372,7 @@ def run_fem(args):
                                         "(plain softmax attention: no value bank, no shifts)"}}
         except Exception as exc:  # context only; the FEM numbers stand without it
             context = {"sdpa": {"unavailable": str(exc)[:200]}}
-        # the two-level gated read (beta = 0 and beta_max reads plus the gate kernel)
+        # the two-level gated read (one pass over the beta = 0 and beta_max banks)
         lam = torch.rand(q.shape, device=device)
         gate = torch.ones(q.shape, device=device)
         gout = torch.empty(q.shape, dtype=torch.float32, device=device)
@@ -387,7 +387,7 @@ def run_fem(args):
         fem.check_device_error(stream)
         gated_ms = g0.elapsed_time(g1) / 5
         context["gated_read"] = {"ms": gated_ms, "what": "fem_fwd_gated: out = g ((1 - lambda) mu + lambda Fmax), "
-                                                         "two reads (beta = 0, beta_max) and one gate kernel"}
+                                                         "one pass: two banks, two accumulators, gated epilogue"}
         del lam, gate, gout
         # the decode read: the last query row against the whole K/V cache (HBM-bound)
         qdec = qd[:, :, -1, :].contiguous()

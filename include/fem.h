@@ -138,11 +138,13 @@ int fem_fwd_noalloc(const void *q, const void *k, const void *v,
  *               and the outer gate g (> 0), already activated by the caller
  *   out, lse  : as fem_fwd; lse does not depend on the gates
  *   d in {64, 128}
- * Runs the tensor-core read twice, at beta = 0 and at beta_max, into a
- * workspace copy of mu and into out, then combines them elementwise in one
- * kernel.  Allocates its workspace stream-ordered on `stream` (about
- * 4 B*H*T*d bytes for mu plus fem_fwd's workspace).  Errors as fem_fwd; a
- * null or misaligned lam or gate is FEM_ERR_INVALID_ARG.
+ * One tensor-core pass (the one-pass form of App. "One-pass implementation"):
+ * the same prior weights mix two value banks, the mean's and beta_max's,
+ * into two accumulators, and the epilogue applies the gates.  Allocates its
+ * workspace stream-ordered on `stream`: fem_fwd's workspace twice (one per
+ * bank) and, when causal, 4 B*H*T*d bytes written only at fix-up rows.
+ * Errors as fem_fwd; a null or misaligned lam or gate is
+ * FEM_ERR_INVALID_ARG.
  */
 int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta_max,
                   const float *lam, const float *gate, float *out, float *lse, int B,

@@ -186,20 +186,8 @@ size_t fem_fwd_workspace_bytes(int B, int H, int T, int d, int causal) {
   return w.total;
 }
 
-int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
-               int T, int d, int causal, void *workspace, size_t workspace_bytes, void *stream) {
-  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
-  if (rc != FEM_OK) return rc;
-  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
-  WsLayout w;
-  ws_layout(B, H, T, d, causal, &w);
-  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return FEM_ERR_INVALID_ARG;
-  if (workspace_bytes < w.total) return FEM_ERR_NO_MEMORY;
-  DeviceState *ds = nullptr;
-  if ((rc = device_state(&ds)) != FEM_OK) return rc;
-
-  const int BH = B * H;
-  uint8_t *ws = static_cast<uint8_t *>(workspace);
+// The read's workspace arrays at `ws` (layout ws_layout).
+static BankWorkspace bank_workspace(uint8_t *ws, const WsLayout &w, int causal) {
   BankWorkspace bw;
   bw.tstat = reinterpret_cast<float4 *>(ws + w.tstat);
   bw.chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
@@ -212,31 +200,78 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
   bw.fixup_rows = reinterpret_cast<int *>(ws + w.count) + 1;
   bw.tilefix = causal ? reinterpret_cast<int2 *>(ws + w.tilefix) : nullptr;
+  return bw;
+}
 
-  CUtensorMap tq, tk, tv, te;
+// Gated part of a read: the mean's pre-pass workspace (ws_layout, non-causal)
+// and its zero beta, the gates, and mu_side (causal only).
+struct GatedArgs {
+  uint8_t *ws0;
+  const float *zero_beta, *lam, *g;
+  float *mu_side;
+};
+
+// The read at beta (the plain read, or with ga the one-pass gated read at
+// beta_max = beta) into out and lse, with the arguments already checked.
+static int fwd_impl(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B,
+                    int H, int T, int d, int causal, uint8_t *ws, const GatedArgs *ga, DeviceState *ds,
+                    cudaStream_t s) {
+  const int BH = B * H;
+  WsLayout w;
+  ws_layout(B, H, T, d, causal, &w);
+  const BankWorkspace bw = bank_workspace(ws, w, causal);
+  CUtensorMap tq, tk, tv, te, te0;
+  int rc;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&tk, k, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&tv, v, BH, T, d)) != FEM_OK) return rc;
   if ((rc = make_map(&te, bw.bank, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT16)) != FEM_OK) return rc;
+  BankWorkspace bw0;
+  TcGate gate;
+  if (ga) {
+    WsLayout w0;
+    ws_layout(B, H, T, d, 0, &w0);
+    bw0 = bank_workspace(ga->ws0, w0, 0);
+    if ((rc = make_map(&te0, bw0.bank, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT16)) != FEM_OK) return rc;
+    gate = TcGate{ga->lam, ga->g, ga->mu_side, bw0.chan};
+  }
 
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 2 * sizeof(int), s);
+  // the mean's bank (every channel linear at beta = 0: v - c with c the channel mean)
+  if (e == cudaSuccess && ga) e = cudaMemsetAsync(bw0.fixup_count, 0, 2 * sizeof(int), s);
+  if (e == cudaSuccess && ga)
+    e = launch_value_bank(v, tv, te0, ga->zero_beta, BH, H, T, d, 0, bw0, ds->err, ds->num_sms, s);
   if (e == cudaSuccess) e = launch_value_bank(v, tv, te, beta, BH, H, T, d, causal, bw, ds->err, ds->num_sms, s);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
   if (e == cudaSuccess)
-    e = launch_tc(d, tq, tk, te, out, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, bw.tilefix, bw.fixups, lse, BH, H, T,
-                  causal, ds->err, s);
+    e = launch_tc(d, tq, tk, te, ga ? &te0 : nullptr, out, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, bw.tilefix,
+                  bw.fixups, lse, BH, H, T, causal, ga ? &gate : nullptr, ds->err, s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess) {
     if (causal)
       e = launch_fixup(q, k, v, beta, bw.shift, out, H, T, d, bw.fixups, bw.fixup_count, bw.fixup_rows,
-                       ds->last_fixup, ds->num_sms, s);
+                       ds->last_fixup, ga ? &gate : nullptr, ds->num_sms, s);
     else
       e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
   }
   return map_cuda(e);
+}
+
+int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
+               int T, int d, int causal, void *workspace, size_t workspace_bytes, void *stream) {
+  int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
+  if (rc != FEM_OK) return rc;
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  WsLayout w;
+  ws_layout(B, H, T, d, causal, &w);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return FEM_ERR_INVALID_ARG;
+  if (workspace_bytes < w.total) return FEM_ERR_NO_MEMORY;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  return fwd_impl(q, k, v, beta, out, lse, B, H, T, d, causal, static_cast<uint8_t *>(workspace), nullptr, ds,
+                  static_cast<cudaStream_t>(stream));
 }
 
 int fem_fwd(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse, int B, int H,
@@ -263,23 +298,27 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
-  // workspace: mu [B, H, T, d] fp32, a zero beta [H, d], then fem_fwd_ws's
+  // workspace: the beta_max read's, the mean's pre-pass (non-causal layout),
+  // a zero beta [H, d], and mu_side [B, H, T, d] fp32 for causal fix-ups
   const size_t n = static_cast<size_t>(B) * H * T * d;
-  const size_t mu_bytes = round256(n * sizeof(float)), zb_bytes = round256(static_cast<size_t>(H) * d * sizeof(float));
-  const size_t ws_bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
+  const size_t ws_bytes = round256(fem_fwd_workspace_bytes(B, H, T, d, causal));
+  const size_t ws0_bytes = round256(fem_fwd_workspace_bytes(B, H, T, d, 0));
+  const size_t zb_bytes = round256(static_cast<size_t>(H) * d * sizeof(float));
+  const size_t mu_bytes = causal ? round256(n * sizeof(float)) : 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *buf = nullptr;
-  cudaError_t e = cudaMallocAsync(&buf, mu_bytes + zb_bytes + ws_bytes, s);
+  cudaError_t e = cudaMallocAsync(&buf, ws_bytes + ws0_bytes + zb_bytes + mu_bytes, s);
   if (e != cudaSuccess) return map_cuda(e);
-  float *mu = static_cast<float *>(buf);
-  float *zero_beta = reinterpret_cast<float *>(static_cast<uint8_t *>(buf) + mu_bytes);
-  void *ws = static_cast<uint8_t *>(buf) + mu_bytes + zb_bytes;
-  e = cudaMemsetAsync(zero_beta, 0, static_cast<size_t>(H) * d * sizeof(float), s);
+  uint8_t *p = static_cast<uint8_t *>(buf);
+  GatedArgs ga;
+  ga.ws0 = p + ws_bytes;
+  ga.zero_beta = reinterpret_cast<const float *>(p + ws_bytes + ws0_bytes);
+  ga.lam = lam;
+  ga.g = gate;
+  ga.mu_side = causal ? reinterpret_cast<float *>(p + ws_bytes + ws0_bytes + zb_bytes) : nullptr;
+  e = cudaMemsetAsync(const_cast<float *>(ga.zero_beta), 0, static_cast<size_t>(H) * d * sizeof(float), s);
   rc = map_cuda(e);
-  // mu: the beta = 0 read; Fmax: the read at beta_max, into out; then the gates
-  if (rc == FEM_OK) rc = fem_fwd_ws(q, k, v, zero_beta, mu, nullptr, B, H, T, d, causal, ws, ws_bytes, stream);
-  if (rc == FEM_OK) rc = fem_fwd_ws(q, k, v, beta_max, out, lse, B, H, T, d, causal, ws, ws_bytes, stream);
-  if (rc == FEM_OK) rc = map_cuda(launch_gate(mu, lam, gate, out, n, ds->num_sms, s));
+  if (rc == FEM_OK) rc = fwd_impl(q, k, v, beta_max, out, lse, B, H, T, d, causal, p, &ga, ds, s);
   e = cudaFreeAsync(buf, s);
   if (rc != FEM_OK) return rc;
   return map_cuda(e);

@@ -34,6 +34,14 @@
 namespace fem {
 
 constexpr int kFixChunk = 8;                // entries per chunk = warps per block
+
+// The entry's output: F itself, or for the one-pass gated read
+// g (mu + lambda (F - mu)) with the mu the tensor-core kernel left aside.
+__device__ __forceinline__ float fix_gated(const TcGate &gate, size_t o, float F) {
+  if (!gate.lam) return F;
+  const float mu = gate.mu_side[o];
+  return gate.g[o] * fmaf(gate.lam[o], F - mu, mu);
+}
 constexpr int kFixThreads = 32 * kFixChunk;
 
 __device__ __forceinline__ float warp_max(float x) {
@@ -79,7 +87,7 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
                                                             int H, int T, const FixupEntry *__restrict__ entries,
                                                             const int *__restrict__ count,
                                                             const int *__restrict__ rows_listed,
-                                                            int *__restrict__ last_rows) {
+                                                            int *__restrict__ last_rows, TcGate gate) {
   // staged row strides in bf16 elements: K and Q rows 16-byte aligned for
   // ldmatrix with consecutive rows four banks apart; V rows an odd number of
   // 32-bit words, so one column read across rows is free of bank conflicts
@@ -193,7 +201,8 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
             if (kt > 0 && a_reg[gi] > 0.f && ent.l_pre > 0.f)
               pre = ent.m_pre + log2f(a_reg[gi]) + (b_reg[gi] * c_reg[gi] - kBankOffset) * kLog2e;
             const float G = lse2_pair(pre, mj + log2f(sj));
-            out[static_cast<size_t>(ent.row) * D + j] = (G - L) * kLn2 / b_reg[gi];
+            const size_t o = static_cast<size_t>(ent.row) * D + j;
+            out[o] = fix_gated(gate, o, (G - L) * kLn2 / b_reg[gi]);
           }
           m = 0;
         }
@@ -222,7 +231,7 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
             float pre = -INFINITY;
             if (kt > 0 && a > 0.f && ent.l_pre > 0.f) pre = ent.m_pre + log2f(a) + (bj * c - kBankOffset) * kLog2e;
             const float G = lse2_pair(pre, mj + log2f(sj));
-            out[o] = (G - L) * kLn2 / bj;
+            out[o] = fix_gated(gate, o, (G - L) * kLn2 / bj);
           }
         }
       }
@@ -233,21 +242,22 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
 
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
                          float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
-                         const int *rows, int *last_rows, int num_sms, cudaStream_t stream) {
+                         const int *rows, int *last_rows, const TcGate *gate, int num_sms, cudaStream_t stream) {
+  const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr};
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = num_sms * 3;
   if (d == 64) {
     const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
     fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
-                                                          last_rows);
+                                                          last_rows, g);
   } else if (d == 128) {
     const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
     cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     fixup_kernel<128><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
-                                                           last_rows);
+                                                           last_rows, g);
   } else {
     return cudaErrorInvalidValue;
   }

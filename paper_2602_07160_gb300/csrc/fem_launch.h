@@ -38,27 +38,37 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
                               int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
                               cudaStream_t stream);
 
+// Gates of the one-pass two-level gated read: o = g (mu + lambda (F - mu))
+// with mu the mean read (its bank v - c_lin, anchors chan0) and F the read at
+// beta_max.  lam, g: [B*H, T, d] fp32 inputs; mu_side: [B*H, T, d] fp32
+// scratch, written only at the fix-up entries (their mu, for the fix-up).
+struct TcGate {
+  const float *lam, *g;
+  float *mu_side;
+  const ChanInfo *chan0;
+};
+
 // Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
 // `out` is the fp32 output [B*H, T, d], 16-byte aligned.  For the
 // rows of a causal diagonal tile that have fix-up entries the kernel writes,
 // in place of the listed channels' outputs, their accumulator before the
-// diagonal tile, and the row's (max, sum) before it into the entry.
-cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, float *out,
-                      const float *beta, const ChanInfo *chan, const float *shift, const float *rfac,
-                      const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H,
-                      int T, int causal, unsigned *err, cudaStream_t stream);
+// diagonal tile, and the row's (max, sum) before it into the entry.  With
+// te0 (the mean's bank) and gate both given it runs the one-pass gated read;
+// with neither the plain read.
+cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
+                      const CUtensorMap *te0, float *out, const float *beta, const ChanInfo *chan, const float *shift,
+                      const float *rfac, const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse,
+                      int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream);
 
 // Completes the listed (row, channel) outputs: the diagonal tile's keys
 // exactly, merged with the state the tensor-core kernel left for the earlier
 // key tiles.
+// gate: nullptr, or the one-pass gated read's gates (the entries' outputs are
+// then gated with the mu the tensor-core kernel left in gate->mu_side).
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
                          float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
-                         const int *rows, int *last_rows, int num_sms, cudaStream_t stream);
+                         const int *rows, int *last_rows, const TcGate *gate, int num_sms, cudaStream_t stream);
 
-// out = g (lambda F + (1 - lambda) mu), elementwise over n floats (n % 4 == 0,
-// 16-byte-aligned arrays); out holds F on entry.
-cudaError_t launch_gate(const float *mu, const float *lam, const float *g, float *out, size_t n, int num_sms,
-                        cudaStream_t stream);
 
 // Decode read of one query per (b, h) against T cached keys: per-CTA key-chunk
 // partials into `part` (decode_workspace_bytes), then their log-add-exp merge.

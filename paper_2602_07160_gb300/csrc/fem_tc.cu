@@ -47,19 +47,25 @@
 
 namespace fem {
 
-template <int D>
+// GATED: the two-level gated read in one pass -- two banks per key tile (the
+// mean's, beta = 0, and beta_max's) into two accumulators of D columns each.
+template <int D, bool GATED>
 struct TcLayout {
+  static constexpr int kNB = GATED ? 2 : 1;  // banks per key tile
   static constexpr uint32_t kTile = D * 128 * 2;
-  static constexpr int kStagesK = 3, kStagesE = 2, kBufS = 3;
+  // 512 TMEM columns: kBufS score buffers of 128 and kNB * D accumulator columns
+  static constexpr int kBufS = (GATED && D == 128) ? 2 : 3;
+  static constexpr int kStagesK = (GATED && D == 128) ? 2 : 3;
+  static constexpr int kSlotsE = GATED ? (D == 128 ? 3 : 6) : 2;  // one bank tile per slot
   static constexpr uint32_t kQ = 0;
-  static constexpr uint32_t kK = kTile;                    // K[0..2]
-  static constexpr uint32_t kE = kK + kStagesK * kTile;    // E[0..1]
-  static constexpr uint32_t kBar = kE + kStagesE * kTile;  // mbarriers
-  static constexpr int kNumBars = 35;
+  static constexpr uint32_t kK = kTile;                    // K stages
+  static constexpr uint32_t kE = kK + kStagesK * kTile;    // E slots
+  static constexpr uint32_t kBar = kE + kSlotsE * kTile;   // mbarriers
+  static constexpr int kNumBars = 41;
   static constexpr uint32_t kTmemSlot = kBar + kNumBars * 8;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kChan = kBar + 512;               // per-channel epilogue coefficients
-  static constexpr uint32_t kMoveBits = kChan + 4 * D * 4;   // 1 bit per key tile: a shift moved
+  static constexpr uint32_t kMoveBits = kChan + 4 * D * 4 + (GATED ? 4 * D : 0);  // 1 bit per key tile: a shift moved
   static constexpr int kMaxKeyTiles = 8192;                  // T <= 1M keys
   // side ring: per key tile its rescale factors exp(beta_j (c_old - c_new)) [D]
   // and moved-channel mask [4], loaded with the K tile, kSideStages tiles deep
@@ -70,23 +76,28 @@ struct TcLayout {
   static constexpr uint32_t kInvL = kAlpha + kBufS * 128 * 4;         // 1/L per row, for the epilogue
   static constexpr uint32_t kBytes = kInvL + 128 * 4;
   static constexpr uint32_t kAlloc = kBytes + 1024;
-  static constexpr uint32_t kAccCol = 384;
+  static constexpr uint32_t kAccCol = kBufS * 128;
+  static constexpr uint32_t kAccB = kAccCol + (GATED ? D : 0);  // the beta (or beta_max) read's accumulator
+  static_assert(kAccCol + kNB * D <= 512, "TMEM columns");
+  static_assert(kBytes <= 227 * 1024 - 1024, "shared memory");
+  static_assert(kNB * D / 32 * 16384 + 4 * 128 * 4 <= (kStagesK * kTile + kSlotsE * kTile),
+                "epilogue staging fits the idle K and E rings");
 };
 
 // mbarrier indices
 enum : int {
   kBarQ = 0,
-  kBarKFull = 1,     // + K stage (3)
-  kBarKEmpty = 4,    // + K stage (3)
-  kBarEFull = 7,     // + E stage (2)
-  kBarEEmpty = 9,    // + E stage (2)
-  kBarSFull = 11,    // + score buffer (3): S_k complete
-  kBarPFull = 14,    // + score buffer (3): P_k written and acc rescaled (256 arrivals)
-  kBarPvDone = 17,   // + score buffer (3): P_k E_k complete
-  kBarAccDone = 20,  // every P E complete
-  kBarSDone = 21,    // every score contraction the S issuer started is complete
-  kBarAlpha = 22,    // + score buffer (3): the softmax's alpha of tile k is in shared memory (128 arrivals)
-  kBarSide = 25      // + side slot (8): tile k's rescale factors and moved-channel mask are in shared memory
+  kBarKFull = 1,     // + K stage (up to 3)
+  kBarKEmpty = 4,    // + K stage (up to 3)
+  kBarEFull = 7,     // + E slot (up to 6)
+  kBarEEmpty = 13,   // + E slot (up to 6)
+  kBarSFull = 19,    // + score buffer (up to 3): S_k complete
+  kBarPFull = 22,    // + score buffer: P_k written and acc rescaled (256 arrivals)
+  kBarPvDone = 25,   // + score buffer: P_k E_k complete
+  kBarAccDone = 28,  // every P E complete
+  kBarSDone = 29,    // every score contraction the S issuer started is complete
+  kBarAlpha = 30,    // + score buffer: the softmax's alpha of tile k is in shared memory (128 arrivals)
+  kBarSide = 33      // + side slot (8): tile k's rescale factors and moved-channel mask are in shared memory
 };
 
 // Bounded wait that also gives up as soon as another role has given up.
@@ -110,16 +121,17 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t *>(&v);
 }
 
-template <int D>
+template <int D, bool GATED>
 __global__ void __launch_bounds__(384, 1)
     fem_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                  const __grid_constant__ CUtensorMap tmap_e, float *__restrict__ out,
-                  const float *__restrict__ beta,
+                  const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_e0,
+                  float *__restrict__ out, const float *__restrict__ beta,
                   const ChanInfo *__restrict__ chan, const float *__restrict__ shift,
                   const float *__restrict__ rfac, const unsigned *__restrict__ colmask,
                   const int2 *__restrict__ tilefix, FixupEntry *__restrict__ fixups, float *__restrict__ lse, int H,
-                  int T, int causal, unsigned *__restrict__ err) {
-  using Lay = TcLayout<D>;
+                  int T, int causal, TcGate gate, unsigned *__restrict__ err) {
+  using Lay = TcLayout<D, GATED>;
+  constexpr int kNB = Lay::kNB, kBufS = Lay::kBufS, kStagesK = Lay::kStagesK, kSlotsE = Lay::kSlotsE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
@@ -142,11 +154,12 @@ __global__ void __launch_bounds__(384, 1)
   const int qt = causal ? n_qt - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x);
   const int nk = causal ? qt + 1 : n_kt_all;  // key tiles this query tile reads
 
-  // K tile kt into K stage kt % 3, with its side data into side slot kt % 8.
-  // Side slot kt % 8 was last read by the correction of tile kt - 8, which
-  // finished before PV(kt - 6), hence before S(kt - 3) released this K stage.
+  // K tile kt into K stage kt % kStagesK, with its side data into side slot
+  // kt % 8.  Side slot kt % 8 was last read by the correction of tile kt - 8,
+  // which finished before PV(kt - 8), hence before S(kt - kStagesK) (which
+  // waited for PV(kt - kStagesK - kBufS)) released this K stage.
   auto load_k = [&](int kt) {
-    const int st = kt % 3, ss = kt % Lay::kSideStages;
+    const int st = kt % kStagesK, ss = kt % Lay::kSideStages;
     mbar_arrive_expect_tx(FEM_BAR(kBarKFull + st), Lay::kTile);
     for (int b = 0; b < D / 64; ++b)
       tma_load_3d(sbase + Lay::kK + st * Lay::kTile + b * 16384, &tmap_k, FEM_BAR(kBarKFull + st), b * 64,
@@ -156,15 +169,18 @@ __global__ void __launch_bounds__(384, 1)
     bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride, rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
     bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride + D * 4, colmask + row * 4, 16, FEM_BAR(kBarSide + ss));
   };
-  // E tile kt into E stage kt % 2
-  auto load_e = [&](int kt) {
-    const int st = kt & 1;
+  // E item e (key tile e / kNB; bank e % kNB, the mean's first when GATED)
+  // into E slot e % kSlotsE
+  auto load_e = [&](int e) {
+    const int st = e % kSlotsE, kt = e / kNB;
+    const CUtensorMap *map = (GATED && e % kNB == 0) ? &tmap_e0 : &tmap_e;
     mbar_arrive_expect_tx(FEM_BAR(kBarEFull + st), Lay::kTile);
     for (int b = 0; b < D / 64; ++b)
-      tma_load_3d(sbase + Lay::kE + st * Lay::kTile + b * 16384, &tmap_e, FEM_BAR(kBarEFull + st), b * 64,
+      tma_load_3d(sbase + Lay::kE + st * Lay::kTile + b * 16384, map, FEM_BAR(kBarEFull + st), b * 64,
                   kt * kBlockK, bh);
   };
-  constexpr int kPreK = 3, kPreE = 2;  // loads the prologue issues (the rings' depths)
+  constexpr int kPreK = kStagesK, kPreE = kSlotsE;  // loads the prologue issues (the rings' depths)
+  const int ne = nk * kNB;                           // E items
 
   if (warp == 3) {
     tmem_alloc(sbase + Lay::kTmemSlot, 512);
@@ -172,15 +188,17 @@ __global__ void __launch_bounds__(384, 1)
   }
   if (tid == 0) {
     mbar_init(FEM_BAR(kBarQ), 1);
-    for (int s = 0; s < 3; ++s) {
+    for (int s = 0; s < kStagesK; ++s) {
       mbar_init(FEM_BAR(kBarKFull + s), 1);
       mbar_init(FEM_BAR(kBarKEmpty + s), 1);
+    }
+    for (int s = 0; s < kBufS; ++s) {
       mbar_init(FEM_BAR(kBarSFull + s), 1);
       mbar_init(FEM_BAR(kBarPFull + s), 256);
       mbar_init(FEM_BAR(kBarAlpha + s), 128);
       mbar_init(FEM_BAR(kBarPvDone + s), 1);
     }
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kSlotsE; ++s) {
       mbar_init(FEM_BAR(kBarEFull + s), 1);
       mbar_init(FEM_BAR(kBarEEmpty + s), 1);
     }
@@ -195,7 +213,7 @@ __global__ void __launch_bounds__(384, 1)
     for (int b = 0; b < D / 64; ++b)
       tma_load_3d(sbase + Lay::kQ + b * 16384, &tmap_q, FEM_BAR(kBarQ), b * 64, qt * kBlockQ, bh);
     for (int kt = 0; kt < min(nk, kPreK); ++kt) load_k(kt);
-    for (int kt = 0; kt < min(nk, kPreE); ++kt) load_e(kt);
+    for (int e = 0; e < min(ne, kPreE); ++e) load_e(e);
   }
   for (int j = tid; j < D; j += 384) {
     const ChanInfo ci = chan[bh * D + j];
@@ -207,6 +225,8 @@ __global__ void __launch_bounds__(384, 1)
       const float c = shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j];
       c_coef[j] = make_float4(0.f, c - kBankOffset / bj, kLn2 / bj, 1.f);
     }
+    // the mean's anchor: its bank holds v - c, so mu = c + acc/L
+    if (GATED) reinterpret_cast<float *>(c_coef + D)[j] = gate.chan0[bh * D + j].c_lin;
   }
   // one bit per key tile: set when some channel's shift moved there
   for (int base = 0; base < nk; base += 384) {
@@ -232,18 +252,18 @@ __global__ void __launch_bounds__(384, 1)
     // ---------------------------------------------------------------- TMA: Q and K
     if (lane == 0) {
       for (int kt = kPreK; kt < nk; ++kt) {
-        const uint32_t use = static_cast<uint32_t>(kt / 3);
-        if (!wait_or_abort(FEM_BAR(kBarKEmpty + kt % 3), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
+        const uint32_t use = static_cast<uint32_t>(kt / kStagesK);
+        if (!wait_or_abort(FEM_BAR(kBarKEmpty + kt % kStagesK), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
         load_k(kt);
       }
     }
   } else if (warp == 3) {
     // ---------------------------------------------------------------- TMA: E
     if (lane == 0) {
-      for (int kt = kPreE; kt < nk; ++kt) {
-        const uint32_t use = static_cast<uint32_t>(kt >> 1);
-        if (!wait_or_abort(FEM_BAR(kBarEEmpty + (kt & 1)), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
-        load_e(kt);
+      for (int e = kPreE; e < ne; ++e) {
+        const uint32_t use = static_cast<uint32_t>(e / kSlotsE);
+        if (!wait_or_abort(FEM_BAR(kBarEEmpty + e % kSlotsE), (use - 1) & 1, err, kErrWaitMma, abort_flag)) break;
+        load_e(e);
       }
       // no contraction may be in flight when the TMEM allocation is released:
       // both issuers commit these barriers on every exit path
@@ -256,14 +276,14 @@ __global__ void __launch_bounds__(384, 1)
       constexpr uint32_t idesc_qk = idesc_f16(128, 128, true, false);
       bool ok = wait_or_abort(FEM_BAR(kBarQ), 0, err, kErrWaitTma, abort_flag);
       for (int kt = 0; ok && kt < nk; ++kt) {
-        const int b = kt % 3;
-        const uint32_t use = static_cast<uint32_t>(kt / 3);
-        if (!(ok = wait_or_abort(FEM_BAR(kBarKFull + b), use & 1, err, kErrWaitTma, abort_flag))) break;
+        const int b = kt % kBufS, ks = kt % kStagesK;
+        const uint32_t use = static_cast<uint32_t>(kt / kBufS);
+        if (!(ok = wait_or_abort(FEM_BAR(kBarKFull + ks), (kt / kStagesK) & 1, err, kErrWaitTma, abort_flag))) break;
         // the buffer's previous tile must have been consumed by its P E
         if (use > 0 && !(ok = wait_or_abort(FEM_BAR(kBarPvDone + b), (use - 1) & 1, err, kErrWaitMma, abort_flag)))
           break;
         tc_fence_after_sync();
-        const uint32_t sK = sbase + Lay::kK + b * Lay::kTile;
+        const uint32_t sK = sbase + Lay::kK + ks * Lay::kTile;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
@@ -271,7 +291,7 @@ __global__ void __launch_bounds__(384, 1)
                      smem_desc_sw128(sK + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
         }
         mma_commit(FEM_BAR(kBarSFull + b));
-        mma_commit(FEM_BAR(kBarKEmpty + b));
+        mma_commit(FEM_BAR(kBarKEmpty + ks));
       }
       mma_commit(FEM_BAR(kBarSDone));
     }
@@ -280,18 +300,25 @@ __global__ void __launch_bounds__(384, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_pv = idesc_f16(128, D, false, true);
       const uint32_t tAcc = tmem + Lay::kAccCol;
-      for (int kt = 0; kt < nk; ++kt) {
-        const int b = kt % 3, st = kt & 1;
-        if (!wait_or_abort(FEM_BAR(kBarPFull + b), (kt / 3) & 1, err, kErrWaitMma, abort_flag)) break;
-        if (!wait_or_abort(FEM_BAR(kBarEFull + st), (kt >> 1) & 1, err, kErrWaitTma, abort_flag)) break;
-        tc_fence_after_sync();
-        const uint32_t sE = sbase + Lay::kE + st * Lay::kTile;
+      bool ok = true;
+      for (int kt = 0; ok && kt < nk; ++kt) {
+        const int b = kt % kBufS;
+        if (!(ok = wait_or_abort(FEM_BAR(kBarPFull + b), (kt / kBufS) & 1, err, kErrWaitMma, abort_flag))) break;
+        // each bank of the tile into its accumulator, D columns apart
 #pragma unroll
-        for (int kk = 0; kk < kBlockK / 16; ++kk)
-          mma_f16_ts(tAcc, tmem + b * 128 + kk * 8, smem_desc_sw128(sE + kk * 2048, 16384, 1024), idesc_pv,
-                     (kt > 0 || kk > 0) ? 1u : 0u);
+        for (int part = 0; part < kNB; ++part) {
+          const int e = kt * kNB + part, st = e % kSlotsE;
+          if (!(ok = wait_or_abort(FEM_BAR(kBarEFull + st), (e / kSlotsE) & 1, err, kErrWaitTma, abort_flag))) break;
+          tc_fence_after_sync();
+          const uint32_t sE = sbase + Lay::kE + st * Lay::kTile;
+#pragma unroll
+          for (int kk = 0; kk < kBlockK / 16; ++kk)
+            mma_f16_ts(tAcc + part * D, tmem + b * 128 + kk * 8, smem_desc_sw128(sE + kk * 2048, 16384, 1024),
+                       idesc_pv, (kt > 0 || kk > 0) ? 1u : 0u);
+          mma_commit(FEM_BAR(kBarEEmpty + st));
+        }
+        if (!ok) break;
         mma_commit(FEM_BAR(kBarPvDone + b));
-        mma_commit(FEM_BAR(kBarEEmpty + st));
       }
       mma_commit(FEM_BAR(kBarAccDone));  // completes once everything this thread issued is done
     }
@@ -303,7 +330,8 @@ __global__ void __launch_bounds__(384, 1)
     const int r = (tid - 128) & 127;  // row within the tile
     const int t_row = qt * kBlockQ + r;
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
-    const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;
+    const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;  // every accumulator column
+    const uint32_t tAccB = tmem + Lay::kAccB + lane_off;   // the beta read's
     float *s_alpha = reinterpret_cast<float *>(smem + Lay::kAlpha);
     float *s_invL = reinterpret_cast<float *>(smem + Lay::kInvL);
     // Rows 0 .. hz_rows-1 of a causal diagonal tile may have fix-up entries
@@ -318,17 +346,20 @@ __global__ void __launch_bounds__(384, 1)
     }
     const bool hz_warp = hz_rows > 32 * (warp & 3);  // warp-uniform
     const bool hz_row = r < hz_rows;
-    const uint32_t tStash = tmem + ((qt + 1) % 3) * 128 + lane_off;
+    // the score buffer no tile after the diagonal one uses; its last P E
+    // completed before the correction of the diagonal tile fills it
+    const uint32_t tStash = tmem + (nk % kBufS) * 128 + lane_off;
     float m_row = -INFINITY, L_row = 0.f;
     bool ok = true;
     if (is_sm) {
       // ------------------------------------------------------------ softmax
       const float qk_scale = kLog2e * rsqrtf(static_cast<float>(D));
       for (int kt = 0; kt < nk; ++kt) {
-        const int b = kt % 3;
+        const int b = kt % kBufS;
         const uint32_t tS = tmem + b * 128 + lane_off;
         // every lane takes the same branch: the wait's outcome is made warp-uniform
-        ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSFull + b), (kt / 3) & 1, err, kErrWaitMma, abort_flag));
+        ok = __all_sync(0xffffffffu,
+                        wait_or_abort(FEM_BAR(kBarSFull + b), (kt / kBufS) & 1, err, kErrWaitMma, abort_flag));
         if (!ok) break;
         tc_fence_after_sync();
         // the whole 128-column score row: four loads in flight, one wait
@@ -397,8 +428,9 @@ __global__ void __launch_bounds__(384, 1)
     else {
       // ------------------------------------------------------------ correction
       for (int kt = 0; kt < nk; ++kt) {
-        const int b = kt % 3;
-        ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAlpha + b), (kt / 3) & 1, err, kErrWaitMma, abort_flag));
+        const int b = kt % kBufS;
+        ok = __all_sync(0xffffffffu,
+                        wait_or_abort(FEM_BAR(kBarAlpha + b), (kt / kBufS) & 1, err, kErrWaitMma, abort_flag));
         if (!ok) break;
         const float alpha = s_alpha[b * 128 + r];
         const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
@@ -423,25 +455,37 @@ __global__ void __launch_bounds__(384, 1)
             for (int i = 0; i < 32; ++i) f0[i] = rf[g0 * 32 + i];
           }
           // acc is final for tile kt-1 once its P E completed
-          const int pb = (kt - 1) % 3;
-          ok = __all_sync(0xffffffffu,
-                          wait_or_abort(FEM_BAR(kBarPvDone + pb), ((kt - 1) / 3) & 1, err, kErrWaitMma, abort_flag));
+          const int pb = (kt - 1) % kBufS;
+          ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarPvDone + pb), ((kt - 1) / kBufS) & 1, err,
+                                                     kErrWaitMma, abort_flag));
           if (!ok) break;
           tc_fence_after_sync();
           if (stash) {
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
               uint32_t v[32];
-              tmem_ld32(tAcc + c * 32, v);
+              tmem_ld32(tAccB + c * 32, v);
               tmem_ld_wait();
               tmem_st32(tStash + c * 32, v);
             }
           }
           if (rowmv) {
+            if (GATED) {
+              // the mean's accumulator: the row maximum's factor only
+#pragma unroll 1
+              for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tAcc + c * 32, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+                tmem_st32(tAcc + c * 32, v);
+              }
+            }
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
               uint32_t v[32];
-              tmem_ld32(tAcc + c * 32, v);
+              tmem_ld32(tAccB + c * 32, v);
               tmem_ld_wait();
               if (colmv) {
 #pragma unroll
@@ -450,29 +494,29 @@ __global__ void __launch_bounds__(384, 1)
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
               }
-              tmem_st32(tAcc + c * 32, v);
+              tmem_st32(tAccB + c * 32, v);
             }
           } else if (colmv) {
             {
               uint32_t v[32];
-              tmem_ld32(tAcc + g0 * 32, v);
+              tmem_ld32(tAccB + g0 * 32, v);
               tmem_ld_wait();
 #pragma unroll
               for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * f0[i]);
-              tmem_st32(tAcc + g0 * 32, v);
+              tmem_st32(tAccB + g0 * 32, v);
             }
 #pragma unroll 1
             for (int c = g0 + 1; c < D / 32; ++c) {
               if (!((gm >> c) & 1u)) continue;
               uint32_t v[32];
-              tmem_ld32(tAcc + c * 32, v);
+              tmem_ld32(tAccB + c * 32, v);
               float f[32];
 #pragma unroll
               for (int i = 0; i < 32; ++i) f[i] = rf[c * 32 + i];
               tmem_ld_wait();
 #pragma unroll
               for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * f[i]);
-              tmem_st32(tAcc + c * 32, v);
+              tmem_st32(tAccB + c * 32, v);
             }
           }
           tmem_st_wait();
@@ -481,37 +525,42 @@ __global__ void __launch_bounds__(384, 1)
         mbar_arrive(FEM_BAR(kBarPFull + b));
       }
     }
-    // ---- epilogue, half the columns per warpgroup.  acc/L is staged in
-    // shared memory (the K ring is idle once every contraction completed) as
-    // 32-column boxes, row r by thread r; the transform then runs
-    // column-parallel and writes each row's 32 columns of a box as one
-    // coalesced 128-byte store.
+    // ---- epilogue, half the channels per warpgroup.  acc/L is staged in
+    // shared memory (the K and E rings are idle once every contraction
+    // completed) as 32-column boxes, row r by thread r; the transform then
+    // runs column-parallel and writes each row's 32 columns of a box as one
+    // coalesced 128-byte store.  GATED: boxes 0 .. D/32-1 hold the mean's
+    // accumulator, boxes D/32 .. 2D/32-1 the beta_max read's.
     if (ok) ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAccDone), 0, err, kErrWaitMma, abort_flag));
     ok = bar_and(1, 256, ok);  // both warpgroups went through every key tile
     if (ok) {
       tc_fence_after_sync();
       const float invL = s_invL[r];
-      constexpr int NC = D / 64;  // 32-column chunks of this warpgroup
+      constexpr int NC = D / 64;             // 32-column chunks of this warpgroup
+      constexpr int kBoxB = (kNB - 1) * (D / 32);  // first box of the beta read
       const int c_lo = is_sm ? 0 : NC;
       // (row, chunk) masks of the channels a fix-up row lists, in the idle
-      // part of the K ring behind the staging boxes
-      unsigned *s_hzm = reinterpret_cast<unsigned *>(smem + Lay::kK + (D / 32) * 16384);
-      uint32_t v[NC][32];
+      // rings behind the staging boxes
+      unsigned *s_hzm = reinterpret_cast<unsigned *>(smem + Lay::kK + kNB * (D / 32) * 16384);
+#pragma unroll 1
+      for (int part = 0; part < kNB; ++part) {
+        uint32_t v[NC][32];
 #pragma unroll
-      for (int c = 0; c < NC; ++c) tmem_ld32(tAcc + (c_lo + c) * 32, v[c]);
-      tmem_ld_wait();
+        for (int c = 0; c < NC; ++c) tmem_ld32(tAcc + part * D + (c_lo + c) * 32, v[c]);
+        tmem_ld_wait();
 #pragma unroll
-      for (int c = 0; c < NC; ++c) {
-        uint8_t *box = smem + Lay::kK + (c_lo + c) * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
+        for (int c = 0; c < NC; ++c) {
+          uint8_t *box = smem + Lay::kK + (part * (D / 32) + c_lo + c) * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
 #pragma unroll
-        for (int i4 = 0; i4 < 8; ++i4)
-          *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) =
-              make_float4(__uint_as_float(v[c][4 * i4]) * invL, __uint_as_float(v[c][4 * i4 + 1]) * invL,
-                          __uint_as_float(v[c][4 * i4 + 2]) * invL, __uint_as_float(v[c][4 * i4 + 3]) * invL);
+          for (int i4 = 0; i4 < 8; ++i4)
+            *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) =
+                make_float4(__uint_as_float(v[c][4 * i4]) * invL, __uint_as_float(v[c][4 * i4 + 1]) * invL,
+                            __uint_as_float(v[c][4 * i4 + 2]) * invL, __uint_as_float(v[c][4 * i4 + 3]) * invL);
+        }
       }
       if (hz_warp) {
-        // listed channels of fix-up rows: the accumulator before the diagonal
-        // tile, staged in place of acc/L and written out untransformed
+        // listed channels of fix-up rows: the beta read's accumulator before
+        // the diagonal tile, staged in place of acc/L and written out untransformed
 #pragma unroll 1
         for (int c = c_lo; c < c_lo + NC; ++c) {
           uint32_t w[32];
@@ -521,7 +570,7 @@ __global__ void __launch_bounds__(384, 1)
           }
           const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
           s_hzm[r * 4 + c] = mc;
-          uint8_t *box = smem + Lay::kK + c * 16384;
+          uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
 #pragma unroll
           for (int i = 0; i < 32; ++i)
             if ((mc >> i) & 1u)
@@ -536,24 +585,42 @@ __global__ void __launch_bounds__(384, 1)
       //   linear bank:  c + log1p(x)/beta with x = beta a, as lg2(1 + x) ln2/beta + c,
       //                 or, for |x| < 2^-6 (also beta = 0), as c + a times the
       //                 series of log1p(x)/x
+      // GATED: mu = c_mean + a_mean, F the beta_max read as above, and
+      // o = g (mu + lambda (F - mu)); a listed fix-up entry gets the stashed
+      // accumulator in out and mu in the gate's side buffer instead.
       const int col = r & 31, row0 = r >> 5;
       const int rows_left = T - qt * kBlockQ;
-      float *out_tile = out + (static_cast<size_t>(bh) * T + static_cast<size_t>(qt) * kBlockQ) * D + col;
+      const size_t tile_off = (static_cast<size_t>(bh) * T + static_cast<size_t>(qt) * kBlockQ) * D + col;
+      float *out_tile = out + tile_off;
 #pragma unroll 1
       for (int c = c_lo; c < c_lo + NC; ++c) {
         const float4 cf = c_coef[c * 32 + col];
+        const float c_mean = GATED ? reinterpret_cast<const float *>(c_coef + D)[c * 32 + col] : 0.f;
         const bool lin = cf.w == 0.f;
         // pairs of rows go through the packed fp32x2 pipe; the lg2 argument is
         // a (shifted) or 1 + beta a (linear)
         const float2 bx2 = make_float2(cf.x, cf.x), y2 = make_float2(cf.y, cf.y), z2 = make_float2(cf.z, cf.z);
         const float2 s12 = lin ? bx2 : make_float2(1.f, 1.f), s02 = make_float2(lin ? 1.f : 0.f, lin ? 1.f : 0.f);
-        const uint8_t *box = smem + Lay::kK + c * 16384 + ((col & 3) << 2);
+        const uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384 + ((col & 3) << 2);
+        const uint8_t *box_m = smem + Lay::kK + c * 16384 + ((col & 3) << 2);
 #pragma unroll 1
         for (int k0 = 0; k0 < 32; k0 += 8) {
           float a[8];
 #pragma unroll
           for (int k = 0; k < 8; ++k)
             a[k] = *reinterpret_cast<const float *>(box + sw128_offset(row0 + 4 * (k0 + k), col >> 2));
+          // GATED: the 8 rows' gates, in flight together with the math below
+          // (rows past T read the tile's last row and are not stored)
+          float lamv[8], gv[8];
+          if (GATED) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const size_t oi =
+                  tile_off + static_cast<size_t>(min(row0 + 4 * (k0 + k), rows_left - 1)) * D + c * 32;
+              lamv[k] = __ldcs(gate.lam + oi);
+              gv[k] = __ldcs(gate.g + oi);
+            }
+          }
           float o[8];
 #pragma unroll
           for (int k = 0; k < 8; k += 2) {
@@ -569,7 +636,20 @@ __global__ void __launch_bounds__(384, 1)
             o[k] = (lin && fabsf(x2.x) < 0.015625f) ? se.x : lg.x;
             o[k + 1] = (lin && fabsf(x2.y) < 0.015625f) ? se.y : lg.y;
           }
-          if (hz_rows > 0) {
+          if (GATED) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const int row = row0 + 4 * (k0 + k);
+              const float mu =
+                  c_mean + *reinterpret_cast<const float *>(box_m + sw128_offset(row0 + 4 * (k0 + k), col >> 2));
+              if (row < hz_rows && ((s_hzm[row * 4 + c] >> col) & 1u)) {
+                o[k] = a[k];
+                gate.mu_side[tile_off + static_cast<size_t>(row) * D + c * 32] = mu;
+              } else {
+                o[k] = gv[k] * fmaf(lamv[k], o[k] - mu, mu);
+              }
+            }
+          } else if (hz_rows > 0) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
               const int row = row0 + 4 * (k0 + k);
@@ -595,33 +675,45 @@ __global__ void __launch_bounds__(384, 1)
 #undef FEM_BAR
 }
 
-template <int D>
+template <int D, bool GATED>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
-                               float *out, const float *beta,
-                               const ChanInfo *chan, const float *shift, const float *rfac, const unsigned *colmask,
-                               const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H, int T, int causal,
+                               const CUtensorMap &te0, float *out, const float *beta, const ChanInfo *chan,
+                               const float *shift, const float *rfac, const unsigned *colmask, const int2 *tilefix,
+                               FixupEntry *fixups, float *lse, int BH, int H, int T, int causal, const TcGate &gate,
                                unsigned *err, cudaStream_t stream) {
+  using Lay = TcLayout<D, GATED>;
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
-  if (n_qt > TcLayout<D>::kMaxKeyTiles || BH > 65535) return cudaErrorInvalidValue;
-  const uint32_t smem = TcLayout<D>::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (n_qt > Lay::kMaxKeyTiles || BH > 65535) return cudaErrorInvalidValue;
+  const uint32_t smem = Lay::kAlloc;
+  cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D, GATED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const dim3 grid(n_qt, BH);
-  fem_tc_kernel<D><<<grid, 384, smem, stream>>>(tq, tk, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, H, T, causal,
-                                                err);
+  fem_tc_kernel<D, GATED><<<grid, 384, smem, stream>>>(tq, tk, te, te0, out, beta, chan, shift, rfac, colmask, tilefix,
+                                                       fixups, lse, H, T, causal, gate, err);
   return cudaGetLastError();
 }
 
-cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te, float *out,
-                      const float *beta, const ChanInfo *chan, const float *shift, const float *rfac,
-                      const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse, int BH, int H,
-                      int T, int causal, unsigned *err, cudaStream_t stream) {
+cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
+                      const CUtensorMap *te0, float *out, const float *beta, const ChanInfo *chan, const float *shift,
+                      const float *rfac, const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse,
+                      int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream) {
+  const TcGate none = {nullptr, nullptr, nullptr, nullptr};
+  if ((te0 != nullptr) != (gate != nullptr)) return cudaErrorInvalidValue;
+  if (gate) {
+    if (d == 64)
+      return launch_tc_d<64, true>(tq, tk, te, *te0, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH,
+                                   H, T, causal, *gate, err, stream);
+    if (d == 128)
+      return launch_tc_d<128, true>(tq, tk, te, *te0, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH,
+                                    H, T, causal, *gate, err, stream);
+    return cudaErrorInvalidValue;
+  }
   if (d == 64)
-    return launch_tc_d<64>(tq, tk, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
-                           err, stream);
+    return launch_tc_d<64, false>(tq, tk, te, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H,
+                                  T, causal, none, err, stream);
   if (d == 128)
-    return launch_tc_d<128>(tq, tk, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H, T, causal,
-                            err, stream);
+    return launch_tc_d<128, false>(tq, tk, te, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H,
+                                   T, causal, none, err, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -77,3 +77,29 @@ def test_gated_read_limits_match_the_plain_reads():
     assert torch.equal(o0, mu * gate)  # (1 - 0) mu + 0 (F - mu) = mu exactly, then times g
     assert torch.allclose(o1, fmax, rtol=0, atol=1e-5)
     assert torch.equal(lse0, lse_f)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_gated_read_fixup_rows(d):
+    """Spikes in small-valued beta_max = 20 channels move the bank shift in the
+    middle of diagonal tiles, so rows before each spike are completed by the
+    fix-up: there the gated output combines the fix-up's exact F with the mean
+    the tensor-core kernel set aside for the entry."""
+    B, H, T = 1, 2, 3000
+    q, k, v, bmax = W.make_custom(B, H, T, d, seed=7)
+    bmax[:, :8] = 20.0
+    vf = v.float()
+    vf[..., :8] *= 0.1
+    for p in (5, 20 * 128 + 64, 23 * 128 + 40):
+        vf[:, :, p, :8] = 3.0
+    v = vf.to(torch.bfloat16).contiguous()
+    lam, gate = _gates(d, q.shape)
+    dev = torch.device("cuda", 0)
+    out, lse = fem.fem_fwd_gated(*(x.to(dev) for x in (q, k, v, bmax, lam, gate)), causal=True)
+    fem.check_device_error()
+    assert fem.last_fixup_rows() >= 2 * (5 + 64 + 40)
+    ref, ref_lse = oracle.gated_read(q, k, v, bmax, lam, gate, True)
+    err = np.abs(out.cpu().double().numpy() - ref)
+    scale = max(1.0, float(gate.abs().max()))
+    assert err.max() <= BF16_MAX * scale and err.mean() <= BF16_MEAN, (err.max(), err.mean())
+    assert np.abs(lse.cpu().double().numpy() - ref_lse).max() <= 2e-3
