@@ -219,7 +219,7 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
   const int BH = B * H;
   WsLayout w;
   ws_layout(B, H, T, d, causal, &w);
-  const BankWorkspace bw = bank_workspace(ws, w, causal);
+  BankWorkspace bw = bank_workspace(ws, w, causal);
   CUtensorMap tq, tk, tv, te, te0;
   int rc;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
@@ -241,7 +241,9 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
   if (e == cudaSuccess && ga) e = cudaMemsetAsync(bw0.fixup_count, 0, 2 * sizeof(int), s);
   if (e == cudaSuccess && ga)
     e = launch_value_bank(v, tv, te0, ga->zero_beta, BH, H, T, d, 0, bw0, ds->err, ds->num_sms, s);
-  if (e == cudaSuccess) e = launch_value_bank(v, tv, te, beta, BH, H, T, d, causal, bw, ds->err, ds->num_sms, s);
+  if (ga) bw.tstat = bw0.tstat;  // the tiles' statistics do not depend on beta
+  if (e == cudaSuccess)
+    e = launch_value_bank(v, tv, te, beta, BH, H, T, d, causal, bw, ds->err, ds->num_sms, s, ga != nullptr);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);

@@ -451,7 +451,7 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
 
 cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtensorMap &te, const float *beta, int BH,
                               int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
-                              cudaStream_t stream) {
+                              cudaStream_t stream, bool stats_ready) {
   const int n_kt = (T + kBlockK - 1) / kBlockK, n_tiles = BH * n_kt;
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = min(n_tiles, 2 * num_sms);
@@ -464,7 +464,8 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(bank_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
     if (e != cudaSuccess) return e;
-    tile_stats_kernel<64><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
+    if (!stats_ready)
+      tile_stats_kernel<64><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
     plan_kernel<64><<<dim3(BH, 2), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, causal, w.chan, w.shift, w.rfac,
                                                      w.colmask, w.bcoef);
     bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, causal, w.fixups,
@@ -477,7 +478,8 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(bank_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
     if (e != cudaSuccess) return e;
-    tile_stats_kernel<128><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
+    if (!stats_ready)
+      tile_stats_kernel<128><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
     plan_kernel<128><<<dim3(BH, 4), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, causal, w.chan, w.shift, w.rfac,
                                                       w.colmask, w.bcoef);
     bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, causal, w.fixups,

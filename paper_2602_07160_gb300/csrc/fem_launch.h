@@ -33,10 +33,11 @@ struct BankWorkspace {
 //   shifted bank  {beta log2 e, (kBankOffset - beta c) log2 e, c, level}
 // with level = c - kHazardTilt/beta when the tile's keys are checked for the
 // causal diagonal hazard, -inf when not (not causal, or the running maximum
-// before the tile already reached it).
+// before the tile already reached it).  stats_ready: w.tstat already holds the
+// tiles' statistics of this V (they do not depend on beta); skip recomputing them.
 cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtensorMap &te, const float *beta, int BH,
                               int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
-                              cudaStream_t stream);
+                              cudaStream_t stream, bool stats_ready = false);
 
 // Gates of the one-pass two-level gated read: o = g (mu + lambda (F - mu))
 // with mu the mean read (its bank v - c_lin, anchors chan0) and F the read at
