@@ -25,6 +25,8 @@
 
 namespace fem {
 
+constexpr float kBankFastBeta = 1.f / 64.f;  // linear bank: (e^y - 1)/beta from here on
+
 // Ring of key tiles a persistent pre-pass block streams through shared
 // memory: kStages slots, one mbarrier each, filled by bulk copies that thread 0
 // issues kStages - 1 tiles ahead.  A block takes the tiles blockIdx.x,
@@ -349,23 +351,48 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
         }
         if (cf.w != cf.w) {
           // linear bank: D = expm1(y)/beta, y = beta (v - c) >= -1 (a = 1/beta,
-          // b = beta), as a Taylor series of expm1(y)/y for |y| < 1/2
-          // (truncation < 4e-6 relative), e^y - 1 beyond
+          // b = beta).  For beta >= kBankFastBeta as (e^y - 1)/beta: the
+          // absolute error of e^y (about 2^-22) over beta stays below 2^-16,
+          // under the fp16 rounding of D.  Smaller beta (and beta = 0): a Taylor
+          // series of expm1(y)/y for |y| < 1/2 (truncation < 4e-6 relative),
+          // e^y - 1 beyond.  Rows go through the packed fp32x2 pipe in pairs.
+          const float2 c2 = make_float2(-cf.z, -cf.z), b2 = make_float2(cf.y, cf.y);
+          const float2 l2 = make_float2(cf.y * kLog2e, cf.y * kLog2e);
+          if (cf.y >= kBankFastBeta) {
 #pragma unroll
-          for (int rb = 0; rb < 4; ++rb) {
-            const float xs = x[rb] - cf.z;
-            const float y = cf.y * xs;
-            float poly = fmaf(y, 1.f / 720.f, 1.f / 120.f);
-            poly = fmaf(y, poly, 1.f / 24.f);
-            poly = fmaf(y, poly, 1.f / 6.f);
-            poly = fmaf(y, poly, 0.5f);
-            poly = fmaf(y, poly, 1.f);
-            res[rb][u] = fabsf(y) < 0.5f ? xs * poly : (ex2_approx(y * kLog2e) - 1.f) * cf.x;
+            for (int rp = 0; rp < 2; ++rp) {
+              const float2 xs = __fadd2_rn(make_float2(x[2 * rp], x[2 * rp + 1]), c2);
+              const float2 t = __fmul2_rn(l2, xs);
+              const float2 d = __fmul2_rn(__fadd2_rn(make_float2(ex2_approx(t.x), ex2_approx(t.y)),
+                                                     make_float2(-1.f, -1.f)),
+                                          make_float2(cf.x, cf.x));
+              res[2 * rp][u] = d.x;
+              res[2 * rp + 1][u] = d.y;
+            }
+          } else {
+#pragma unroll
+            for (int rp = 0; rp < 2; ++rp) {
+              const float2 xs = __fadd2_rn(make_float2(x[2 * rp], x[2 * rp + 1]), c2);
+              const float2 y = __fmul2_rn(b2, xs);
+              float2 poly = __ffma2_rn(y, make_float2(1.f / 720.f, 1.f / 720.f), make_float2(1.f / 120.f, 1.f / 120.f));
+              poly = __ffma2_rn(y, poly, make_float2(1.f / 24.f, 1.f / 24.f));
+              poly = __ffma2_rn(y, poly, make_float2(1.f / 6.f, 1.f / 6.f));
+              poly = __ffma2_rn(y, poly, make_float2(0.5f, 0.5f));
+              poly = __ffma2_rn(y, poly, make_float2(1.f, 1.f));
+              const float2 lin = __fmul2_rn(xs, poly);
+              res[2 * rp][u] = fabsf(y.x) < 0.5f ? lin.x : (ex2_approx(y.x * kLog2e) - 1.f) * cf.x;
+              res[2 * rp + 1][u] = fabsf(y.y) < 0.5f ? lin.y : (ex2_approx(y.y * kLog2e) - 1.f) * cf.x;
+            }
           }
         } else {
           // shifted bank: E = 2^(a v + b)
 #pragma unroll
-          for (int rb = 0; rb < 4; ++rb) res[rb][u] = ex2_approx(fmaf(cf.x, x[rb], cf.y));
+          for (int rp = 0; rp < 2; ++rp) {
+            const float2 t = __ffma2_rn(make_float2(cf.x, cf.x), make_float2(x[2 * rp], x[2 * rp + 1]),
+                                        make_float2(cf.y, cf.y));
+            res[2 * rp][u] = ex2_approx(t.x);
+            res[2 * rp + 1][u] = ex2_approx(t.y);
+          }
         }
         int first = 0;
         if (cf.w > -INFINITY) {  // hazard check of a shifted channel
