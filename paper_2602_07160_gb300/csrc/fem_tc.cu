@@ -100,6 +100,8 @@ enum : int {
   kBarSide = 33      // + side slot (8): tile k's rescale factors and moved-channel mask are in shared memory
 };
 
+constexpr int kHeadGroup = 16;  // heads whose query tiles the launch order interleaves
+
 // Bounded wait that also gives up as soon as another role has given up.
 __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, unsigned *err, unsigned code,
                                               volatile int *abort_flag) {
@@ -148,10 +150,15 @@ __global__ void __launch_bounds__(384, 1)
   const int wg = __shfl_sync(0xffffffffu, tid >> 7, 0);  // warpgroup, provably warp-uniform
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   const int n_kt_all = (T + kBlockK - 1) / kBlockK;
-  // grid = (query tiles, B*H): CTAs in flight share a few heads' K and E in L2,
-  // and within a head the heaviest causal tiles start first
-  const int bh = blockIdx.y, h = bh % H;
-  const int qt = causal ? n_qt - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x);
+  // CTAs in launch order take the heads in groups of kHeadGroup: within a
+  // group the query tiles go heaviest first across its heads (causal), so the
+  // launch ends on the lightest tiles and the SMs finish together, while the
+  // CTAs in flight share the K and E of at most two groups in L2
+  const int rank = static_cast<int>(blockIdx.y * gridDim.x + blockIdx.x), BH = static_cast<int>(gridDim.y);
+  const int g0 = rank / (kHeadGroup * n_qt) * kHeadGroup, gsz = min(kHeadGroup, BH - g0);
+  const int idx = rank - g0 * n_qt;
+  const int bh = g0 + idx % gsz, h = bh % H;
+  const int qt = causal ? n_qt - 1 - idx / gsz : idx / gsz;
   const int nk = causal ? qt + 1 : n_kt_all;  // key tiles this query tile reads
 
   // K tile kt into K stage kt % kStagesK, with its side data into side slot
