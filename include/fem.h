@@ -57,8 +57,9 @@ typedef enum {
  *   out     : device, float32 [B, H, T, d]
  *   lse     : device, float32 [B, H, T], or NULL
  *   B, H, T : >= 1;  d in {64, 128};  causal: 0 (full prior) or 1
- * Allocates its workspace stream-ordered (cudaMallocAsync/cudaFreeAsync on
- * `stream`).  Accuracy: the score contraction takes bf16 q, k; the second
+ * Allocates its workspace stream-ordered on `stream` from a memory pool the
+ * library keeps per device (freed memory stays in the pool for the next
+ * call; the entry points that allocate all use it).  Accuracy: the score contraction takes bf16 q, k; the second
  * contraction takes the prior weights and the per-channel value bank in fp16
  * (11-bit significand); both accumulate in fp32.
  */
@@ -92,10 +93,14 @@ int fem_fwd_f32(const float *q, const float *k, const float *v,
 
 /*
  * fem_fwd_host -- fem_fwd on HOST buffers: copies q, k, v, beta to the
- * device, runs the read and copies out (and lse, if non-NULL) back, all on
- * `stream`, then synchronises it.  Host buffers should be pinned for full
- * copy bandwidth.  Device buffers come from cudaMallocAsync on `stream` and
- * are freed before return.  Returns after the results are in host memory.
+ * device, runs the read and copies out (and lse, if non-NULL) back, then
+ * synchronises `stream`.  The work is split into chunks of consecutive heads
+ * (about eight in all): the copies in of one chunk, the read of the previous
+ * one (on `stream`) and the copies out of the one before overlap, on two copy
+ * streams the library creates once per device.  Host buffers should be pinned
+ * for full copy bandwidth.  Device buffers come stream-ordered from the
+ * library's pool and are freed before return.  Returns after the results are
+ * in host memory; fem_last_fixup_rows then reports the last chunk's count.
  */
 int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
                  float *out, float *lse, int B, int H, int T, int d, int causal,
@@ -107,7 +112,7 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
  * allowed to allocate, or a service that reserves all device memory up
  * front).  The paper has no counterpart; this is an interface convenience.
  * Same arguments, layout and results as fem_fwd; the caller still passes
- * every input and output.  Instead of cudaMallocAsync it uses a fixed
+ * every input and output.  Instead of a stream-ordered allocation it uses a fixed
  * 16 MiB scratch array compiled into the library, which every GPU that
  * loads the library holds until the process exits.  Problems needing more
  * workspace than that (fem_fwd_workspace_bytes() > 16 MiB, about 2*d + 60

@@ -9,7 +9,9 @@
 //      diagonal tile, merged with the state fem_tc left for the earlier tiles
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
+#include <vector>
 
 #include "fem.h"
 #include "fem_launch.h"
@@ -27,6 +29,11 @@ struct DeviceState {
   unsigned *err = nullptr;
   int *last_fixup = nullptr;
   int num_sms = 0;
+  // stream-ordered workspaces come from this pool, which keeps freed memory for
+  // the next call instead of returning it to the driver at every synchronisation
+  cudaMemPool_t pool = nullptr;
+  // copy streams of fem_fwd_host, created on its first call
+  cudaStream_t copy_in = nullptr, copy_out = nullptr;
 };
 
 std::mutex g_mutex;
@@ -52,6 +59,13 @@ int device_state(DeviceState **out) {
     if (cudaGetSymbolAddress(reinterpret_cast<void **>(&s.last_fixup), g_last_fixup) != cudaSuccess)
       return FEM_ERR_CUDA;
     if (cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return FEM_ERR_CUDA;
+    cudaMemPoolProps props = {};
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    if (cudaMemPoolCreate(&s.pool, &props) != cudaSuccess) return FEM_ERR_CUDA;
+    uint64_t keep = ~uint64_t(0);
+    if (cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess) return FEM_ERR_CUDA;
     if (!g_encode) {
       cudaDriverEntryPointQueryResult q;
       void *fn = nullptr;
@@ -65,6 +79,11 @@ int device_state(DeviceState **out) {
   }
   *out = &s;
   return FEM_OK;
+}
+
+// Stream-ordered workspace from the device's library pool (free with cudaFreeAsync).
+cudaError_t ws_alloc(const DeviceState *ds, void **p, size_t bytes, cudaStream_t s) {
+  return cudaMallocFromPoolAsync(p, bytes, ds->pool, s);
 }
 
 // [BH, T, d] row-major tensor; boxes of box_rows rows x 128 bytes (64 16-bit
@@ -281,10 +300,12 @@ int fem_fwd(const void *q, const void *k, const void *v, const float *beta, floa
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
   if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
   const size_t bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
-  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
+  cudaError_t e = ws_alloc(ds, &ws, bytes, s);
   if (e != cudaSuccess) return map_cuda(e);
   rc = fem_fwd_ws(q, k, v, beta, out, lse, B, H, T, d, causal, ws, bytes, stream);
   e = cudaFreeAsync(ws, s);
@@ -309,7 +330,7 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   const size_t mu_bytes = causal ? round256(n * sizeof(float)) : 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *buf = nullptr;
-  cudaError_t e = cudaMallocAsync(&buf, ws_bytes + ws0_bytes + zb_bytes + mu_bytes, s);
+  cudaError_t e = ws_alloc(ds, &buf, ws_bytes + ws0_bytes + zb_bytes + mu_bytes, s);
   if (e != cudaSuccess) return map_cuda(e);
   uint8_t *p = static_cast<uint8_t *>(buf);
   GatedArgs ga;
@@ -354,7 +375,7 @@ int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc,
   if (rc != FEM_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
-  cudaError_t e = cudaMallocAsync(&ws, tdc_workspace_bytes(B, T, Hc), st);
+  cudaError_t e = ws_alloc(ds, &ws, tdc_workspace_bytes(B, T, Hc), st);
   if (e != cudaSuccess) return map_cuda(e);
   rc = map_cuda(launch_tdc(s, u, h, B, T, Hc, ws, st));
   e = cudaFreeAsync(ws, st);
@@ -380,7 +401,7 @@ int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *l
   const size_t bytes = gla_workspace_bytes(B * H, T, m, d, ds->num_sms, nullptr, nullptr);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
-  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
+  cudaError_t e = ws_alloc(ds, &ws, bytes, s);
   if (e != cudaSuccess) return map_cuda(e);
   rc = map_cuda(launch_gla(qf, kf, v, logdecay, beta, out, logz, B * H, H, T, m, d, ws, ds->num_sms, s));
   e = cudaFreeAsync(ws, s);
@@ -405,7 +426,7 @@ int fem_decode(const void *q, const void *k, const void *v, const float *beta, f
   const size_t bytes = decode_workspace_bytes(BH, T, d, ds->num_sms);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
-  cudaError_t e = cudaMallocAsync(&ws, bytes, s);
+  cudaError_t e = ws_alloc(ds, &ws, bytes, s);
   if (e != cudaSuccess) return map_cuda(e);
   CUtensorMap tk;
   if ((rc = make_map(&tk, k, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, kDecodeKeysPerCta)) != FEM_OK) {
@@ -433,33 +454,83 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
   if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0 || (causal != 0 && causal != 1)) return FEM_ERR_INVALID_ARG;
   if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  {
+    std::lock_guard<std::mutex> lock(g_mutex);
+    if (!ds->copy_in && cudaStreamCreateWithFlags(&ds->copy_in, cudaStreamNonBlocking) != cudaSuccess)
+      return FEM_ERR_CUDA;
+    if (!ds->copy_out && cudaStreamCreateWithFlags(&ds->copy_out, cudaStreamNonBlocking) != cudaSuccess)
+      return FEM_ERR_CUDA;
+  }
+  // Chunks of consecutive heads of one batch element (contiguous in every
+  // [B, H, T, d] array): the copies in of chunk c+1, the read of chunk c and
+  // the copies out of chunk c-1 overlap (two copy streams, the caller's stream
+  // computing).  About eight chunks in all.
+  const int per_b = std::max(1, std::min(H, 8 / B));
+  const int hc = (H + per_b - 1) / per_b;  // heads per chunk
+  const int n_chunks = B * ((H + hc - 1) / hc);
   const size_t n = static_cast<size_t>(B) * H * T * d;
   const size_t rows = static_cast<size_t>(B) * H * T;
   const size_t in_b = round256(n * 2), beta_b = round256(static_cast<size_t>(H) * d * 4), out_b = round256(n * 4),
-               lse_b = round256(rows * 4), ws_b = fem_fwd_workspace_bytes(B, H, T, d, causal);
+               lse_b = round256(rows * 4), ws_b = round256(fem_fwd_workspace_bytes(1, hc, T, d, causal));
   const size_t total = 3 * in_b + beta_b + out_b + lse_b + ws_b;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t *buf = nullptr;
-  cudaError_t e = cudaMallocAsync(reinterpret_cast<void **>(&buf), total, s);
+  cudaError_t e = ws_alloc(ds, reinterpret_cast<void **>(&buf), total, s);
   if (e != cudaSuccess) return map_cuda(e);
   uint8_t *dq = buf, *dk = dq + in_b, *dv = dk + in_b, *db = dv + in_b, *dout = db + beta_b, *dlse = dout + out_b,
           *dws = dlse + lse_b;
-  e = cudaMemcpyAsync(dq, q, n * 2, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(dk, k, n * 2, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(dv, v, n * 2, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(db, beta, static_cast<size_t>(H) * d * 4, cudaMemcpyHostToDevice, s);
-  int rc = map_cuda(e);
-  if (rc == FEM_OK)
-    rc = fem_fwd_ws(dq, dk, dv, reinterpret_cast<float *>(db), reinterpret_cast<float *>(dout),
-                    lse ? reinterpret_cast<float *>(dlse) : nullptr, B, H, T, d, causal, dws, ws_b, stream);
-  if (rc == FEM_OK) {
-    e = cudaMemcpyAsync(out, dout, n * 4, cudaMemcpyDeviceToHost, s);
-    if (e == cudaSuccess && lse) e = cudaMemcpyAsync(lse, dlse, rows * 4, cudaMemcpyDeviceToHost, s);
-    rc = map_cuda(e);
+  std::vector<cudaEvent_t> ev(2 * n_chunks + 2, nullptr);
+  for (auto &x : ev)
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x, cudaEventDisableTiming);
+  // the copy streams start after the allocation, in the caller's stream order
+  if (e == cudaSuccess) e = cudaEventRecord(ev[2 * n_chunks], s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(ds->copy_in, ev[2 * n_chunks], 0);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(ds->copy_out, ev[2 * n_chunks], 0);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(db, beta, static_cast<size_t>(H) * d * 4, cudaMemcpyHostToDevice, ds->copy_in);
+  rc = map_cuda(e);
+  int c = 0;
+  for (int b = 0; b < B && rc == FEM_OK; ++b) {
+    for (int h0 = 0; h0 < H && rc == FEM_OK; h0 += hc, ++c) {
+      const int nh = std::min(hc, H - h0);
+      const size_t e0 = (static_cast<size_t>(b) * H + h0) * T * d, ne = static_cast<size_t>(nh) * T * d;
+      const size_t r0 = (static_cast<size_t>(b) * H + h0) * T, nr = static_cast<size_t>(nh) * T;
+      const uint8_t *hq = static_cast<const uint8_t *>(q), *hk = static_cast<const uint8_t *>(k),
+                    *hv = static_cast<const uint8_t *>(v);
+      e = cudaMemcpyAsync(dq + e0 * 2, hq + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(dk + e0 * 2, hk + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(dv + e0 * 2, hv + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
+      if (e == cudaSuccess) e = cudaEventRecord(ev[2 * c], ds->copy_in);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[2 * c], 0);
+      rc = map_cuda(e);
+      if (rc == FEM_OK)
+        rc = fem_fwd_ws(dq + e0 * 2, dk + e0 * 2, dv + e0 * 2, reinterpret_cast<const float *>(db) + h0 * d,
+                        reinterpret_cast<float *>(dout) + e0, lse ? reinterpret_cast<float *>(dlse) + r0 : nullptr, 1,
+                        nh, T, d, causal, dws, ws_b, stream);
+      if (rc != FEM_OK) break;
+      e = cudaEventRecord(ev[2 * c + 1], s);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(ds->copy_out, ev[2 * c + 1], 0);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(out + e0, reinterpret_cast<float *>(dout) + e0, ne * 4, cudaMemcpyDeviceToHost,
+                            ds->copy_out);
+      if (e == cudaSuccess && lse)
+        e = cudaMemcpyAsync(lse + r0, reinterpret_cast<float *>(dlse) + r0, nr * 4, cudaMemcpyDeviceToHost,
+                            ds->copy_out);
+      rc = map_cuda(e);
+    }
   }
+  // the caller's stream frees the buffers once every copy out has landed
+  cudaError_t ej = cudaEventRecord(ev[2 * n_chunks + 1], ds->copy_out);
+  if (ej == cudaSuccess) ej = cudaStreamWaitEvent(s, ev[2 * n_chunks + 1], 0);
   cudaError_t ef = cudaFreeAsync(buf, s);
   cudaError_t es = cudaStreamSynchronize(s);
+  for (auto &x : ev)
+    if (x) cudaEventDestroy(x);
   if (rc != FEM_OK) return rc;
+  if (ej != cudaSuccess) return map_cuda(ej);
   if (ef != cudaSuccess) return map_cuda(ef);
   return map_cuda(es);
 }

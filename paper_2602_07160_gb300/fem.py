@@ -262,6 +262,11 @@ def fem_fwd_f32(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=N
 def fem_fwd_host(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None, device=None):
     """The read on HOST (ideally pinned) bf16 tensors: copies in, computes, copies out."""
     B, H, T, d = _check_qkvb(q, k, v, beta, torch.bfloat16, "cpu")
+    # outputs it allocates are pinned: copies into pageable memory do not overlap the read
+    if out is None:
+        out = torch.empty(q.shape, dtype=torch.float32).pin_memory()
+    if lse is None:
+        lse = torch.empty(q.shape[:3], dtype=torch.float32).pin_memory()
     out, lse = _outputs(q, out, lse, "cpu")
     dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
     rc = load().fem_fwd_host(_ptr(q), _ptr(k), _ptr(v), _ptr(beta), _ptr(out), None if lse is False else _ptr(lse),

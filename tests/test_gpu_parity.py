@@ -137,6 +137,17 @@ def test_host_entry_point_matches():
     assert torch.equal(o1.cpu(), o2) and torch.equal(l1.cpu(), l2)
 
 
+@pytest.mark.parametrize("causal", [True, False])
+def test_host_entry_point_chunks(causal):
+    """B = 3, H = 5: the host entry point copies and reads chunks of three and two heads per
+    batch element, overlapped; every chunk matches the device entry point."""
+    q, k, v, beta = W.make_custom(3, 5, 200, 64, seed=9)
+    dev = torch.device("cuda", 0)
+    o1, l1 = fem.fem_fwd(*(x.to(dev) for x in (q, k, v, beta)), causal=causal)
+    o2, l2 = fem.fem_fwd_host(q.pin_memory(), k.pin_memory(), v.pin_memory(), beta.pin_memory(), causal=causal)
+    assert torch.equal(o1.cpu(), o2) and torch.equal(l1.cpu(), l2)
+
+
 # ---------------------------------------------------------------------------
 # fp32-input path
 # ---------------------------------------------------------------------------
