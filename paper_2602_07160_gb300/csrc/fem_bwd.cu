@@ -21,22 +21,32 @@ namespace fem {
 
 constexpr int kBwdMaxPerLane = 8;  // d <= 256
 
-// For y = v - o, x = b y and the log prior weight lp = s - lse, the
+// For y = v - o, x = b y and the log prior weight lp2 = (s - lse) log2 e, the
 // p-weighted terms q = p e^x, p expm1(x)/b and p phi(x)/b^2, formed without
 // e^x alone (which can overflow where p is tiny) and continuous at b = 0.
-__device__ __forceinline__ void bwd_terms(float b, float y, float lp, float &qv, float &ds, float &dbt) {
-  const float x = b * y, p = expf(lp);
-  qv = expf(lp + x);
+// The exponentials go to the special-function unit in base 2 (relative error
+// about 2^-22); expm1(x)/b for |x| < 1/2 is y times the Taylor series of
+// expm1(x)/x (truncation below 4e-6 relative); inv_b and inv_b2 are 1/b and
+// 1/b^2 (0 at b = 0, where only the series branches are taken).
+__device__ __forceinline__ void bwd_terms(float b, float inv_b, float inv_b2, float y, float lp2, float &qv,
+                                          float &ds, float &dbt) {
+  const float x = b * y, p = ex2_approx(lp2);
+  qv = ex2_approx(fmaf(x, kLog2e, lp2));
   if (fabsf(x) < 0.5f) {
-    ds = p * (b != 0.f ? expm1f(x) / b : y);
+    float poly = fmaf(x, 1.f / 720.f, 1.f / 120.f);
+    poly = fmaf(x, poly, 1.f / 24.f);
+    poly = fmaf(x, poly, 1.f / 6.f);
+    poly = fmaf(x, poly, 0.5f);
+    poly = fmaf(x, poly, 1.f);
+    ds = p * y * poly;
   } else {
-    ds = (qv - p) / b;
+    ds = (qv - p) * inv_b;
   }
   if (fabsf(x) < 0.1f) {
     // phi(x) = x^2/2 + x^3/3 + x^4/8 + x^5/30 + x^6/144 + ..., divided by b^2
     dbt = p * y * y * fmaf(x, fmaf(x, fmaf(x, fmaf(x, 1.f / 144.f, 1.f / 30.f), 0.125f), 1.f / 3.f), 0.5f);
   } else {
-    dbt = fmaf(x - 1.f, qv, p) / (b * b);  // p phi(x) = p + (x - 1) q
+    dbt = fmaf(x - 1.f, qv, p) * inv_b2;  // p phi(x) = p + (x - 1) q
   }
 }
 
@@ -58,13 +68,14 @@ __global__ void __launch_bounds__(128) fem_bwd_kernel(const float *__restrict__ 
   const int per = (d + 31) / 32;
   const float inv_sqrt_d = rsqrtf(static_cast<float>(d));
   const size_t base = static_cast<size_t>(bh) * T * d;
-  float bj[kBwdMaxPerLane], own[kBwdMaxPerLane], own2[kBwdMaxPerLane], own3[kBwdMaxPerLane];
+  float bj[kBwdMaxPerLane], ib[kBwdMaxPerLane], own[kBwdMaxPerLane], own2[kBwdMaxPerLane], own3[kBwdMaxPerLane];
   float acc1[kBwdMaxPerLane], acc2[kBwdMaxPerLane];
 #pragma unroll
   for (int u = 0; u < kBwdMaxPerLane; ++u) {
     const int j = lane + 32 * u;
     const bool ok = u < per && j < d;
     bj[u] = ok ? beta[h * d + j] : 0.f;
+    ib[u] = bj[u] != 0.f ? 1.f / bj[u] : 0.f;
     // MODE 0: own = q_t, own2 = o_t, own3 = dout_t;  MODE 1: own = k_i, own2 = v_i
     own[u] = ok ? (MODE == 0 ? q : k)[base + static_cast<size_t>(r) * d + j] : 0.f;
     own2[u] = ok ? (MODE == 0 ? out : v)[base + static_cast<size_t>(r) * d + j] : 0.f;
@@ -77,6 +88,7 @@ __global__ void __launch_bounds__(128) fem_bwd_kernel(const float *__restrict__ 
   // rows (causal ? i : 0) .. T-1 for a key
   const int lo = MODE == 0 ? 0 : (causal ? r : 0);
   const int hi = MODE == 0 ? (causal ? r + 1 : T) : T;
+#pragma unroll 2
   for (int o = lo; o < hi; ++o) {
     const size_t ob = base + static_cast<size_t>(o) * d;
     float part = 0.f;
@@ -87,7 +99,7 @@ __global__ void __launch_bounds__(128) fem_bwd_kernel(const float *__restrict__ 
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
-    const float lp = part * inv_sqrt_d - (MODE == 0 ? lse_t : lse[bh * T + o]);  // log p_{t,i}
+    const float lp2 = (part * inv_sqrt_d - (MODE == 0 ? lse_t : lse[bh * T + o])) * kLog2e;  // log2 p_{t,i}
     float dS = 0.f;
 #pragma unroll
     for (int u = 0; u < kBwdMaxPerLane; ++u) {
@@ -97,7 +109,7 @@ __global__ void __launch_bounds__(128) fem_bwd_kernel(const float *__restrict__ 
       const float y = MODE == 0 ? v[ob + j] - own2[u] : own2[u] - out[ob + j];
       const float g = MODE == 0 ? own3[u] : dout[ob + j];
       float qv, ds, dbt;
-      bwd_terms(bj[u], y, lp, qv, ds, dbt);
+      bwd_terms(bj[u], ib[u], ib[u] * ib[u], y, lp2, qv, ds, dbt);
       dS = fmaf(g, ds, dS);
       if (MODE == 0) acc2[u] = fmaf(g, dbt, acc2[u]);  // dbeta terms of this row
       else acc2[u] = fmaf(g, qv, acc2[u]);             // dv_i: sum_t dout_{t,j} q_{t,i,j}
