@@ -20,7 +20,10 @@ def lib():
 
 
 @pytest.mark.parametrize("B,T,Hc,s_scale", [(1, 1, 8, 0.2), (2, 127, 32, 0.2), (2, 129, 64, 0.05),
-                                            (1, 1000, 48, 0.2), (4, 2000, 64, 0.01)])
+                                            (1, 1000, 48, 0.2), (4, 2000, 64, 0.01),
+                                            # 157 segments (several per combine lane) and more
+                                            # channels than a block's threads
+                                            (1, 5000, 40, 0.01), (1, 1200, 300, 0.05)])
 def test_tdc_matches_oracle(B, T, Hc, s_scale):
     g = torch.Generator().manual_seed(T + Hc)
     s = s_scale * torch.nn.functional.softplus(torch.randn((B, T, Hc), generator=g))
