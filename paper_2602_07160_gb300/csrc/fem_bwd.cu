@@ -11,15 +11,13 @@
 //
 // (sum_i p_i e^x = 1 turns KL = beta (E_q v - o) into the cancellation-free
 // sum of p phi(x) >= 0; at beta = 0 they become v - o and (v - o)^2 / 2).
-// Two passes, each one warp per row like the forward: rows (dq and dbeta,
+// Two passes, each a warp per group of consecutive rows: rows (dq and dbeta,
 // with dS_{t,i} = sum_j dout_{t,j} dF_{t,j}/ds_{t,i}), then keys (dk and dv,
 // summing over the rows that see the key).
 #include "fem_common.cuh"
 #include "fem_launch.h"
 
 namespace fem {
-
-constexpr int kBwdMaxPerLane = 8;  // d <= 256
 
 // For y = v - o, x = b y and the log prior weight lp2 = (s - lse) log2 e, the
 // p-weighted terms q = p e^x, p expm1(x)/b and p phi(x)/b^2, formed without
@@ -50,100 +48,146 @@ __device__ __forceinline__ void bwd_terms(float b, float inv_b, float inv_b2, fl
   }
 }
 
-// MODE 0: one warp per query row t -> dq_t and the row's dbeta terms.
-// MODE 1: one warp per key row i  -> dk_i and dv_i.
-template <int MODE>
+// MODE 0: a warp per R consecutive query rows t -> dq_t and the rows' dbeta terms.
+// MODE 1: a warp per R consecutive key rows i  -> dk_i and dv_i.
+// Lane l holds channels l + 32 u (u < PER); the R rows share every load of
+// the other side's row and their butterfly sums interleave.
+template <int MODE, int R, int PER>
 __global__ void __launch_bounds__(128) fem_bwd_kernel(const float *__restrict__ q, const float *__restrict__ k,
                                                        const float *__restrict__ v, const float *__restrict__ beta,
                                                        const float *__restrict__ out, const float *__restrict__ lse,
                                                        const float *__restrict__ dout, float *__restrict__ da,
                                                        float *__restrict__ db, float *__restrict__ dbeta, int H,
-                                                       int T, int d, int causal, long long n_rows) {
+                                                       int T, int d, int causal, long long n_groups) {
   const int lane = threadIdx.x & 31;
-  const long long row = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (row >= n_rows) return;
-  const long long bh = row / T;
-  const int r = static_cast<int>(row % T);
+  const long long grp = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (grp >= n_groups) return;
+  const int gpb = (T + R - 1) / R;  // row groups per (b, h)
+  const long long bh = grp / gpb;
+  const int r0 = static_cast<int>(grp % gpb) * R;
+  const int nr = min(R, T - r0);  // rows of this group
   const int h = static_cast<int>(bh % H);
-  const int per = (d + 31) / 32;
   const float inv_sqrt_d = rsqrtf(static_cast<float>(d));
   const size_t base = static_cast<size_t>(bh) * T * d;
-  float bj[kBwdMaxPerLane], ib[kBwdMaxPerLane], own[kBwdMaxPerLane], own2[kBwdMaxPerLane], own3[kBwdMaxPerLane];
-  float acc1[kBwdMaxPerLane], acc2[kBwdMaxPerLane];
+  float bj[PER], ib[PER];
+  float own[R][PER], own2[R][PER], own3[R][PER], acc1[R][PER], acc2[R][PER], lse_r[R];
 #pragma unroll
-  for (int u = 0; u < kBwdMaxPerLane; ++u) {
+  for (int u = 0; u < PER; ++u) {
     const int j = lane + 32 * u;
-    const bool ok = u < per && j < d;
-    bj[u] = ok ? beta[h * d + j] : 0.f;
+    bj[u] = j < d ? beta[h * d + j] : 0.f;
     ib[u] = bj[u] != 0.f ? 1.f / bj[u] : 0.f;
-    // MODE 0: own = q_t, own2 = o_t, own3 = dout_t;  MODE 1: own = k_i, own2 = v_i
-    own[u] = ok ? (MODE == 0 ? q : k)[base + static_cast<size_t>(r) * d + j] : 0.f;
-    own2[u] = ok ? (MODE == 0 ? out : v)[base + static_cast<size_t>(r) * d + j] : 0.f;
-    own3[u] = ok && MODE == 0 ? dout[base + static_cast<size_t>(r) * d + j] : 0.f;
-    acc1[u] = 0.f;
-    acc2[u] = 0.f;
   }
-  const float lse_t = MODE == 0 ? lse[bh * T + r] : 0.f;
-  // the other side of the score: keys 0 .. (causal ? t : T-1) for a row,
-  // rows (causal ? i : 0) .. T-1 for a key
-  const int lo = MODE == 0 ? 0 : (causal ? r : 0);
-  const int hi = MODE == 0 ? (causal ? r + 1 : T) : T;
-#pragma unroll 2
+#pragma unroll
+  for (int w = 0; w < R; ++w) {
+    const int r = min(r0 + w, T - 1);  // rows past T repeat the last one; their results are not stored
+    lse_r[w] = MODE == 0 ? lse[bh * T + r] : 0.f;
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int j = lane + 32 * u;
+      const bool ok = j < d;
+      // MODE 0: own = q_t, own2 = o_t, own3 = dout_t;  MODE 1: own = k_i, own2 = v_i
+      own[w][u] = ok ? (MODE == 0 ? q : k)[base + static_cast<size_t>(r) * d + j] : 0.f;
+      own2[w][u] = ok ? (MODE == 0 ? out : v)[base + static_cast<size_t>(r) * d + j] : 0.f;
+      own3[w][u] = ok && MODE == 0 ? dout[base + static_cast<size_t>(r) * d + j] : 0.f;
+      acc1[w][u] = 0.f;
+      acc2[w][u] = 0.f;
+    }
+  }
+  // the other side of the score: keys 0 .. (causal ? last row : T-1) for rows,
+  // rows (causal ? first key : 0) .. T-1 for keys
+  const int lo = MODE == 0 ? 0 : (causal ? r0 : 0);
+  const int hi = MODE == 0 ? (causal ? r0 + nr : T) : T;
   for (int o = lo; o < hi; ++o) {
     const size_t ob = base + static_cast<size_t>(o) * d;
-    float part = 0.f;
+    float oth[PER], oth2[PER], oth3[PER];
 #pragma unroll
-    for (int u = 0; u < kBwdMaxPerLane; ++u) {
+    for (int u = 0; u < PER; ++u) {
       const int j = lane + 32 * u;
-      if (u < per && j < d) part = fmaf(own[u], (MODE == 0 ? k : q)[ob + j], part);
+      const bool ok = j < d;
+      oth[u] = ok ? (MODE == 0 ? k : q)[ob + j] : 0.f;
+      oth2[u] = ok ? (MODE == 0 ? v : out)[ob + j] : 0.f;
+      oth3[u] = ok && MODE == 1 ? dout[ob + j] : 0.f;
+    }
+    const float lse_o = MODE == 1 ? lse[bh * T + o] : 0.f;
+    float part[R];
+#pragma unroll
+    for (int w = 0; w < R; ++w) {
+      part[w] = 0.f;
+#pragma unroll
+      for (int u = 0; u < PER; ++u) part[w] = fmaf(own[w][u], oth[u], part[w]);
     }
 #pragma unroll
-    for (int off = 16; off; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
-    const float lp2 = (part * inv_sqrt_d - (MODE == 0 ? lse_t : lse[bh * T + o])) * kLog2e;  // log2 p_{t,i}
-    float dS = 0.f;
+    for (int off = 16; off; off >>= 1)
 #pragma unroll
-    for (int u = 0; u < kBwdMaxPerLane; ++u) {
-      const int j = lane + 32 * u;
-      if (!(u < per && j < d)) continue;
-      // y = v_{i,j} - o_{t,j} with (i, t) = (o, r) for rows and (r, o) for keys
-      const float y = MODE == 0 ? v[ob + j] - own2[u] : own2[u] - out[ob + j];
-      const float g = MODE == 0 ? own3[u] : dout[ob + j];
-      float qv, ds, dbt;
-      bwd_terms(bj[u], ib[u], ib[u] * ib[u], y, lp2, qv, ds, dbt);
-      dS = fmaf(g, ds, dS);
-      if (MODE == 0) acc2[u] = fmaf(g, dbt, acc2[u]);  // dbeta terms of this row
-      else acc2[u] = fmaf(g, qv, acc2[u]);             // dv_i: sum_t dout_{t,j} q_{t,i,j}
+      for (int w = 0; w < R; ++w) part[w] += __shfl_xor_sync(0xffffffffu, part[w], off);
+    float dS[R];
+#pragma unroll
+    for (int w = 0; w < R; ++w) {
+      // the pair (query row, key) is visible: key <= row when causal
+      const int rw = r0 + w;
+      const bool vis = !causal || (MODE == 0 ? o <= rw : rw <= o);
+      const float lp2 = vis ? (part[w] * inv_sqrt_d - (MODE == 0 ? lse_r[w] : lse_o)) * kLog2e : -INFINITY;
+      dS[w] = 0.f;
+#pragma unroll
+      for (int u = 0; u < PER; ++u) {
+        // y = v_{i,j} - o_{t,j} with (i, t) = (o, row) for rows and (row, o) for keys
+        const float y = MODE == 0 ? oth2[u] - own2[w][u] : own2[w][u] - oth2[u];
+        const float g = MODE == 0 ? own3[w][u] : oth3[u];
+        float qv, ds, dbt;
+        bwd_terms(bj[u], ib[u], ib[u] * ib[u], y, lp2, qv, ds, dbt);
+        dS[w] = fmaf(g, ds, dS[w]);
+        if (MODE == 0) acc2[w][u] = fmaf(g, dbt, acc2[w][u]);  // dbeta terms of this row
+        else acc2[w][u] = fmaf(g, qv, acc2[w][u]);             // dv_i: sum_t dout_{t,j} q_{t,i,j}
+      }
     }
 #pragma unroll
-    for (int off = 16; off; off >>= 1) dS += __shfl_xor_sync(0xffffffffu, dS, off);
+    for (int off = 16; off; off >>= 1)
 #pragma unroll
-    for (int u = 0; u < kBwdMaxPerLane; ++u) {
-      const int j = lane + 32 * u;
-      if (u < per && j < d) acc1[u] = fmaf(dS, (MODE == 0 ? k : q)[ob + j], acc1[u]);
-    }
+      for (int w = 0; w < R; ++w) dS[w] += __shfl_xor_sync(0xffffffffu, dS[w], off);
+#pragma unroll
+    for (int w = 0; w < R; ++w)
+#pragma unroll
+      for (int u = 0; u < PER; ++u) acc1[w][u] = fmaf(dS[w], oth[u], acc1[w][u]);
   }
 #pragma unroll
-  for (int u = 0; u < kBwdMaxPerLane; ++u) {
-    const int j = lane + 32 * u;
-    if (!(u < per && j < d)) continue;
-    da[base + static_cast<size_t>(r) * d + j] = acc1[u] * inv_sqrt_d;
-    if (MODE == 0) atomicAdd(&dbeta[h * d + j], acc2[u]);
-    else db[base + static_cast<size_t>(r) * d + j] = acc2[u];
+  for (int w = 0; w < R; ++w) {
+    if (w >= nr) break;
+    const int r = r0 + w;
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int j = lane + 32 * u;
+      if (j >= d) continue;
+      da[base + static_cast<size_t>(r) * d + j] = acc1[w][u] * inv_sqrt_d;
+      if (MODE == 0) atomicAdd(&dbeta[h * d + j], acc2[w][u]);
+      else db[base + static_cast<size_t>(r) * d + j] = acc2[w][u];
+    }
   }
+}
+
+template <int R, int PER>
+static cudaError_t launch_bwd_rp(const float *q, const float *k, const float *v, const float *beta, const float *out,
+                                 const float *lse, const float *dout, float *dq, float *dk, float *dv, float *dbeta,
+                                 int B, int H, int T, int d, int causal, cudaStream_t stream) {
+  const long long n_groups = static_cast<long long>(B) * H * ((T + R - 1) / R);
+  const unsigned blocks = static_cast<unsigned>((n_groups + 3) / 4);
+  fem_bwd_kernel<0, R, PER><<<blocks, 128, 0, stream>>>(q, k, v, beta, out, lse, dout, dq, nullptr, dbeta, H, T, d,
+                                                        causal, n_groups);
+  fem_bwd_kernel<1, R, PER><<<blocks, 128, 0, stream>>>(q, k, v, beta, out, lse, dout, dk, dv, nullptr, H, T, d,
+                                                        causal, n_groups);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_bwd_f32(const float *q, const float *k, const float *v, const float *beta, const float *out,
                            const float *lse, const float *dout, float *dq, float *dk, float *dv, float *dbeta, int B,
                            int H, int T, int d, int causal, cudaStream_t stream) {
-  const long long n_rows = static_cast<long long>(B) * H * T;
-  const unsigned blocks = static_cast<unsigned>((n_rows + 3) / 4);
   cudaError_t e = cudaMemsetAsync(dbeta, 0, static_cast<size_t>(H) * d * sizeof(float), stream);
   if (e != cudaSuccess) return e;
-  fem_bwd_kernel<0><<<blocks, 128, 0, stream>>>(q, k, v, beta, out, lse, dout, dq, nullptr, dbeta, H, T, d, causal,
-                                                n_rows);
-  fem_bwd_kernel<1><<<blocks, 128, 0, stream>>>(q, k, v, beta, out, lse, dout, dk, dv, nullptr, H, T, d, causal,
-                                                n_rows);
-  return cudaGetLastError();
+  // rows per warp: four while a lane holds at most two channels, fewer beyond
+  if (d <= 32) return launch_bwd_rp<4, 1>(q, k, v, beta, out, lse, dout, dq, dk, dv, dbeta, B, H, T, d, causal, stream);
+  if (d <= 64) return launch_bwd_rp<4, 2>(q, k, v, beta, out, lse, dout, dq, dk, dv, dbeta, B, H, T, d, causal, stream);
+  if (d <= 128) return launch_bwd_rp<2, 4>(q, k, v, beta, out, lse, dout, dq, dk, dv, dbeta, B, H, T, d, causal, stream);
+  if (d <= 256) return launch_bwd_rp<1, 8>(q, k, v, beta, out, lse, dout, dq, dk, dv, dbeta, B, H, T, d, causal, stream);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace fem

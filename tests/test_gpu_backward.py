@@ -21,7 +21,9 @@ def lib():
 
 
 @pytest.mark.parametrize("B,H,T,d,causal", [(1, 2, 1, 16, True), (2, 2, 33, 32, True), (1, 2, 100, 64, False),
-                                            (2, 1, 257, 128, True), (1, 3, 150, 64, True)])
+                                            (2, 1, 257, 128, True), (1, 3, 150, 64, True),
+                                            # channels not a multiple of 32 per lane, and d > 128
+                                            (1, 2, 65, 96, False), (1, 1, 70, 200, True)])
 def test_backward_matches_oracle(B, H, T, d, causal):
     q, k, v, beta = W.make_custom(B, H, T, d, dtype="f32", seed=T + d)
     beta[0, :2] = 0.0
