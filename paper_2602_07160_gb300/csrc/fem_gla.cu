@@ -24,8 +24,8 @@
 // from its start state, writing the outputs.  Within a segment four lanes
 // share a channel, each keeping a quarter of its m-float state in registers
 // (a warp holds 7 channels and the constant channel), and the block stages
-// qf, kf, exp(g), g and v for kGlaSteps steps in shared memory.  fp32 on CUDA
-// cores.
+// qf, kf, g and v for kGlaSteps steps in shared memory, in two buffers filled
+// by asynchronous copies one stage ahead.  fp32 on CUDA cores.
 #include "fem_common.cuh"
 #include "fem_launch.h"
 
@@ -36,6 +36,12 @@ constexpr int kGlaParts = 4;                          // lanes per channel
 constexpr int kGlaChPerWarp = 32 / kGlaParts - 1;     // real channels per warp (the 8th is the normaliser)
 constexpr int kGlaMaxD = 155;
 constexpr int kGlaMaxWarps = (kGlaMaxD + kGlaChPerWarp - 1) / kGlaChPerWarp;
+
+__device__ __forceinline__ void cp_async4(float *dst, const float *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // Per-lane role within a block of one (b, h).
 struct GlaLane {
@@ -65,11 +71,13 @@ __global__ void __launch_bounds__(32 * kGlaMaxWarps) gla_seg_kernel(
     const float *__restrict__ logdecay, const float *__restrict__ beta, float *__restrict__ out,
     float *__restrict__ logz, int H, int T, int d, int seg_len, float *__restrict__ state, float *__restrict__ phi) {
   constexpr int MP = M / kGlaParts;  // state floats per lane
-  __shared__ __align__(16) float s_q[kGlaSteps][M];
-  __shared__ __align__(16) float s_k[kGlaSteps][M];
-  __shared__ float s_v[kGlaSteps][kGlaMaxD];
+  // the staged inputs in two buffers: the next stage's copies land while this one runs
+  __shared__ __align__(16) float s_q[2][kGlaSteps][M];
+  __shared__ __align__(16) float s_k[2][kGlaSteps][M];
+  __shared__ float s_v[2][kGlaSteps][kGlaMaxD];
+  __shared__ float s_g[2][kGlaSteps];
   __shared__ float s_o[kGlaSteps][kGlaMaxD];
-  __shared__ float s_a[kGlaSteps], s_g[kGlaSteps], s_lz[kGlaSteps];
+  __shared__ float s_a[kGlaSteps], s_lz[kGlaSteps];
   const int tid = threadIdx.x, p = blockIdx.x, n_seg = gridDim.x, bh = blockIdx.y, h = bh % H;
   const GlaLane L = gla_lane(beta, h, d);
   const size_t row0 = static_cast<size_t>(bh) * T;
@@ -86,21 +94,30 @@ __global__ void __launch_bounds__(32 * kGlaMaxWarps) gla_seg_kernel(
     lam = st[MP];
   }
   float phi_acc = 0.f;
-  for (int t0 = t_begin; t0 < t_end; t0 += kGlaSteps) {
+  // a stage's inputs by asynchronous 4-byte copies (any d), one commit group per stage
+  auto stage = [&](int ts, int buf) {
+    const int ns = min(kGlaSteps, t_end - ts);
+    for (int e = tid; e < ns * M; e += blockDim.x) {
+      cp_async4(&s_q[buf][e / M][e % M], qf + (row0 + ts) * M + e);
+      cp_async4(&s_k[buf][e / M][e % M], kf + (row0 + ts) * M + e);
+    }
+    for (int e = tid; e < ns * d; e += blockDim.x) cp_async4(&s_v[buf][e / d][e % d], v + (row0 + ts) * d + e);
+    for (int e = tid; e < ns; e += blockDim.x) cp_async4(&s_g[buf][e], logdecay + row0 + ts + e);
+    cp_async_commit();
+  };
+  if (t_begin < t_end) stage(t_begin, 0);
+  int buf = 0;
+  for (int t0 = t_begin; t0 < t_end; t0 += kGlaSteps, buf ^= 1) {
     const int n = min(kGlaSteps, t_end - t0);
-    for (int e = tid; e < n * M; e += blockDim.x) {
-      s_q[e / M][e % M] = qf[(row0 + t0) * M + e];
-      s_k[e / M][e % M] = kf[(row0 + t0) * M + e];
-    }
-    for (int e = tid; e < n * d; e += blockDim.x) s_v[e / d][e % d] = v[(row0 + t0) * d + e];
-    for (int e = tid; e < n; e += blockDim.x) {
-      const float g = logdecay[row0 + t0 + e];
-      s_g[e] = g;
-      s_a[e] = expf(g);
-    }
+    // this stage's copies have landed, and every thread is done with the
+    // previous stage (whose buffer the next prefetch overwrites)
+    cp_async_wait_all();
+    __syncthreads();
+    if (t0 + kGlaSteps < t_end) stage(t0 + kGlaSteps, buf ^ 1);
+    for (int e = tid; e < n; e += blockDim.x) s_a[e] = expf(s_g[buf][e]);
     __syncthreads();
     for (int u = 0; u < n; ++u) {
-      const float x = L.real ? s_v[u][L.j] : 0.f;
+      const float x = L.real ? s_v[buf][u][L.j] : 0.f;
       float E, a;
       if (!L.real) {
         E = 1.f;
@@ -109,15 +126,15 @@ __global__ void __launch_bounds__(32 * kGlaMaxWarps) gla_seg_kernel(
         E = x;
         a = s_a[u];
       } else {
-        const float le = L.b * x, lo = lam + s_g[u];
+        const float le = L.b * x, lo = lam + s_g[buf][u];
         const float ln = fmaxf(lo, le);
         a = expf(lo - ln);  // 0 on the first step of a zero state
         E = expf(le - ln);
         lam = ln;
       }
-      if (MODE == 0) phi_acc += s_g[u];
-      const float4 *k4 = reinterpret_cast<const float4 *>(&s_k[u][L.part * MP]);
-      const float4 *q4 = reinterpret_cast<const float4 *>(&s_q[u][L.part * MP]);
+      if (MODE == 0) phi_acc += s_g[buf][u];
+      const float4 *k4 = reinterpret_cast<const float4 *>(&s_k[buf][u][L.part * MP]);
+      const float4 *q4 = reinterpret_cast<const float4 *>(&s_q[buf][u][L.part * MP]);
       float n0 = 0.f, n1 = 0.f;
 #pragma unroll
       for (int i4 = 0; i4 < MP / 4; ++i4) {
@@ -143,8 +160,8 @@ __global__ void __launch_bounds__(32 * kGlaMaxWarps) gla_seg_kernel(
         if (L.warp == 0 && L.lane == kGlaChPerWarp * kGlaParts) s_lz[u] = logf(den);
       }
     }
-    __syncthreads();  // the staged inputs are consumed (and the steps' outputs are in shared memory)
     if (MODE == 1) {
+      __syncthreads();  // the steps' outputs are in shared memory
       for (int e = tid; e < n * d; e += blockDim.x) out[(row0 + t0) * d + e] = s_o[e / d][e % d];
       if (logz)
         for (int e = tid; e < n; e += blockDim.x) logz[row0 + t0 + e] = s_lz[e];
