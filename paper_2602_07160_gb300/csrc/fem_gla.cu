@@ -214,13 +214,34 @@ __global__ void __launch_bounds__(32 * kGlaMaxWarps) gla_combine_kernel(const fl
   }
 }
 
+// Resident blocks per SM of the output pass (the heavier of the two passes).
+static int gla_blocks_per_sm(int m, int threads) {
+  int n = 0;
+  cudaError_t e = cudaErrorInvalidValue;
+  if (m == 16) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gla_seg_kernel<16, 1>, threads, 0);
+  if (m == 32) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gla_seg_kernel<32, 1>, threads, 0);
+  if (m == 64) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gla_seg_kernel<64, 1>, threads, 0);
+  return e == cudaSuccess && n > 0 ? n : 1;
+}
+
 size_t gla_workspace_bytes(int BH, int T, int m, int d, int num_sms, int *seg_len_out, int *n_seg_out) {
   const int warps = (d + kGlaChPerWarp - 1) / kGlaChPerWarp;
-  // about sixteen warps per SM scheduler across the grid (the scan is
-  // latency-bound), segments of at least 64 steps
-  const int want = max(1, (64 * num_sms + BH * warps - 1) / (BH * warps));
+  // Segments of at least 64 steps.  A pass takes about (waves of resident
+  // blocks) x (segment length) steps of time, so the count minimises that
+  // product: whole waves of the grid, not a fraction of a last one.
+  const long long cap = static_cast<long long>(gla_blocks_per_sm(m, 32 * warps)) * num_sms;
   const int max_seg = max(1, (T + 63) / 64);
-  const int n_seg0 = min(want, max_seg);
+  int n_seg0 = 1;
+  long long best = -1;
+  for (int ns = 1; ns <= max_seg; ++ns) {
+    const long long waves = (static_cast<long long>(BH) * ns + cap - 1) / cap;
+    const long long cost = waves * ((T + ns - 1) / ns);
+    if (best < 0 || cost < best) {
+      best = cost;
+      n_seg0 = ns;
+    }
+    if (waves > 4) break;
+  }
   const int seg_len = (T + n_seg0 - 1) / n_seg0;
   const int n_seg = (T + seg_len - 1) / seg_len;
   if (seg_len_out) *seg_len_out = seg_len;
