@@ -131,7 +131,7 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += causal ? round256(BH * n_kt * kBlockQ * sizeof(FixupEntry)) : 0;
   w->tilefix = off;
   off += causal ? round256(BH * n_kt * sizeof(int2)) : 0;
-  w->count = off;  // fix-up slots, fix-up rows
+  w->count = off;  // fix-up slots, fix-up rows, the fix-up's chunk counter
   off += 256;
   w->total = off;
   return true;
@@ -218,6 +218,7 @@ static BankWorkspace bank_workspace(uint8_t *ws, const WsLayout &w, int causal) 
   bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
   bw.fixup_rows = reinterpret_cast<int *>(ws + w.count) + 1;
+  bw.fixup_next = reinterpret_cast<int *>(ws + w.count) + 2;
   bw.tilefix = causal ? reinterpret_cast<int2 *>(ws + w.tilefix) : nullptr;
   return bw;
 }
@@ -255,9 +256,9 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
     gate = TcGate{ga->lam, ga->g, ga->mu_side, bw0.chan};
   }
 
-  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 2 * sizeof(int), s);
+  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 3 * sizeof(int), s);
   // the mean's bank (every channel linear at beta = 0: v - c with c the channel mean)
-  if (e == cudaSuccess && ga) e = cudaMemsetAsync(bw0.fixup_count, 0, 2 * sizeof(int), s);
+  if (e == cudaSuccess && ga) e = cudaMemsetAsync(bw0.fixup_count, 0, 3 * sizeof(int), s);
   if (e == cudaSuccess && ga)
     e = launch_value_bank(v, tv, te0, ga->zero_beta, BH, H, T, d, 0, bw0, ds->err, ds->num_sms, s);
   if (ga) bw.tstat = bw0.tstat;  // the tiles' statistics do not depend on beta
@@ -273,7 +274,7 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
   if (e == cudaSuccess) {
     if (causal)
       e = launch_fixup(q, k, v, beta, bw.shift, out, H, T, d, bw.fixups, bw.fixup_count, bw.fixup_rows,
-                       ds->last_fixup, ga ? &gate : nullptr, ds->num_sms, s);
+                       bw.fixup_next, ds->last_fixup, ga ? &gate : nullptr, ds->num_sms, s);
     else
       e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
   }

@@ -20,7 +20,8 @@
 //
 // Entries come in chunks of 8 consecutive rows of one diagonal tile (the
 // pre-pass pads each tile's entries to a multiple of 8 with rows -1).  One
-// 256-thread block takes a chunk at a time (grid-stride): it stages the tile's
+// 256-thread block takes a chunk at a time, claimed from a counter so that
+// blocks that drew cheap chunks take more of them: it stages the tile's
 // K and V rows k0 .. k0+r_max and the chunk's 8 query rows in shared memory,
 // scores the 8 rows against the keys with warp-level bf16 MMAs (16 keys per
 // warp, fp32 accumulation), then each warp completes one entry: its lanes
@@ -87,6 +88,7 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
                                                             int H, int T, const FixupEntry *__restrict__ entries,
                                                             const int *__restrict__ count,
                                                             const int *__restrict__ rows_listed,
+                                                            int *__restrict__ next_chunk,
                                                             int *__restrict__ last_rows, TcGate gate) {
   // staged row strides in bf16 elements: K and Q rows 16-byte aligned for
   // ldmatrix with consecutive rows four banks apart; V rows an odd number of
@@ -97,21 +99,26 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
   __nv_bfloat16 *sV = sK + kBlockK * KS;
   __nv_bfloat16 *sQ = sV + kBlockK * VS;  // 16 rows (8 entries, 8 unused) of KS
   __shared__ float sS[kFixChunk][kBlockK];  // the chunk's scores, log2 units
-  __shared__ int s_nk;
+  __shared__ int s_nk, s_ch;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_chunks = *count / kFixChunk;
   if (blockIdx.x == 0 && tid == 0 && last_rows) *last_rows = *rows_listed;
   const float scale = kLog2e * rsqrtf(static_cast<float>(D));
   const int n_kt = (T + kBlockK - 1) / kBlockK;
 
-  for (int ch = blockIdx.x; ch < n_chunks; ch += gridDim.x) {
+  for (;;) {
+    if (tid == 0) {
+      s_ch = atomicAdd(next_chunk, 1);
+      s_nk = 0;
+    }
+    __syncthreads();
+    const int ch = s_ch;
+    if (ch >= n_chunks) break;
     const FixupEntry ent = entries[ch * kFixChunk + warp];
     const int row0 = entries[ch * kFixChunk].row;  // the chunk's first entry is a real row
     const int bh = row0 / T, h = bh % H;
     const int kt = (row0 % T) / kBlockK, k0 = kt * kBlockK;
     const int r = ent.row >= 0 ? ent.row - bh * T - k0 : -1;  // this warp's row in the tile
-    if (tid == 0) s_nk = 0;
-    __syncthreads();
     if (lane == 0 && r >= 0) atomicMax(&s_nk, r + 1);
     __syncthreads();
     const int nk = s_nk;  // keys k0 .. k0+nk-1 serve every row of the chunk
@@ -242,7 +249,8 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
 
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
                          float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
-                         const int *rows, int *last_rows, const TcGate *gate, int num_sms, cudaStream_t stream) {
+                         const int *rows, int *next_chunk, int *last_rows, const TcGate *gate, int num_sms,
+                         cudaStream_t stream) {
   const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr};
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
@@ -250,14 +258,14 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
   if (d == 64) {
     const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
     fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
-                                                          last_rows, g);
+                                                          next_chunk, last_rows, g);
   } else if (d == 128) {
     const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
     cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     fixup_kernel<128><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
-                                                           last_rows, g);
+                                                           next_chunk, last_rows, g);
   } else {
     return cudaErrorInvalidValue;
   }

@@ -20,6 +20,7 @@ struct BankWorkspace {
   FixupEntry *fixups;       // exact-recompute list (causal)
   int *fixup_count;         // its length in slots, a multiple of 8 (zeroed before the pre-pass)
   int *fixup_rows;          // rows listed (zeroed before the pre-pass)
+  int *fixup_next;          // the fix-up's next unclaimed chunk (zeroed before the pre-pass)
   int2 *tilefix;            // [B*H, key tiles] (causal): {first entry, number of rows} of the tile's
                             // entries, which list the tile's rows 0 .. number-1 in order
 };
@@ -66,9 +67,11 @@ cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const
 // key tiles.
 // gate: nullptr, or the one-pass gated read's gates (the entries' outputs are
 // then gated with the mu the tensor-core kernel left in gate->mu_side).
+// next_chunk: a zeroed counter from which the blocks claim chunks of entries.
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
                          float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
-                         const int *rows, int *last_rows, const TcGate *gate, int num_sms, cudaStream_t stream);
+                         const int *rows, int *next_chunk, int *last_rows, const TcGate *gate, int num_sms,
+                         cudaStream_t stream);
 
 
 // Decode read of one query per (b, h) against T cached keys: per-CTA key-chunk
