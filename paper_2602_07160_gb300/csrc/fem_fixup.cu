@@ -72,6 +72,20 @@ __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// Asynchronous global -> shared copies (16 bytes: both addresses 16-byte
+// aligned; 4 bytes: both 4-byte aligned), so that every staged row is in
+// flight at once.
+__device__ __forceinline__ void fix_cp16(uint32_t dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void fix_cp4(uint32_t dst, const void *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void fix_cp_wait_all() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
 // log2(2^a + 2^b) for a, b possibly -inf
 __device__ __forceinline__ float lse2_pair(float a, float b) {
   const float mx = fmaxf(a, b);
@@ -125,14 +139,10 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
     for (int idx = tid; idx < nk * (D / 8); idx += kFixThreads) {
       const int i = idx / (D / 8), c = idx % (D / 8);
       const size_t g = (static_cast<size_t>(bh) * T + k0 + i) * D + 8 * c;
-      const uint4 kr = *reinterpret_cast<const uint4 *>(k + g);
-      const uint4 vr = *reinterpret_cast<const uint4 *>(v + g);
-      *reinterpret_cast<uint4 *>(sK + i * KS + 8 * c) = kr;
-      uint32_t *dv = reinterpret_cast<uint32_t *>(sV + i * VS + 8 * c);
-      dv[0] = vr.x;
-      dv[1] = vr.y;
-      dv[2] = vr.z;
-      dv[3] = vr.w;
+      fix_cp16(smem_u32(sK + i * KS + 8 * c), k + g);
+      const uint32_t dv = smem_u32(sV + i * VS + 8 * c);
+#pragma unroll
+      for (int w = 0; w < 4; ++w) fix_cp4(dv + 4 * w, v + g + 2 * w);
     }
     for (int idx = tid; idx < kFixChunk * (D / 8); idx += kFixThreads) {
       const int w = idx / (D / 8), c = idx % (D / 8);
@@ -140,6 +150,7 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
       *reinterpret_cast<uint4 *>(sQ + w * KS + 8 * c) =
           erow >= 0 ? *reinterpret_cast<const uint4 *>(q + static_cast<size_t>(erow) * D + 8 * c) : make_uint4(0, 0, 0, 0);
     }
+    fix_cp_wait_all();
     __syncthreads();
     // S[8 x nk] = Q K^T: warp w takes keys 16w .. 16w+15 (two n8 blocks) over
     // D/16 k-steps of m16n8k16 (rows 8..15 of A are unused)
