@@ -134,6 +134,18 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
     const int kt = (row0 % T) / kBlockK, k0 = kt * kBlockK;
     const int r = ent.row >= 0 ? ent.row - bh * T - k0 : -1;  // this warp's row in the tile
     if (lane == 0 && r >= 0) atomicMax(&s_nk, r + 1);
+    // the entry's stashed accumulators over the earlier key tiles, the
+    // previous tile's shifts and beta, lane l holding channels l + 32 g: loaded
+    // now so that they arrive while the chunk's rows are staged and scored
+    float a_reg[D / 32], c_reg[D / 32], b_reg[D / 32];
+#pragma unroll
+    for (int gi = 0; gi < D / 32; ++gi) {
+      const int j = lane + 32 * gi;
+      const bool listed = r >= 0 && ent.mask[gi];
+      a_reg[gi] = listed ? out[static_cast<size_t>(ent.row) * D + j] : 0.f;
+      c_reg[gi] = (listed && kt > 0) ? shift[(static_cast<size_t>(bh) * n_kt + kt - 1) * D + j] : 0.f;
+      b_reg[gi] = beta[h * D + j];
+    }
     __syncthreads();
     const int nk = s_nk;  // keys k0 .. k0+nk-1 serve every row of the chunk
     for (int idx = tid; idx < nk * (D / 8); idx += kFixThreads) {
@@ -192,17 +204,7 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
       sm = warp_sum(sm);
       const float L = lse2_pair(ent.l_pre > 0.f ? ent.m_pre + log2f(ent.l_pre) : -INFINITY, mx + log2f(sm));
       // each listed channel's tilted log-sum-exp, merged with the tensor-core
-      // kernel's state over the earlier key tiles: the row's stashed
-      // accumulators, the previous tile's shifts and beta, lane l holding
-      // channels l + 32 g, all loaded at once
-      float a_reg[D / 32], c_reg[D / 32], b_reg[D / 32];
-#pragma unroll
-      for (int gi = 0; gi < D / 32; ++gi) {
-        const int j = lane + 32 * gi;
-        a_reg[gi] = ent.mask[gi] ? out[static_cast<size_t>(ent.row) * D + j] : 0.f;
-        c_reg[gi] = (ent.mask[gi] && kt > 0) ? shift[(static_cast<size_t>(bh) * n_kt + kt - 1) * D + j] : 0.f;
-        b_reg[gi] = beta[h * D + j];
-      }
+      // kernel's state over the earlier key tiles (a_reg, c_reg, b_reg)
 #pragma unroll
       for (int gi = 0; gi < D / 32; ++gi) {
         unsigned m = ent.mask[gi];
