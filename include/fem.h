@@ -61,7 +61,9 @@ typedef enum {
  * library keeps per device (freed memory stays in the pool for the next
  * call; the entry points that allocate all use it).  Accuracy: the score contraction takes bf16 q, k; the second
  * contraction takes the prior weights and the per-channel value bank in fp16
- * (11-bit significand); both accumulate in fp32.
+ * (11-bit significand); both accumulate in fp32.  Every output whose 16-bit
+ * operands could have lost more than 2^-7 to underflow is recomputed
+ * exactly in fp32, so the result holds for any prior (peaked or flat).
  */
 int fem_fwd(const void *q, const void *k, const void *v, const float *beta,
             float *out, float *lse, int B, int H, int T, int d, int causal,
@@ -115,14 +117,15 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
  * every input and output.  Instead of a stream-ordered allocation it uses a fixed
  * 16 MiB scratch array compiled into the library, which every GPU that
  * loads the library holds until the process exits.  Problems needing more
- * workspace than that (fem_fwd_workspace_bytes() > 16 MiB, about 2*d + 60
- * bytes per row (b, h, t) for a causal read) return FEM_ERR_NO_MEMORY before
- * anything is enqueued.  It calls no allocation routine.  The first call on
- * a device looks up the scratch address on that device (cudaGetSymbolAddress),
- * so make that first call outside any stream capture.  All calls share the one
- * array and it keeps the previous call's contents (the call clears what must
- * start at zero): calls that overlap on the GPU, from any stream or thread,
- * race and must be serialised by the caller.
+ * workspace than that (fem_fwd_workspace_bytes() > 16 MiB, about 2*d + 80
+ * bytes per row (b, h, t)) return FEM_ERR_NO_MEMORY before anything is
+ * enqueued.  It calls no allocation routine and creates no memory pool.  The
+ * first call on a device looks up the scratch address and the library's
+ * per-device error word on that device (cudaGetSymbolAddress), so make that
+ * first call outside any stream capture.  All calls share the one array and
+ * it keeps the previous call's contents (the call clears what must start at
+ * zero): calls that overlap on the GPU, from any stream or thread, race and
+ * must be serialised by the caller.
  */
 int fem_fwd_noalloc(const void *q, const void *k, const void *v,
                     const float *beta, float *out, float *lse, int B, int H,
@@ -243,8 +246,10 @@ int fem_check_device_error(void *stream);
 /*
  * fem_last_fixup_rows -- synchronises `stream` and returns the number of rows
  * the last bf16 read on the current device recomputed exactly for some of
- * their channels (causal rows whose visible values lie far below the shared
- * value-bank shift).  Diagnostic; -1 on error.
+ * their channels: the entries whose 16-bit operands could have lost more
+ * than 2^-7 of the output to underflow (peaked priors at large beta, and the
+ * first rows of causal diagonal tiles whose value-bank shift includes keys
+ * they do not see).  Diagnostic; -1 on error.
  */
 int fem_last_fixup_rows(void *stream);
 

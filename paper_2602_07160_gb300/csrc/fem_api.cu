@@ -3,10 +3,11 @@
 //
 // bf16 path, in stream order:
 //   1. tile_stats, plan, bank: channel modes, shift schedule, the fp16 value
-//      bank (once per key tile), the fix-up list
-//   2. fem_tc (tcgen05): the read for every row and channel
-//   3. fixup (causal only): the listed entries completed exactly over their
-//      diagonal tile, merged with the state fem_tc left for the earlier tiles
+//      bank (once per key tile) and its column sums
+//   2. fem_tc (tcgen05): the read for every row and channel, and the list of
+//      entries its underflow guard rejects
+//   3. fixup: the listed entries recomputed exactly, from the state fem_tc
+//      left before their diagonal tile or over every key tile
 #include <cudaTypedefs.h>
 
 #include <algorithm>
@@ -48,7 +49,7 @@ int map_cuda(cudaError_t e) {
 }
 
 // Per-device addresses of the error word and fix-up counter, SM count and the
-// tensor-map encoder, set up once with the device current.
+// tensor-map encoder, set up once with the device current.  No allocation.
 int device_state(DeviceState **out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FEM_ERR_CUDA;
@@ -59,13 +60,6 @@ int device_state(DeviceState **out) {
     if (cudaGetSymbolAddress(reinterpret_cast<void **>(&s.last_fixup), g_last_fixup) != cudaSuccess)
       return FEM_ERR_CUDA;
     if (cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return FEM_ERR_CUDA;
-    cudaMemPoolProps props = {};
-    props.allocType = cudaMemAllocationTypePinned;
-    props.location.type = cudaMemLocationTypeDevice;
-    props.location.id = dev;
-    if (cudaMemPoolCreate(&s.pool, &props) != cudaSuccess) return FEM_ERR_CUDA;
-    uint64_t keep = ~uint64_t(0);
-    if (cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess) return FEM_ERR_CUDA;
     if (!g_encode) {
       cudaDriverEntryPointQueryResult q;
       void *fn = nullptr;
@@ -81,8 +75,30 @@ int device_state(DeviceState **out) {
   return FEM_OK;
 }
 
-// Stream-ordered workspace from the device's library pool (free with cudaFreeAsync).
-cudaError_t ws_alloc(const DeviceState *ds, void **p, size_t bytes, cudaStream_t s) {
+// Stream-ordered workspace from the device's library pool (free with
+// cudaFreeAsync).  The pool is created by the first entry point that
+// allocates on the device.
+cudaError_t ws_alloc(DeviceState *ds, void **p, size_t bytes, cudaStream_t s) {
+  {
+    std::lock_guard<std::mutex> lock(g_mutex);
+    if (!ds->pool) {
+      int dev = 0;
+      cudaError_t e = cudaGetDevice(&dev);
+      if (e != cudaSuccess) return e;
+      cudaMemPoolProps props = {};
+      props.allocType = cudaMemAllocationTypePinned;
+      props.location.type = cudaMemLocationTypeDevice;
+      props.location.id = dev;
+      cudaMemPool_t pool = nullptr;
+      if ((e = cudaMemPoolCreate(&pool, &props)) != cudaSuccess) return e;
+      uint64_t keep = ~uint64_t(0);
+      if ((e = cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep)) != cudaSuccess) {
+        cudaMemPoolDestroy(pool);
+        return e;
+      }
+      ds->pool = pool;
+    }
+  }
   return cudaMallocFromPoolAsync(p, bytes, ds->pool, s);
 }
 
@@ -105,10 +121,11 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-  size_t tstat, chan, bcoef, shift, rfac, colmask, bank, fixups, tilefix, count, total;
+  size_t tstat, chan, bcoef, shift, rfac, colsum, colmask, bank, fixups, count, total;
 };
 
 bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
+  (void)causal;  // the guard's fix-up list serves both forms of the read
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0) return false;
   const size_t BH = static_cast<size_t>(B) * H;
   const size_t n_kt = (static_cast<size_t>(T) + kBlockK - 1) / kBlockK;
@@ -125,12 +142,12 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += round256(BH * n_kt * d * sizeof(float));
   w->rfac = off;
   off += round256(BH * n_kt * d * sizeof(float));
+  w->colsum = off;
+  off += round256(BH * n_kt * d * sizeof(float));
   w->colmask = off;
   off += round256(BH * n_kt * 4 * sizeof(unsigned));
   w->fixups = off;
-  off += causal ? round256(BH * n_kt * kBlockQ * sizeof(FixupEntry)) : 0;
-  w->tilefix = off;
-  off += causal ? round256(BH * n_kt * sizeof(int2)) : 0;
+  off += round256(fixup_capacity(BH, static_cast<size_t>(T)) * sizeof(FixupEntry));
   w->count = off;  // fix-up slots, fix-up rows, the fix-up's chunk counter
   off += 256;
   w->total = off;
@@ -147,6 +164,13 @@ int check_common(const void *q, const void *k, const void *v, const float *beta,
     return FEM_ERR_INVALID_ARG;
   const long long rows = static_cast<long long>(B) * H * T;
   if (rows >= (1ll << 31) || static_cast<long long>(B) * H > 65535) return FEM_ERR_UNSUPPORTED;
+  return FEM_OK;
+}
+
+// Sizes the tensor-core read takes: d in {64, 128} and T up to kMaxSeqLen.
+int check_tc_sizes(int T, int d) {
+  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if (T > kMaxSeqLen) return FEM_ERR_UNSUPPORTED;
   return FEM_OK;
 }
 
@@ -206,20 +230,20 @@ size_t fem_fwd_workspace_bytes(int B, int H, int T, int d, int causal) {
 }
 
 // The read's workspace arrays at `ws` (layout ws_layout).
-static BankWorkspace bank_workspace(uint8_t *ws, const WsLayout &w, int causal) {
+static BankWorkspace bank_workspace(uint8_t *ws, const WsLayout &w) {
   BankWorkspace bw;
   bw.tstat = reinterpret_cast<float4 *>(ws + w.tstat);
   bw.chan = reinterpret_cast<ChanInfo *>(ws + w.chan);
   bw.bcoef = reinterpret_cast<float4 *>(ws + w.bcoef);
   bw.shift = reinterpret_cast<float *>(ws + w.shift);
   bw.rfac = reinterpret_cast<float *>(ws + w.rfac);
+  bw.colsum = reinterpret_cast<float *>(ws + w.colsum);
   bw.colmask = reinterpret_cast<unsigned *>(ws + w.colmask);
   bw.bank = reinterpret_cast<__half *>(ws + w.bank);
   bw.fixups = reinterpret_cast<FixupEntry *>(ws + w.fixups);
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
   bw.fixup_rows = reinterpret_cast<int *>(ws + w.count) + 1;
   bw.fixup_next = reinterpret_cast<int *>(ws + w.count) + 2;
-  bw.tilefix = causal ? reinterpret_cast<int2 *>(ws + w.tilefix) : nullptr;
   return bw;
 }
 
@@ -239,7 +263,7 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
   const int BH = B * H;
   WsLayout w;
   ws_layout(B, H, T, d, causal, &w);
-  BankWorkspace bw = bank_workspace(ws, w, causal);
+  BankWorkspace bw = bank_workspace(ws, w);
   CUtensorMap tq, tk, tv, te, te0;
   int rc;
   if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
@@ -251,33 +275,28 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
   if (ga) {
     WsLayout w0;
     ws_layout(B, H, T, d, 0, &w0);
-    bw0 = bank_workspace(ga->ws0, w0, 0);
+    bw0 = bank_workspace(ga->ws0, w0);
     if ((rc = make_map(&te0, bw0.bank, BH, T, d, CU_TENSOR_MAP_DATA_TYPE_FLOAT16)) != FEM_OK) return rc;
-    gate = TcGate{ga->lam, ga->g, ga->mu_side, bw0.chan};
+    gate = TcGate{ga->lam, ga->g, ga->mu_side, bw0.chan, bw0.colsum};
   }
 
   cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 3 * sizeof(int), s);
   // the mean's bank (every channel linear at beta = 0: v - c with c the channel mean)
-  if (e == cudaSuccess && ga) e = cudaMemsetAsync(bw0.fixup_count, 0, 3 * sizeof(int), s);
   if (e == cudaSuccess && ga)
-    e = launch_value_bank(v, tv, te0, ga->zero_beta, BH, H, T, d, 0, bw0, ds->err, ds->num_sms, s);
+    e = launch_value_bank(v, tv, te0, ga->zero_beta, BH, H, T, d, bw0, ds->err, ds->num_sms, s);
   if (ga) bw.tstat = bw0.tstat;  // the tiles' statistics do not depend on beta
   if (e == cudaSuccess)
-    e = launch_value_bank(v, tv, te, beta, BH, H, T, d, causal, bw, ds->err, ds->num_sms, s, ga != nullptr);
+    e = launch_value_bank(v, tv, te, beta, BH, H, T, d, bw, ds->err, ds->num_sms, s, ga != nullptr);
   const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
   t_ev_start = t_ev_stop = nullptr;
   if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
   if (e == cudaSuccess)
-    e = launch_tc(d, tq, tk, te, ga ? &te0 : nullptr, out, beta, bw.chan, bw.shift, bw.rfac, bw.colmask, bw.tilefix,
-                  bw.fixups, lse, BH, H, T, causal, ga ? &gate : nullptr, ds->err, s);
+    e = launch_tc(d, tq, tk, te, ga ? &te0 : nullptr, out, beta, bw, lse, BH, H, T, causal, ga ? &gate : nullptr,
+                  ds->err, s);
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
-  if (e == cudaSuccess) {
-    if (causal)
-      e = launch_fixup(q, k, v, beta, bw.shift, out, H, T, d, bw.fixups, bw.fixup_count, bw.fixup_rows,
-                       bw.fixup_next, ds->last_fixup, ga ? &gate : nullptr, ds->num_sms, s);
-    else
-      e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
-  }
+  if (e == cudaSuccess)
+    e = launch_fixup(q, k, v, beta, bw.chan, bw.shift, out, H, T, d, causal, bw.fixups, bw.fixup_count,
+                     bw.fixup_rows, bw.fixup_next, ds->last_fixup, ga ? &gate : nullptr, ds->num_sms, s);
   return map_cuda(e);
 }
 
@@ -285,7 +304,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
                int T, int d, int causal, void *workspace, size_t workspace_bytes, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
-  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
   WsLayout w;
   ws_layout(B, H, T, d, causal, &w);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return FEM_ERR_INVALID_ARG;
@@ -300,7 +319,7 @@ int fem_fwd(const void *q, const void *k, const void *v, const float *beta, floa
             int T, int d, int causal, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
-  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
   const size_t bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
@@ -319,7 +338,7 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   int rc = check_common(q, k, v, beta_max, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
   if (!lam || !gate || !aligned16(lam) || !aligned16(gate)) return FEM_ERR_INVALID_ARG;
-  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
   // workspace: the beta_max read's, the mean's pre-pass (non-causal layout),
@@ -454,7 +473,7 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
                  int H, int T, int d, int causal, void *stream) {
   if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0 || (causal != 0 && causal != 1)) return FEM_ERR_INVALID_ARG;
-  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if (check_tc_sizes(T, d) != FEM_OK) return FEM_ERR_UNSUPPORTED;
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
@@ -540,7 +559,7 @@ int fem_fwd_noalloc(const void *q, const void *k, const void *v, const float *be
                     int H, int T, int d, int causal, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
-  if (d != 64 && d != 128) return FEM_ERR_UNSUPPORTED;
+  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
   const size_t need = fem_fwd_workspace_bytes(B, H, T, d, causal);
   if (need == 0 || need > kStaticScratchBytes) return FEM_ERR_NO_MEMORY;
   void *scratch = nullptr;

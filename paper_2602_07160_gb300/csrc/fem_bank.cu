@@ -10,16 +10,17 @@
 //                                  beta*(max - c) > kShiftLag); a per-tile mask
 //                                  of the channels whose shift moved; the
 //                                  bank's coefficients for every tile
-//   bank        (persistent)       E = bank(v) in fp16 with the tile's shift;
-//                                  causal: the (row, 32-channel group) entries
-//                                  of the tile's diagonal rows whose visible
-//                                  maximum lies more than kHazardTilt/beta below
-//                                  the shift, for the exact fix-up
+//   bank        (persistent)       E = bank(v) in fp16 with the tile's shift,
+//                                  and per channel the sum of |E| over the
+//                                  tile's keys (the tensor-core kernel's bound
+//                                  on the error of 16-bit prior weights)
 //
 // The shift is the per-channel LSE stabilisation of App. E ("Numerical
-// stability"), made online over key tiles; only keys < T enter it, and a
-// query tile's last key tile is its diagonal tile, so keys beyond a tile's
-// last row never raise the shift that tile's rows use.
+// stability"), made online over key tiles; only keys < T enter it.  On a
+// causal diagonal tile it also includes keys later than some of the tile's
+// rows; the tensor-core kernel's guard finds the rows for which that (or a
+// peaked prior) leaves the 16-bit operands too little range, and the exact
+// fix-up completes them.
 #include "fem_common.cuh"
 #include "fem_launch.h"
 
@@ -155,7 +156,7 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
 // ---------------------------------------------------------------------------
 template <int D>
 __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta,
-                                                   int H, int T, int n_kt, int causal, ChanInfo *__restrict__ chan,
+                                                   int H, int T, int n_kt, ChanInfo *__restrict__ chan,
                                                    float *__restrict__ shift, float *__restrict__ rfac,
                                                    unsigned *__restrict__ colmask, float4 *__restrict__ bcoef) {
   constexpr int kParts = 4, kPer = 16, kWin = kParts * kPer;
@@ -217,7 +218,6 @@ __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ ts
         for (int u = 0; u < kPer; ++u) {
           const int kt = w0 + stage * kPer + u;
           if (kt < n_kt) {
-            const float cp_prev = cp;
             cp = fmaxf(cp, tmx[u]);
             const float prev = cl;
             if (lin) {
@@ -230,19 +230,8 @@ __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ ts
             const bool moved = !lin && kt > 0 && cl != prev;
             rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
             if (moved) atomicOr(&s_mask[stage * kPer + u], 1u << (j & 31));
-            // Diagonal hazard of a shifted channel: a row of the tile is safe
-            // once its visible maximum reaches cl - kHazardTilt/beta, so the
-            // bank checks the tile's keys against that level unless an earlier
-            // tile already reached it.
-            float4 bc;
-            if (lin) {
-              bc = make_float4(b > 0.f ? 1.f / b : 0.f, b, cl, __int_as_float(0x7fc00000));
-            } else {
-              const float thr = cl - kHazardTilt / b;
-              const bool check = causal && !(kt > 0 && cp_prev >= thr);
-              bc = make_float4(b * kLog2e, (kBankOffset - b * cl) * kLog2e, cl, check ? thr : -INFINITY);
-            }
-            bcoef[o] = bc;
+            bcoef[o] = lin ? make_float4(b > 0.f ? 1.f / b : 0.f, b, cl, __int_as_float(0x7fc00000))
+                           : make_float4(b * kLog2e, (kBankOffset - b * cl) * kLog2e, cl, 0.f);
           }
         }
       }
@@ -269,9 +258,10 @@ __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ ts
 // x 128 rows with the 128-byte swizzle (the layout the tensor-core kernel
 // reads the bank in) and the tile's BankCoef.  Warp w owns the 16-byte chunks
 // (8 channels) w*CPW .. w*CPW + CPW - 1; lane l handles rows l, 32 + l, 64 + l,
-// 96 + l of a chunk, so each channel's form (linear or shifted) and hazard
-// check are uniform across the warp.  The bank overwrites V in the slot and
-// leaves with one TMA store per box.
+// 96 + l of a chunk, so each channel's form (linear or shifted) is uniform
+// across the warp.  The bank overwrites V in the slot and leaves with one TMA
+// store per box; the column sums of |bank| over the tile's valid rows go to
+// colsum[tile][channel].
 // ---------------------------------------------------------------------------
 template <int D>
 struct BankMap {
@@ -293,19 +283,39 @@ __device__ __forceinline__ void bank_issue(const CUtensorMap *tv, const float4 *
   bulk_load(slot + M::kTileBytes, bcoef + static_cast<size_t>(g) * D, D * 16, bar);
 }
 
+// Sum of x[u] over the warp's 32 lanes for u = 0..7 in 9 shuffles: each
+// exchange halves the values a lane keeps (lanes keep the half named by the
+// exchanged bit), then the last value is summed over the remaining two bits.
+// Lane l ends with the sum for u = 4 ((l >> 4) & 1) + 2 ((l >> 3) & 1) +
+// ((l >> 2) & 1).
+__device__ __forceinline__ float warp_sum8_transposed(const float (&x)[8], int lane) {
+  float a[4], b[2];
+  const bool h16 = lane & 16, h8 = lane & 8, h4 = lane & 4;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const float keep = h16 ? x[u + 4] : x[u], send = h16 ? x[u] : x[u + 4];
+    a[u] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const float keep = h8 ? a[u + 2] : a[u], send = h8 ? a[u] : a[u + 2];
+    b[u] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+  }
+  float c = (h4 ? b[1] : b[0]) + __shfl_xor_sync(0xffffffffu, h4 ? b[0] : b[1], 4);
+  c += __shfl_xor_sync(0xffffffffu, c, 2);
+  c += __shfl_xor_sync(0xffffffffu, c, 1);
+  return c;
+}
+
 template <int D>
 __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CUtensorMap tv,
                                                        const __grid_constant__ CUtensorMap te,
                                                        const float4 *__restrict__ bcoef, int T, int n_kt,
-                                                       int n_tiles, int causal, FixupEntry *__restrict__ fixups,
-                                                       int *__restrict__ fixup_count, int *__restrict__ fixup_rows,
-                                                       int2 *__restrict__ tilefix, unsigned *__restrict__ err) {
+                                                       int n_tiles, float *__restrict__ colsum,
+                                                       unsigned *__restrict__ err) {
   using M = BankMap<D>;
   extern __shared__ uint8_t bank_smem[];
   __shared__ __align__(8) uint64_t s_full[kStages];
-  __shared__ int s_first[2][D];  // first row of the tile at or above the channel's hazard level
-  __shared__ int s_wmax[2][8];
-  __shared__ int s_base;
   const uint32_t base_addr = (smem_u32(bank_smem) + 1023u) & ~1023u;  // 128-byte swizzle wants 1024-B alignment
   uint8_t *const ring = bank_smem + (base_addr - smem_u32(bank_smem));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -319,7 +329,7 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
   }
   __syncthreads();
   for (int i = 0; i < my_n; ++i) {
-    const int st = i % kStages, g = blockIdx.x + i * gridDim.x, buf = i & 1;
+    const int st = i % kStages, g = blockIdx.x + i * gridDim.x;
     const int bh = g / n_kt, kt = g % n_kt, rows = min(kBlockK, T - kt * kBlockK);
     if (!mbar_wait(smem_u32(&s_full[st]), (i / kStages) & 1, err, kErrWaitTma)) {
       if (tid == 0) bulk_wait_group_read0();
@@ -327,7 +337,6 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
     }
     uint8_t *const tile = ring + st * M::kSlotBytes;
     const float4 *const coef = reinterpret_cast<const float4 *>(tile + M::kTileBytes);
-    int wmax = 0;
 #pragma unroll
     for (int q = 0; q < M::CPW; ++q) {
       const int ch = warp * M::CPW + q;  // chunk: channels 8 ch .. 8 ch + 7
@@ -339,10 +348,10 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
         cell[rb] = tile + (ch >> 3) * 16384 + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
         raw[rb] = *reinterpret_cast<const uint4 *>(cell[rb]);
       }
-      float res[4][8];
+      float res[4][8], csum[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        const float4 cf = coef[ch * 8 + u];  // {a, b, c, hazard level}; level NaN: linear bank
+        const float4 cf = coef[ch * 8 + u];  // {a, b, c, w}; w NaN: linear bank
         float x[4];
 #pragma unroll
         for (int rb = 0; rb < 4; ++rb) {
@@ -394,17 +403,11 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
             res[2 * rp + 1][u] = ex2_approx(t.y);
           }
         }
-        int first = 0;
-        if (cf.w > -INFINITY) {  // hazard check of a shifted channel
-          first = kBlockK;
+        // |bank| summed over this lane's valid rows (rows past T are padding)
+        float cs = 0.f;
 #pragma unroll
-          for (int rb = 0; rb < 4; ++rb) {
-            const unsigned hit = __ballot_sync(0xffffffffu, x[rb] >= cf.w && rb * 32 + lane < rows);
-            if (hit && first == kBlockK) first = rb * 32 + __ffs(hit) - 1;
-          }
-        }
-        if (lane == 0) s_first[buf][ch * 8 + u] = first;
-        wmax = max(wmax, first);
+        for (int rb = 0; rb < 4; ++rb) cs += rb * 32 + lane < rows ? fabsf(res[rb][u]) : 0.f;
+        csum[u] = cs;
       }
 #pragma unroll
       for (int rb = 0; rb < 4; ++rb) {
@@ -417,8 +420,11 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
         }
         *reinterpret_cast<uint4 *>(cell[rb]) = o;
       }
+      const float tot = warp_sum8_transposed(csum, lane);
+      if ((lane & 3) == 0)
+        colsum[static_cast<size_t>(g) * D + ch * 8 + ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] =
+            tot;
     }
-    if (lane == 0) s_wmax[buf][warp] = wmax;
     fence_proxy_async_smem();
     __syncthreads();
     if (tid == 0) {
@@ -434,50 +440,12 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
                       base_addr + sn * M::kSlotBytes, smem_u32(&s_full[sn]));
       }
     }
-    if (!causal) continue;
-    // rows r < max_j first_j of this tile get one entry with their channel masks
-    int hz_max = 0;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) hz_max = max(hz_max, s_wmax[buf][w]);
-    const int n_rows = min(hz_max, rows);
-    int2 *tf = tilefix + g;
-    if (n_rows <= 0) {
-      if (tid == 0) *tf = make_int2(0, 0);
-      continue;
-    }
-    // the tile's entries take a multiple of 8 slots (padding rows -1), so the
-    // fix-up's 8-entry chunks never straddle two tiles
-    const int n_slots = (n_rows + 7) & ~7;
-    if (tid == 0) {
-      s_base = atomicAdd(fixup_count, n_slots);
-      atomicAdd(fixup_rows, n_rows);
-      *tf = make_int2(s_base, n_rows);
-    }
-    __syncthreads();
-    const int fbase = s_base;
-    for (int r = tid; r < n_slots; r += 256) {
-      FixupEntry e;
-      e.row = r < n_rows ? bh * T + kt * kBlockQ + r : -1;
-#pragma unroll
-      for (int gq = 0; gq < 4; ++gq) {
-        unsigned m = 0;
-        for (int c = 0; c < 32; ++c) {
-          const int j = 32 * gq + c;
-          if (j < D && r < n_rows && s_first[buf][j] > r) m |= 1u << c;
-        }
-        e.mask[gq] = m;
-      }
-      e.m_pre = -INFINITY;
-      e.l_pre = 0.f;
-      e.pad = 0;
-      fixups[fbase + r] = e;
-    }
   }
   if (tid == 0) bulk_wait_group_read<0>();
 }
 
 cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtensorMap &te, const float *beta, int BH,
-                              int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
+                              int H, int T, int d, const BankWorkspace &w, unsigned *err, int num_sms,
                               cudaStream_t stream, bool stats_ready) {
   const int n_kt = (T + kBlockK - 1) / kBlockK, n_tiles = BH * n_kt;
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
@@ -493,10 +461,9 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
     if (e != cudaSuccess) return e;
     if (!stats_ready)
       tile_stats_kernel<64><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
-    plan_kernel<64><<<dim3(BH, 2), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, causal, w.chan, w.shift, w.rfac,
-                                                     w.colmask, w.bcoef);
-    bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, causal, w.fixups,
-                                                      w.fixup_count, w.fixup_rows, w.tilefix, err);
+    plan_kernel<64><<<dim3(BH, 2), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.shift, w.rfac, w.colmask,
+                                                     w.bcoef);
+    bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, w.colsum, err);
   } else if (d == 128) {
     using SM = StatsMap<128>;
     using BM = BankMap<128>;
@@ -507,10 +474,9 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
     if (e != cudaSuccess) return e;
     if (!stats_ready)
       tile_stats_kernel<128><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
-    plan_kernel<128><<<dim3(BH, 4), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, causal, w.chan, w.shift, w.rfac,
-                                                      w.colmask, w.bcoef);
-    bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, causal, w.fixups,
-                                                       w.fixup_count, w.fixup_rows, w.tilefix, err);
+    plan_kernel<128><<<dim3(BH, 4), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.shift, w.rfac, w.colmask,
+                                                      w.bcoef);
+    bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, w.colsum, err);
   } else {
     return cudaErrorInvalidValue;
   }

@@ -34,21 +34,38 @@ namespace fem {
 // with a running shift c_j and reads o = c + (log(acc/L) - kBankOffset)/beta.
 // Until c_j moves, E <= exp(kShiftLag + kBankOffset) = e^11 < 65504 (fp16);
 // a larger lag means fewer tiles on which acc must be rescaled for a moved
-// shift, a smaller offset that values more than about kHazardTilt/beta below
-// c leave fp16's normal range, which only happens on causal diagonal tiles
-// and is handled by the exact fix-up.
+// shift.
+//
+// Underflow guard.  The prior weights P <= 2^kRowMaxLag and the bank are
+// rounded to fp16, whose normal range ends at 2^-14; below it values keep an
+// absolute error up to 2^-25 (subnormal or flushed).  In the units of the
+// final row maximum and shift, with L = sum_i P_i (fp32) and
+// Ecol_j = sum_i |bank_ij| over the keys read, the accumulator's error from
+// the subnormal range is at most 2^-25 (L + Ecol_j) (shifted bank; the P side
+// through Ecol_j, the bank side through L) or 2^-25 Ecol_j in value units
+// (linear bank, whose own subnormals are absolute errors in v).  An entry
+// whose bound exceeds kGuardTau times what it can cost, i.e.
+//   shifted: 2^-25 (L + Ecol_j) > kGuardTau * beta_j * acc_j,
+//   linear:  2^-25 Ecol_j       > kGuardTau * (L + beta_j * acc_j),
+// would move o_tj by more than kGuardTau and is recomputed exactly (peaked
+// priors at large beta, where the read is carried by keys of tiny prior
+// weight or a heavy key's value lies far below the shift; the first rows of
+// a causal diagonal tile, whose shift includes keys they do not see).
 // ---------------------------------------------------------------------------
 constexpr float kLinearLowTilt = 1.0f;
 constexpr float kLinearBankMax = 30000.f;  // fp16 holds values up to 65504
 constexpr float kBankOffset = 4.0f;        // natural-log offset of the shifted bank
 constexpr float kShiftLag = 7.0f;          // c_j moves only when beta*(new max - c) > this
 constexpr float kRowMaxLag = 8.0f;         // row max moves only when it grows by > 2^this
-constexpr float kHazardTilt = 14.0f;       // row/channel recomputed exactly when beta*(c - visible max) > this
+constexpr float kGuardTau = 0.0078125f;    // 2^-7: largest output error the guard lets through
+constexpr float kGuardUlp = 2.98023224e-08f * 1.0078125f;  // 2^-25 (fp16 subnormal half-spacing), with slack
+                                                           // for sums taken before the fp16 rounding
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
 constexpr int kBlockQ = 128;  // query rows per tile (TMEM lanes)
 constexpr int kBlockK = 128;  // keys per tile
+constexpr int kFixChunk = 8;  // fix-up entries per chunk: rows scored together, one warp each
 
 // Error bits of the per-device error word.
 constexpr unsigned kErrWaitTma = 1u;
@@ -63,15 +80,20 @@ struct ChanInfo {
   float linear;  // 1.0f when the channel uses the linear bank, else 0.0f
 };
 
-// One fix-up entry: row = (b*H + h)*T + t of a causal diagonal tile; channel
-// 32*g + bit is completed for every set bit of mask[g].  The tensor-core
-// kernel fills m_pre and l_pre: the row's running maximum (log2 units) and
-// sum of 2^(s - m_pre) over the key tiles before the diagonal one.
+// One fix-up entry, written by the tensor-core kernel in blocks padded to a
+// multiple of kFixChunk: row = (b*H + h)*T + t (-1: padding); channel 32*g + bit is recomputed exactly for every set bit of
+// mask[g], over the key tiles kt0 .. the row's last one.  With kt0 > 0 (a
+// causal row whose state before its diagonal tile passed the guard) the
+// recomputation starts from that state: m_pre and l_pre, the row's running
+// maximum (log2 units) and sum of 2^(s log2 e - m_pre) over the key tiles
+// before kt0, and, in out[row][j], channel j's accumulator over them (the bank
+// of tile kt0 - 1's shift).  With kt0 = 0 every key is taken again, and l_pre
+// is 1 when the gated read's mean must be recomputed as well, 0 otherwise.
 struct __align__(32) FixupEntry {
   int row;
   unsigned mask[4];
   float m_pre, l_pre;
-  int pad;
+  int kt0;
 };
 
 // ---------------------------------------------------------------------------

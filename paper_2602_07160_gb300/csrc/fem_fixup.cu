@@ -1,48 +1,53 @@
-// Completion of the (row, channel) entries listed by the pre-pass.
+// Exact completion of the (row, channel) entries the tensor-core kernel's
+// underflow guard rejected.
 //
-// These are rows t of a causal diagonal key tile whose visible values of a
-// shifted channel all lie far below the tile's bank shift (the shift includes
-// keys the row cannot see), so the bank underflows for them on that tile
-// only.  The tensor-core kernel leaves, for each entry, the state over the
-// key tiles before the diagonal one: the row's running maximum m and sum l of
-// 2^(s' - m) (s' = s log2 e, in the entry), and, in place of each listed
-// channel's output, its accumulator
-//   a_j = sum_{i < k0} 2^(s'_i - m) exp(beta_j (v_ij - c_j) + kappa),
-// c_j the bank shift of tile kt - 1.  This kernel takes the diagonal tile's
-// keys k0 .. t exactly in fp32 and merges, in base 2,
-//   G_j = log2 sum_{i <= t} 2^(s'_i + beta_j v_ij log2 e)
-//       = log2( 2^(m + log2 a_j + (beta_j c_j - kappa) log2 e) + sum_{k0 <= i <= t} 2^(s'_i + beta_j v_ij log2 e) )
-//   L   = log2( 2^m l + sum_{k0 <= i <= t} 2^(s'_i) )
-// and writes o_tj = (G_j - L) ln 2 / beta_j, the read's definition
-// (Sec. 2.3, Eq. "fem-free-energy-main", with the softmax prior of App. C),
-// each log-sum-exp stabilised by its own maximum (App. E, "Numerical
-// stability").
+// For an entry of row t (b, h) the kernel restarts the read of the listed
+// channels from the entry's key tile kt0 and takes every later key the row
+// sees exactly in fp32, the way the fp32 read does: with the row's running
+// maximum m of s' = s log2 e, P_i = 2^(s'_i - m), and per channel j a running
+// shift c_j (the largest visible value so far) and
+//   L   = sum_i P_i
+//   A_j = sum_i P_i exp(beta_j (v_ij - c_j))
+//   W_j = sum_i P_i expm1(beta_j (v_ij - c_j)) / beta_j   (v_ij - c_j at beta 0)
+// The read is then o = c + log1p(beta W / L) / beta when beta W / L > -1/2
+// (W is kept for beta < kFixWBeta only), c + log(A / L) / beta otherwise,
+// c + W / L at beta = 0: the read's
+// definition (Sec. 2.3, Eq. "fem-free-energy-main", with the softmax prior of
+// App. C), free of the cancellation in the LSE difference at small beta and
+// each sum stabilised by its own maximum (App. E, "Numerical stability").
 //
-// Entries come in chunks of 8 consecutive rows of one diagonal tile (the
-// pre-pass pads each tile's entries to a multiple of 8 with rows -1).  One
-// 256-thread block takes a chunk at a time, claimed from a counter so that
-// blocks that drew cheap chunks take more of them: it stages the tile's
-// K and V rows k0 .. k0+r_max and the chunk's 8 query rows in shared memory,
-// scores the 8 rows against the keys with warp-level bf16 MMAs (16 keys per
-// warp, fp32 accumulation), then each warp completes one entry: its lanes
-// take four keys each and reduce
-// the row's log-sum-exp and, channel by channel, each listed channel's with
-// warp shuffles; a 32-channel group with three or more listed channels is
-// done with lane = channel instead, walking the keys in turn.
+// kt0 > 0: the row's earlier key tiles passed the guard, and the kernel
+// starts from the state the tensor-core kernel left before tile kt0 (m, L in
+// the entry; channel j's accumulator a_j in out[row][j], over the bank of tile
+// kt0 - 1: shifted, A = a e^-kappa at that tile's shift and W = (A - L)/beta;
+// linear, W = a at the anchor and A = L + beta W).  kt0 = 0: from nothing.
+// The one-pass gated read's entries are gated, o = g (mu + lambda (F - mu)),
+// with the mu the tensor-core kernel left aside, or, when the mean bank's own
+// guard rejected it (kt0 = 0 and l_pre = 1), with mu recomputed as
+// sum_i P_i (v_ij - c0_j) / L + c0_j.
+//
+// Entries come in chunks of kFixChunk = 8 rows of one query tile with the
+// same kt0 (the tensor-core kernel pads each block to a multiple of 8 with
+// rows -1).  One 256-thread block (two per SM) takes a chunk at a time,
+// claimed from a counter (the next claim already in flight while the current
+// chunk runs) so that blocks that drew cheap chunks take more of them, and
+// walks its key tiles: it stages the chunk's query rows and the tile's K and V
+// rows in shared memory with asynchronous copies, scores the 8 rows against
+// them with warp-level bf16 MMAs (16 keys per warp, fp32 accumulation), then
+// each warp folds the tile into one entry's state: its
+// lanes take four keys each for the row's sums and, channel by channel, for
+// each listed channel's; a 32-channel group with three or more listed
+// channels is folded with lane = channel instead, walking the keys in turn in
+// one pass.
 #include "fem_common.cuh"
 #include "fem_launch.h"
 
 namespace fem {
 
-constexpr int kFixChunk = 8;                // entries per chunk = warps per block
-
-// The entry's output: F itself, or for the one-pass gated read
-// g (mu + lambda (F - mu)) with the mu the tensor-core kernel left aside.
-__device__ __forceinline__ float fix_gated(const TcGate &gate, size_t o, float F) {
-  if (!gate.lam) return F;
-  const float mu = gate.mu_side[o];
-  return gate.g[o] * fmaf(gate.lam[o], F - mu, mu);
-}
+// Channels with beta below this carry W (the read o = c + log1p(beta W / L) / beta,
+// free of cancellation when A / L is near 1); from here on log(A / L) / beta
+// loses at most a few fp32 ulps of A / L over beta and W is not needed.
+constexpr float kFixWBeta = 0.25f;
 constexpr int kFixThreads = 32 * kFixChunk;
 
 __device__ __forceinline__ float warp_max(float x) {
@@ -86,11 +91,48 @@ __device__ __forceinline__ void fix_cp_wait_all() {
   asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
-// log2(2^a + 2^b) for a, b possibly -inf
-__device__ __forceinline__ float lse2_pair(float a, float b) {
-  const float mx = fmaxf(a, b);
-  if (mx == -INFINITY) return -INFINITY;
-  return mx + log2f(exp2f(a - mx) + exp2f(b - mx));
+// expm1(y)/beta for y = beta x <= 0, given e = exp(y): the series of
+// expm1(y)/y times x for |y| < 1/2 (truncation below 4e-6 relative), (e - 1)
+// times 1/beta beyond; x itself at beta = 0.
+__device__ __forceinline__ float em1_over_beta(float x, float y, float e, float rb) {
+  if (fabsf(y) < 0.5f) {
+    float p = fmaf(y, 1.f / 720.f, 1.f / 120.f);
+    p = fmaf(y, p, 1.f / 24.f);
+    p = fmaf(y, p, 1.f / 6.f);
+    p = fmaf(y, p, 0.5f);
+    p = fmaf(y, p, 1.f);
+    return x * p;
+  }
+  return (e - 1.f) * rb;
+}
+
+// The running state of one channel moves from shift c to c_new >= c:
+// A <- r A, W <- r W + expm1(beta (c - c_new))/beta L with r = exp(beta (c - c_new)).
+__device__ __forceinline__ void shift_state(float &c, float &A, float &W, float c_new, float b, float rb, float L) {
+  if (!(c_new > c)) return;
+  if (c == -INFINITY) {
+    A = 0.f;
+    W = 0.f;
+  } else {
+    const float x = c - c_new, y = b * x, e = exp2f(y * kLog2e);
+    W = fmaf(e, W, em1_over_beta(x, y, e, rb) * L);
+    A *= e;
+  }
+  c = c_new;
+}
+
+// Folds a tile's sums (a, w) over keys of prior mass lt, taken at the tile's
+// own shift vt, into the running state (c, A, W) of prior mass L.
+__device__ __forceinline__ void fold_tile(float &c, float &A, float &W, float L, float vt, float a, float w, float lt,
+                                          float b, float rb) {
+  float A2 = a, W2 = w, c2 = vt;
+  if (vt >= c) {
+    shift_state(c, A, W, vt, b, rb, L);
+  } else {
+    shift_state(c2, A2, W2, c, b, rb, lt);
+  }
+  A += A2;
+  W += W2;
 }
 
 template <int D>
@@ -98,8 +140,10 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
                                                             const __nv_bfloat16 *__restrict__ k,
                                                             const __nv_bfloat16 *__restrict__ v,
                                                             const float *__restrict__ beta,
+                                                            const ChanInfo *__restrict__ chan,
                                                             const float *__restrict__ shift, float *__restrict__ out,
-                                                            int H, int T, const FixupEntry *__restrict__ entries,
+                                                            int H, int T, int causal,
+                                                            const FixupEntry *__restrict__ entries,
                                                             const int *__restrict__ count,
                                                             const int *__restrict__ rows_listed,
                                                             int *__restrict__ next_chunk,
@@ -107,178 +151,273 @@ __global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 
   // staged row strides in bf16 elements: K and Q rows 16-byte aligned for
   // ldmatrix with consecutive rows four banks apart; V rows an odd number of
   // 32-bit words, so one column read across rows is free of bank conflicts
-  constexpr int KS = D + 8, VS = D + 2;
+  constexpr int KS = D + 8, VS = D + 2, G = D / 32;
   extern __shared__ __align__(16) uint8_t fix_smem[];
   __nv_bfloat16 *sK = reinterpret_cast<__nv_bfloat16 *>(fix_smem);
   __nv_bfloat16 *sV = sK + kBlockK * KS;
   __nv_bfloat16 *sQ = sV + kBlockK * VS;  // 16 rows (8 entries, 8 unused) of KS
-  __shared__ float sS[kFixChunk][kBlockK];  // the chunk's scores, log2 units
-  __shared__ int s_nk, s_ch;
+  __shared__ float sS[kFixChunk][kBlockK];  // the chunk's scores (log2 units), then the tile's P
+  __shared__ int s_ch;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_chunks = *count / kFixChunk;
   if (blockIdx.x == 0 && tid == 0 && last_rows) *last_rows = *rows_listed;
   const float scale = kLog2e * rsqrtf(static_cast<float>(D));
   const int n_kt = (T + kBlockK - 1) / kBlockK;
+  const bool gated = gate.lam != nullptr;
 
+  int claim = 0;  // thread 0: the next chunk, claimed one chunk ahead
+  if (tid == 0) claim = atomicAdd(next_chunk, 1);
   for (;;) {
     if (tid == 0) {
-      s_ch = atomicAdd(next_chunk, 1);
-      s_nk = 0;
+      s_ch = claim;
+      if (claim < n_chunks) claim = atomicAdd(next_chunk, 1);
     }
     __syncthreads();
     const int ch = s_ch;
     if (ch >= n_chunks) break;
     const FixupEntry ent = entries[ch * kFixChunk + warp];
-    const int row0 = entries[ch * kFixChunk].row;  // the chunk's first entry is a real row
-    const int bh = row0 / T, h = bh % H;
-    const int kt = (row0 % T) / kBlockK, k0 = kt * kBlockK;
-    const int r = ent.row >= 0 ? ent.row - bh * T - k0 : -1;  // this warp's row in the tile
-    if (lane == 0 && r >= 0) atomicMax(&s_nk, r + 1);
-    // the entry's stashed accumulators over the earlier key tiles, the
-    // previous tile's shifts and beta, lane l holding channels l + 32 g: loaded
-    // now so that they arrive while the chunk's rows are staged and scored
-    float a_reg[D / 32], c_reg[D / 32], b_reg[D / 32];
+    const FixupEntry ent0 = entries[ch * kFixChunk];  // the chunk's first entry is a real row
+    const int bh = ent0.row / T, h = bh % H;
+    const int qt = (ent0.row % T) / kBlockQ, kt0 = ent0.kt0;
+    const int kt_end = causal ? qt : n_kt - 1;
+    const int t = ent.row >= 0 ? ent.row - bh * T : -1;  // this warp's row
+    const bool need_mu = gated && kt0 == 0 && ent.l_pre > 0.f;  // the gated read's mean recomputed too
+    // the entry's state, lane l holding channels l + 32 g
+    float m = -INFINITY, L = 0.f;
+    float c_reg[G], A_reg[G], W_reg[G], M_reg[G], b_reg[G], rb_reg[G], c0_reg[G];
 #pragma unroll
-    for (int gi = 0; gi < D / 32; ++gi) {
-      const int j = lane + 32 * gi;
-      const bool listed = r >= 0 && ent.mask[gi];
-      a_reg[gi] = listed ? out[static_cast<size_t>(ent.row) * D + j] : 0.f;
-      c_reg[gi] = (listed && kt > 0) ? shift[(static_cast<size_t>(bh) * n_kt + kt - 1) * D + j] : 0.f;
-      b_reg[gi] = beta[h * D + j];
+    for (int g = 0; g < G; ++g) {
+      const int j = lane + 32 * g;
+      const float bj = beta[h * D + j];
+      b_reg[g] = bj;
+      rb_reg[g] = bj != 0.f ? 1.f / bj : 0.f;
+      c_reg[g] = -INFINITY;
+      A_reg[g] = W_reg[g] = M_reg[g] = 0.f;
+      c0_reg[g] = need_mu ? gate.chan0[bh * D + j].c_lin : 0.f;  // the mean's anchor
     }
-    __syncthreads();
-    const int nk = s_nk;  // keys k0 .. k0+nk-1 serve every row of the chunk
-    for (int idx = tid; idx < nk * (D / 8); idx += kFixThreads) {
-      const int i = idx / (D / 8), c = idx % (D / 8);
-      const size_t g = (static_cast<size_t>(bh) * T + k0 + i) * D + 8 * c;
-      fix_cp16(smem_u32(sK + i * KS + 8 * c), k + g);
-      const uint32_t dv = smem_u32(sV + i * VS + 8 * c);
+    if (t >= 0 && kt0 > 0) {
+      m = ent.m_pre;
+      L = ent.l_pre;
 #pragma unroll
-      for (int w = 0; w < 4; ++w) fix_cp4(dv + 4 * w, v + g + 2 * w);
+      for (int g = 0; g < G; ++g) {
+        const int j = lane + 32 * g;
+        if (!((ent.mask[g] >> lane) & 1u)) continue;
+        const float a = out[static_cast<size_t>(ent.row) * D + j];
+        const ChanInfo ci = chan[bh * D + j];
+        if (ci.linear != 0.f) {
+          c_reg[g] = ci.c_lin;
+          W_reg[g] = a;
+          A_reg[g] = fmaf(b_reg[g], a, L);
+        } else {
+          c_reg[g] = shift[(static_cast<size_t>(bh) * n_kt + kt0 - 1) * D + j];
+          A_reg[g] = a * 0.018315638888734f;  // e^-kappa
+          W_reg[g] = (A_reg[g] - L) * rb_reg[g];
+        }
+      }
     }
+    // the chunk's query rows, once, in flight with the first tile's K and V
+    // (a padding row scores the chunk's first row and is never read)
     for (int idx = tid; idx < kFixChunk * (D / 8); idx += kFixThreads) {
       const int w = idx / (D / 8), c = idx % (D / 8);
       const int erow = entries[ch * kFixChunk + w].row;
-      *reinterpret_cast<uint4 *>(sQ + w * KS + 8 * c) =
-          erow >= 0 ? *reinterpret_cast<const uint4 *>(q + static_cast<size_t>(erow) * D + 8 * c) : make_uint4(0, 0, 0, 0);
+      fix_cp16(smem_u32(sQ + w * KS + 8 * c), q + static_cast<size_t>(erow >= 0 ? erow : ent0.row) * D + 8 * c);
     }
-    fix_cp_wait_all();
-    __syncthreads();
-    // S[8 x nk] = Q K^T: warp w takes keys 16w .. 16w+15 (two n8 blocks) over
-    // D/16 k-steps of m16n8k16 (rows 8..15 of A are unused)
-    if (16 * warp < nk) {
-      float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
+    // the chunk's last row (every warp from the entries' rows, no barrier)
+    int t_last = lane < kFixChunk ? entries[ch * kFixChunk + lane].row : -1;
 #pragma unroll
-      for (int ks = 0; ks < D / 16; ++ks) {
-        uint32_t a[4], bfr[4];
-        ldmatrix_x4(a, smem_u32(sQ + (lane % 16) * KS + 16 * ks + (lane / 16) * 8));
-        const int mm = lane / 8;  // matrices: (keys lo, d lo) (keys lo, d hi) (keys hi, d lo) (keys hi, d hi)
-        ldmatrix_x4(bfr, smem_u32(sK + (16 * warp + (mm / 2) * 8 + lane % 8) * KS + 16 * ks + (mm % 2) * 8));
-        mma_bf16_16816(c0, a, bfr[0], bfr[1]);
-        mma_bf16_16816(c1, a, bfr[2], bfr[3]);
+    for (int off = 16; off; off >>= 1) t_last = max(t_last, __shfl_xor_sync(0xffffffffu, t_last, off));
+    t_last -= bh * T;
+    for (int kt = kt0; kt <= kt_end; ++kt) {
+      const int k0 = kt * kBlockK;
+      const bool diag = causal && kt == qt;
+      // keys k0 .. k0+nk-1 serve every row of the chunk
+      const int nk = diag ? t_last - k0 + 1 : min(kBlockK, T - k0);
+      for (int idx = tid; idx < nk * (D / 8); idx += kFixThreads) {
+        const int i = idx / (D / 8), c = idx % (D / 8);
+        const size_t gk = (static_cast<size_t>(bh) * T + k0 + i) * D + 8 * c;
+        fix_cp16(smem_u32(sK + i * KS + 8 * c), k + gk);
+        const uint32_t dv = smem_u32(sV + i * VS + 8 * c);
+#pragma unroll
+        for (int w = 0; w < 4; ++w) fix_cp4(dv + 4 * w, v + gk + 2 * w);
       }
-      // fragment rows lane/4 (and lane/4 + 8, unused), columns 2 (lane % 4) + {0, 1}
-      const int rr = lane / 4, cc = 16 * warp + 2 * (lane % 4);
-      sS[rr][cc] = c0[0] * scale;
-      sS[rr][cc + 1] = c0[1] * scale;
-      sS[rr][cc + 8] = c1[0] * scale;
-      sS[rr][cc + 9] = c1[1] * scale;
-    }
-    __syncthreads();
-    if (r >= 0) {
-      // scores of keys i = lane + 32u (log2 units), -inf past the row
-      float s[kBlockK / 32];
+      fix_cp_wait_all();
+      __syncthreads();
+      // S[16 x nk] = Q K^T: warp w takes keys 16w .. 16w+15 (two n8 blocks) over
+      // D/16 k-steps of m16n8k16; keys past nk read stale rows and are masked below
+      if (16 * warp < nk) {
+        float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int u = 0; u < kBlockK / 32; ++u) {
-        const int i = lane + 32 * u;
-        s[u] = i <= r ? sS[warp][i] : -INFINITY;
-      }
-      // the row's score log-sum-exp over all its keys
-      float mx = s[0];
-#pragma unroll
-      for (int u = 1; u < kBlockK / 32; ++u) mx = fmaxf(mx, s[u]);
-      mx = warp_max(mx);
-      float sm = 0.f;
-#pragma unroll
-      for (int u = 0; u < kBlockK / 32; ++u) sm += s[u] == -INFINITY ? 0.f : exp2f(s[u] - mx);
-      sm = warp_sum(sm);
-      const float L = lse2_pair(ent.l_pre > 0.f ? ent.m_pre + log2f(ent.l_pre) : -INFINITY, mx + log2f(sm));
-      // each listed channel's tilted log-sum-exp, merged with the tensor-core
-      // kernel's state over the earlier key tiles (a_reg, c_reg, b_reg)
-#pragma unroll
-      for (int gi = 0; gi < D / 32; ++gi) {
-        unsigned m = ent.mask[gi];
-        if (__popc(m) >= 3) {
-          // many listed channels in this group: lane = channel, keys walked in turn
-          const int j = 32 * gi + lane;
-          const float bl = b_reg[gi] * kLog2e;
-          float mj = -INFINITY;
-          for (int i = 0; i <= r; ++i) mj = fmaxf(mj, fmaf(bl, __bfloat162float(sV[i * VS + j]), sS[warp][i]));
-          float sj = 0.f;
-          for (int i = 0; i <= r; ++i) sj += exp2f(fmaf(bl, __bfloat162float(sV[i * VS + j]), sS[warp][i]) - mj);
-          if ((m >> lane) & 1u) {
-            float pre = -INFINITY;
-            if (kt > 0 && a_reg[gi] > 0.f && ent.l_pre > 0.f)
-              pre = ent.m_pre + log2f(a_reg[gi]) + (b_reg[gi] * c_reg[gi] - kBankOffset) * kLog2e;
-            const float G = lse2_pair(pre, mj + log2f(sj));
-            const size_t o = static_cast<size_t>(ent.row) * D + j;
-            out[o] = fix_gated(gate, o, (G - L) * kLn2 / b_reg[gi]);
-          }
-          m = 0;
+        for (int ks = 0; ks < D / 16; ++ks) {
+          uint32_t a[4], bfr[4];
+          ldmatrix_x4(a, smem_u32(sQ + (lane % 16) * KS + 16 * ks + (lane / 16) * 8));
+          const int mm = lane / 8;  // matrices: (keys lo, d lo) (keys lo, d hi) (keys hi, d lo) (keys hi, d hi)
+          ldmatrix_x4(bfr, smem_u32(sK + (16 * warp + (mm / 2) * 8 + lane % 8) * KS + 16 * ks + (mm % 2) * 8));
+          mma_bf16_16816(c0, a, bfr[0], bfr[1]);
+          mma_bf16_16816(c1, a, bfr[2], bfr[3]);
         }
-        while (m) {
-          const int jl = __ffs(m) - 1, j = 32 * gi + jl;
-          m &= m - 1;
-          const float bj = __shfl_sync(0xffffffffu, b_reg[gi], jl);
-          const float a = __shfl_sync(0xffffffffu, a_reg[gi], jl);  // accumulator over the earlier key tiles
-          const float c = __shfl_sync(0xffffffffu, c_reg[gi], jl);
-          const size_t o = static_cast<size_t>(ent.row) * D + j;
-          const float bl = bj * kLog2e;
-          float x[kBlockK / 32];
-          float mj = -INFINITY;
-#pragma unroll
-          for (int u = 0; u < kBlockK / 32; ++u) {
-            const int i = lane + 32 * u;
-            x[u] = i <= r ? fmaf(bl, __bfloat162float(sV[i * VS + j]), s[u]) : -INFINITY;
-            mj = fmaxf(mj, x[u]);
-          }
-          mj = warp_max(mj);
-          float sj = 0.f;
-#pragma unroll
-          for (int u = 0; u < kBlockK / 32; ++u) sj += x[u] == -INFINITY ? 0.f : exp2f(x[u] - mj);
-          sj = warp_sum(sj);
-          if (lane == 0) {
-            float pre = -INFINITY;
-            if (kt > 0 && a > 0.f && ent.l_pre > 0.f) pre = ent.m_pre + log2f(a) + (bj * c - kBankOffset) * kLog2e;
-            const float G = lse2_pair(pre, mj + log2f(sj));
-            out[o] = fix_gated(gate, o, (G - L) * kLn2 / bj);
-          }
+        // fragment rows lane/4 and lane/4 + 8, columns 2 (lane % 4) + {0, 1}
+        const int rr = lane / 4, cc = 16 * warp + 2 * (lane % 4);
+        sS[rr][cc] = c0[0] * scale;
+        sS[rr][cc + 1] = c0[1] * scale;
+        sS[rr][cc + 8] = c1[0] * scale;
+        sS[rr][cc + 9] = c1[1] * scale;
+        if (kFixChunk > 8) {
+          sS[rr + 8][cc] = c0[2] * scale;
+          sS[rr + 8][cc + 1] = c0[3] * scale;
+          sS[rr + 8][cc + 8] = c1[2] * scale;
+          sS[rr + 8][cc + 9] = c1[3] * scale;
         }
       }
+      __syncthreads();
+      if (t >= 0) {
+        // keys i = lane + 32u visible to the row: i < nk, and k0 + i <= t when causal
+        const int n_vis = diag ? t - k0 + 1 : nk;
+        float s[kBlockK / 32];
+        float mt = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < kBlockK / 32; ++u) {
+          const int i = lane + 32 * u;
+          s[u] = i < n_vis ? sS[warp][i] : -INFINITY;
+          mt = fmaxf(mt, s[u]);
+        }
+        mt = warp_max(mt);
+        if (mt > m) {  // the row maximum moves: every sum scales by 2^(m_old - m_new)
+          const float al = exp2f(m - mt);
+          L *= al;
+#pragma unroll
+          for (int g = 0; g < G; ++g) {
+            A_reg[g] *= al;
+            W_reg[g] *= al;
+            M_reg[g] *= al;
+          }
+          m = mt;
+        }
+        float p[kBlockK / 32], lt = 0.f;
+#pragma unroll
+        for (int u = 0; u < kBlockK / 32; ++u) {
+          p[u] = s[u] == -INFINITY ? 0.f : exp2f(s[u] - m);
+          lt += p[u];
+        }
+        lt = warp_sum(lt);
+        __syncwarp();
+#pragma unroll
+        for (int u = 0; u < kBlockK / 32; ++u) sS[warp][lane + 32 * u] = p[u];  // this row's P, for the walks
+        __syncwarp();
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          unsigned mk = ent.mask[g];
+          if (__popc(mk) >= 3) {
+            // many listed channels in this group: lane = channel, keys walked in
+            // turn, first for the visible maximum, then for the sums at it
+            const int j = 32 * g + lane;
+            float vt = -INFINITY;
+            for (int i = 0; i < n_vis; ++i) vt = fmaxf(vt, __bfloat162float(sV[i * VS + j]));
+            float c = c_reg[g], A = A_reg[g], W = W_reg[g];
+            const float b = b_reg[g], rb = rb_reg[g], bl = b * kLog2e;
+            const bool with_w = b < kFixWBeta;
+            shift_state(c, A, W, vt, b, rb, L);
+            float sm = 0.f;
+            for (int i = 0; i < n_vis; ++i) {
+              const float pi = sS[warp][i], x = __bfloat162float(sV[i * VS + j]);
+              const float xs = x - c, e = exp2f(bl * xs);
+              A = fmaf(pi, e, A);
+              if (with_w) W = fmaf(pi, em1_over_beta(xs, b * xs, e, rb), W);
+              if (need_mu) sm = fmaf(pi, x - c0_reg[g], sm);
+            }
+            if ((mk >> lane) & 1u) {
+              c_reg[g] = c;
+              A_reg[g] = A;
+              W_reg[g] = W;
+              M_reg[g] += sm;
+            }
+            mk = 0;
+          }
+          while (mk) {
+            // lanes = keys for one listed channel: the tile's sums at the tile's
+            // own maximum vt, folded into the state by the lane holding it (jl)
+            const int jl = __ffs(mk) - 1, j = 32 * g + jl;
+            mk &= mk - 1;
+            const float b = __shfl_sync(0xffffffffu, b_reg[g], jl), rb = b != 0.f ? 1.f / b : 0.f;
+            const float c0 = need_mu ? __shfl_sync(0xffffffffu, c0_reg[g], jl) : 0.f;
+            float x[kBlockK / 32], vt = -INFINITY;
+#pragma unroll
+            for (int u = 0; u < kBlockK / 32; ++u) {
+              const int i = lane + 32 * u;
+              x[u] = i < n_vis ? __bfloat162float(sV[i * VS + j]) : -INFINITY;
+              vt = fmaxf(vt, x[u]);
+            }
+            vt = warp_max(vt);
+            const float bl = b * kLog2e;
+            float sa = 0.f, sw = 0.f, sm = 0.f;
+#pragma unroll
+            for (int u = 0; u < kBlockK / 32; ++u) {
+              if (p[u] == 0.f) continue;
+              const float xs = x[u] - vt, y = b * xs, e = exp2f(bl * xs);
+              sa = fmaf(p[u], e, sa);
+              if (b < kFixWBeta) sw = fmaf(p[u], em1_over_beta(xs, y, e, rb), sw);
+              if (need_mu) sm = fmaf(p[u], x[u] - c0, sm);
+            }
+            sa = warp_sum(sa);
+            if (b < kFixWBeta) sw = warp_sum(sw);
+            if (need_mu) sm = warp_sum(sm);
+            if (lane == jl) {
+              fold_tile(c_reg[g], A_reg[g], W_reg[g], L, vt, sa, sw, lt, b, rb);
+              M_reg[g] += sm;
+            }
+          }
+        }
+        L += lt;
+      }
+      __syncthreads();  // the staged rows are rewritten by the next tile or chunk
     }
-    __syncthreads();  // the staged rows are rewritten by the next chunk
+    if (t >= 0) {
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        if (!((ent.mask[g] >> lane) & 1u)) continue;
+        const int j = lane + 32 * g;
+        const float b = b_reg[g], c = c_reg[g];
+        float o;
+        if (b == 0.f) {
+          o = c + W_reg[g] / L;
+        } else {
+          const float z = b * W_reg[g] / L;
+          o = (b < kFixWBeta && z > -0.5f) ? c + log1pf(z) * rb_reg[g] : c + logf(A_reg[g] / L) * rb_reg[g];
+        }
+        const size_t oi = static_cast<size_t>(ent.row) * D + j;
+        if (gated) {
+          const float mu = (kt0 == 0 && ent.l_pre > 0.f) ? c0_reg[g] + M_reg[g] / L : gate.mu_side[oi];
+          o = gate.g[oi] * fmaf(gate.lam[oi], o - mu, mu);
+        }
+        out[oi] = o;
+      }
+    }
+    __syncthreads();  // s_ch and the staged query rows are rewritten by the next chunk
   }
 }
 
-cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
-                         float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
-                         const int *rows, int *next_chunk, int *last_rows, const TcGate *gate, int num_sms,
-                         cudaStream_t stream) {
-  const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr};
+cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const ChanInfo *chan,
+                         const float *shift, float *out, int H, int T, int d, int causal, const FixupEntry *entries,
+                         const int *count, const int *rows, int *next_chunk, int *last_rows, const TcGate *gate,
+                         int num_sms, cudaStream_t stream) {
+  const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr, nullptr};
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = num_sms * 3;
   if (d == 64) {
     const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
-    fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
-                                                          next_chunk, last_rows, g);
+    fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, chan, shift, out, H, T, causal, entries,
+                                                          count, rows, next_chunk, last_rows, g);
   } else if (d == 128) {
     const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
     cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
+    // two blocks per SM need the largest shared-memory carveout
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
-    fixup_kernel<128><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, shift, out, H, T, entries, count, rows,
-                                                           next_chunk, last_rows, g);
+    fixup_kernel<128><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, chan, shift, out, H, T, causal, entries,
+                                                           count, rows, next_chunk, last_rows, g);
   } else {
     return cudaErrorInvalidValue;
   }

@@ -8,7 +8,8 @@
 
 namespace fem {
 
-// Device workspace of the value-bank pre-pass (all arrays caller-owned).
+// Device workspace of one read (all arrays caller-owned): the value-bank
+// pre-pass's arrays and the exact fix-up's entry list.
 struct BankWorkspace {
   float4 *tstat;            // [B*H, key tiles, d]: max, min, sum of v per tile
   ChanInfo *chan;           // [B*H, d]
@@ -16,62 +17,73 @@ struct BankWorkspace {
   float *shift;             // [B*H, key tiles, d]: the bank's shift for each tile
   float *rfac;              // [B*H, key tiles, d]: exp(beta (shift[kt-1] - shift[kt])), 1 if unmoved
   unsigned *colmask;        // [B*H, key tiles, 4]: bit j set when channel j's shift moved at the tile
+  float *colsum;            // [B*H, key tiles, d]: sum of |bank| over the tile's keys
   __half *bank;             // [B*H, T, d]: the value bank, fp16
-  FixupEntry *fixups;       // exact-recompute list (causal)
+  FixupEntry *fixups;       // exact-recompute list, written by the tensor-core kernel
   int *fixup_count;         // its length in slots, a multiple of 8 (zeroed before the pre-pass)
   int *fixup_rows;          // rows listed (zeroed before the pre-pass)
   int *fixup_next;          // the fix-up's next unclaimed chunk (zeroed before the pre-pass)
-  int2 *tilefix;            // [B*H, key tiles] (causal): {first entry, number of rows} of the tile's
-                            // entries, which list the tile's rows 0 .. number-1 in order
 };
 
-// Statistics, plan and value bank (two reads of V, one write of the bank).
-// `tv` and `te` map V (bf16) and the bank (fp16) like the tensor-core kernel's
-// operands: boxes of 64 channels x 128 rows, 128-byte swizzle.
+// Capacity of the fix-up list in entries: every row, plus the padding of each
+// query tile's two blocks of entries to multiples of kFixChunk.
+inline size_t fixup_capacity(size_t BH, size_t T) {
+  const size_t n_qt = (T + kBlockQ - 1) / kBlockQ;
+  return BH * n_qt * (kBlockQ + 2 * (kFixChunk - 1));
+}
+
+// Statistics, plan and value bank (two reads of V, one write of the bank),
+// and the bank's column sums per key tile.  `tv` and `te` map V (bf16) and the
+// bank (fp16) like the tensor-core kernel's operands: boxes of 64 channels x
+// 128 rows, 128-byte swizzle.
 //
 // BankCoef, one float4 per (b, h, key tile, channel), written by the plan:
 //   linear bank   {1/beta (0 at beta = 0), beta, c_lin, NaN}
-//   shifted bank  {beta log2 e, (kBankOffset - beta c) log2 e, c, level}
-// with level = c - kHazardTilt/beta when the tile's keys are checked for the
-// causal diagonal hazard, -inf when not (not causal, or the running maximum
-// before the tile already reached it).  stats_ready: w.tstat already holds the
-// tiles' statistics of this V (they do not depend on beta); skip recomputing them.
+//   shifted bank  {beta log2 e, (kBankOffset - beta c) log2 e, c, 0}
+// stats_ready: w.tstat already holds the tiles' statistics of this V (they do
+// not depend on beta); skip recomputing them.
 cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtensorMap &te, const float *beta, int BH,
-                              int H, int T, int d, int causal, const BankWorkspace &w, unsigned *err, int num_sms,
+                              int H, int T, int d, const BankWorkspace &w, unsigned *err, int num_sms,
                               cudaStream_t stream, bool stats_ready = false);
 
 // Gates of the one-pass two-level gated read: o = g (mu + lambda (F - mu))
-// with mu the mean read (its bank v - c_lin, anchors chan0) and F the read at
-// beta_max.  lam, g: [B*H, T, d] fp32 inputs; mu_side: [B*H, T, d] fp32
-// scratch, written only at the fix-up entries (their mu, for the fix-up).
+// with mu the mean read (its bank v - c_lin, anchors chan0, column sums
+// colsum0) and F the read at beta_max.  lam, g: [B*H, T, d] fp32 inputs;
+// mu_side: [B*H, T, d] fp32 scratch, written only at the fix-up entries
+// (their mu, for the fix-up).
 struct TcGate {
   const float *lam, *g;
   float *mu_side;
   const ChanInfo *chan0;
+  const float *colsum0;
 };
 
-// Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d.
-// `out` is the fp32 output [B*H, T, d], 16-byte aligned.  For the
-// rows of a causal diagonal tile that have fix-up entries the kernel writes,
-// in place of the listed channels' outputs, their accumulator before the
-// diagonal tile, and the row's (max, sum) before it into the entry.  With
-// te0 (the mean's bank) and gate both given it runs the one-pass gated read;
-// with neither the plain read.
+// Tensor-core read.  Returns cudaErrorInvalidValue for an unsupported d or
+// size.  `out` is the fp32 output [B*H, T, d], 16-byte aligned.  Entries the
+// underflow guard rejects are listed in w.fixups (w.fixup_count slots,
+// w.fixup_rows rows) for the fix-up; for entries that restart from the state
+// before their diagonal tile the kernel writes, in place of the listed
+// channels' outputs, their accumulator before that tile.  With te0 (the mean's
+// bank) and gate both given it runs the one-pass gated read; with neither the
+// plain read.
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
-                      const CUtensorMap *te0, float *out, const float *beta, const ChanInfo *chan, const float *shift,
-                      const float *rfac, const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse,
+                      const CUtensorMap *te0, float *out, const float *beta, const BankWorkspace &w, float *lse,
                       int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream);
 
-// Completes the listed (row, channel) outputs: the diagonal tile's keys
-// exactly, merged with the state the tensor-core kernel left for the earlier
-// key tiles.
-// gate: nullptr, or the one-pass gated read's gates (the entries' outputs are
-// then gated with the mu the tensor-core kernel left in gate->mu_side).
+// Largest sequence length launch_tc takes (its shared-memory bitmap of moved key tiles).
+constexpr int kMaxSeqLen = 8192 * kBlockK;
+
+// Recomputes the listed (row, channel) outputs exactly in fp32, from the
+// entry's kt0 on (see FixupEntry), for the read at beta with channel modes
+// `chan` and shifts `shift` (those of the bank the tensor-core kernel used).
+// gate: nullptr, or the one-pass gated read's gates (an entry restarting
+// from its diagonal tile is then gated with the mu the tensor-core kernel
+// left in gate->mu_side; a full recomputation computes mu as well).
 // next_chunk: a zeroed counter from which the blocks claim chunks of entries.
-cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const float *shift,
-                         float *out, int H, int T, int d, const FixupEntry *entries, const int *count,
-                         const int *rows, int *next_chunk, int *last_rows, const TcGate *gate, int num_sms,
-                         cudaStream_t stream);
+cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const ChanInfo *chan,
+                         const float *shift, float *out, int H, int T, int d, int causal, const FixupEntry *entries,
+                         const int *count, const int *rows, int *next_chunk, int *last_rows, const TcGate *gate,
+                         int num_sms, cudaStream_t stream);
 
 
 // Decode read of one query per (b, h) against T cached keys: per-CTA key-chunk

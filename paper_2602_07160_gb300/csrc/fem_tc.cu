@@ -24,10 +24,21 @@
 //                the joint online rescale of acc by alpha * exp(beta_j (c_old -
 //                c_new)), over every column when a row maximum moved, over the
 //                moved channels when only channel shifts moved.  Off the
-//                softmax's path, it overlaps the next tile's exponentials
+//                softmax's path, it overlaps the next tile's exponentials.
+//                Thread j also keeps channel j's sum of |bank| over the key
+//                tiles read, rescaled with the shifts (the guard's Ecol_j)
 //   warps 4-11   epilogue, half the columns each:
 //                o = c + log1p(beta acc/L)/beta (linear bank) or
-//                o = c + (log(acc/L) - kappa)/beta (shifted bank); lse = m + log L.
+//                o = c + (log(acc/L) - kappa)/beta (shifted bank); lse = m + log L;
+//                the underflow guard (kGuardTau) on every entry, and the
+//                rejected entries listed for the exact fix-up.
+//
+// Causal diagonal tile (the last key tile of a query tile, when there are
+// earlier ones): its P E goes into a free score buffer instead of acc, and
+// the epilogue adds acc (rescaled by that tile's alpha and shift factors) to
+// it.  acc therefore still holds the state before the diagonal tile, from
+// which the fix-up restarts rows whose final state fails the guard but whose
+// earlier state passes it.
 //
 // sum_i exp(s_i - m) E_ij is the free energy's numerator up to the
 // stabilising shifts and L its normaliser (Sec. 2.3, Eq.
@@ -36,7 +47,8 @@
 // implementation").
 //
 // TMEM (512 columns): score buffers [0,128) [128,256) [256,384), acc
-// [384, 384 + D).  Shared memory: Q, K[3], E[2] tiles of [128 x D] 16-bit
+// [384, 384 + D); the diagonal tile's P E goes to score buffer nk mod 3.
+// Shared memory: Q, K[3], E[2] tiles of [128 x D] 16-bit
 // elements in the 128-byte-swizzle layout TMA writes (64-element column
 // blocks of 128 rows x 128 bytes, chunk c of row r at chunk c ^ (r & 7)),
 // then barriers and per-channel state.  Every mbarrier completes once per use
@@ -66,21 +78,30 @@ struct TcLayout {
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kChan = kBar + 512;               // per-channel epilogue coefficients
   static constexpr uint32_t kMoveBits = kChan + 4 * D * 4 + (GATED ? 4 * D : 0);  // 1 bit per key tile: a shift moved
-  static constexpr int kMaxKeyTiles = 8192;                  // T <= 1M keys
-  // side ring: per key tile its rescale factors exp(beta_j (c_old - c_new)) [D]
-  // and moved-channel mask [4], loaded with the K tile, kSideStages tiles deep
+  static constexpr int kMaxKeyTiles = kMaxSeqLen / kBlockK;  // T <= 1M keys
+  // side ring: per key tile its rescale factors exp(beta_j (c_old - c_new)) [D],
+  // the bank's column sums [D] (GATED: also the mean bank's [D]) and the
+  // moved-channel mask [4], loaded with the K tile, kSideStages tiles deep
   static constexpr int kSideStages = 8;
+  static constexpr int kSideArrays = GATED ? 3 : 2;
   static constexpr uint32_t kSide = kMoveBits + kMaxKeyTiles / 8;
-  static constexpr uint32_t kSideStride = D * 4 + 128;
+  static constexpr uint32_t kSideMask = kSideArrays * D * 4;  // offset of the mask in a slot
+  static constexpr uint32_t kSideStride = kSideMask + 128;
   static constexpr uint32_t kAlpha = kSide + kSideStages * kSideStride;  // alpha per row, per score buffer
   static constexpr uint32_t kInvL = kAlpha + kBufS * 128 * 4;         // 1/L per row, for the epilogue
-  static constexpr uint32_t kBytes = kInvL + 128 * 4;
+  static constexpr uint32_t kPre = kInvL + 128 * 4;  // per row (m, L) before the diagonal tile
+  static constexpr uint32_t kGco = kPre + 128 * 8;   // per channel guard coefficients {X, Z, Y, Zp}
+  static constexpr uint32_t kThr = kGco + D * 16;    // per channel: the guard as a < A + B / L, {A, B}
+  static constexpr uint32_t kFlag = kThr + D * 8;    // per row and 32-channel group: entries the guard rejects
+  static constexpr uint32_t kBad = kFlag + 128 * 16;  // per row: restart from the diagonal tile not possible
+  static constexpr uint32_t kMisc = kBad + 128 * 4;   // entry counts and bases, guard bounds, row flags
+  static constexpr uint32_t kBytes = kMisc + 128;
   static constexpr uint32_t kAlloc = kBytes + 1024;
   static constexpr uint32_t kAccCol = kBufS * 128;
   static constexpr uint32_t kAccB = kAccCol + (GATED ? D : 0);  // the beta (or beta_max) read's accumulator
   static_assert(kAccCol + kNB * D <= 512, "TMEM columns");
   static_assert(kBytes <= 227 * 1024 - 1024, "shared memory");
-  static_assert(kNB * D / 32 * 16384 + 4 * 128 * 4 <= (kStagesK * kTile + kSlotsE * kTile),
+  static_assert(kNB * D / 32 * 16384 <= (kStagesK * kTile + kSlotsE * kTile),
                 "epilogue staging fits the idle K and E rings");
 };
 
@@ -101,6 +122,8 @@ enum : int {
 };
 
 constexpr int kHeadGroup = 8;  // heads whose query tiles the launch order interleaves
+
+__device__ __forceinline__ int pad_chunk(int n) { return (n + kFixChunk - 1) / kFixChunk * kFixChunk; }
 
 // Bounded wait that also gives up as soon as another role has given up.
 __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, unsigned *err, unsigned code,
@@ -127,11 +150,8 @@ template <int D, bool GATED>
 __global__ void __launch_bounds__(384, 1)
     fem_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_e0,
-                  float *__restrict__ out, const float *__restrict__ beta,
-                  const ChanInfo *__restrict__ chan, const float *__restrict__ shift,
-                  const float *__restrict__ rfac, const unsigned *__restrict__ colmask,
-                  const int2 *__restrict__ tilefix, FixupEntry *__restrict__ fixups, float *__restrict__ lse, int H,
-                  int T, int causal, TcGate gate, unsigned *__restrict__ err) {
+                  float *__restrict__ out, const float *__restrict__ beta, const BankWorkspace w,
+                  float *__restrict__ lse, int H, int T, int causal, TcGate gate, unsigned *__restrict__ err) {
   using Lay = TcLayout<D, GATED>;
   constexpr int kNB = Lay::kNB, kBufS = Lay::kBufS, kStagesK = Lay::kStagesK, kSlotsE = Lay::kSlotsE;
   extern __shared__ uint8_t smem_raw[];
@@ -161,6 +181,10 @@ __global__ void __launch_bounds__(384, 1)
   const int bh = g0 + idx % gsz, h = bh % H;
   const int qt = causal ? n_qt - 1 - idx / gsz : idx / gsz;
   const int nk = causal ? qt + 1 : n_kt_all;  // key tiles this query tile reads
+  // causal with earlier key tiles: the diagonal tile's P E (of the beta bank)
+  // goes to the score buffer no other tile uses from then on, so acc keeps
+  // the state before it
+  const bool split = causal && nk > 1;
 
   // K tile kt into K stage kt % kStagesK, with its side data into side slot
   // kt % 8.  Side slot kt % 8 was last read by the correction of tile kt - 8,
@@ -173,9 +197,12 @@ __global__ void __launch_bounds__(384, 1)
       tma_load_3d(sbase + Lay::kK + st * Lay::kTile + b * 16384, &tmap_k, FEM_BAR(kBarKFull + st), b * 64,
                   kt * kBlockK, bh);
     const size_t row = static_cast<size_t>(bh) * n_kt_all + kt;
-    mbar_arrive_expect_tx(FEM_BAR(kBarSide + ss), D * 4 + 16);
-    bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride, rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
-    bulk_load(sbase + Lay::kSide + ss * Lay::kSideStride + D * 4, colmask + row * 4, 16, FEM_BAR(kBarSide + ss));
+    const uint32_t slot = sbase + Lay::kSide + ss * Lay::kSideStride;
+    mbar_arrive_expect_tx(FEM_BAR(kBarSide + ss), Lay::kSideMask + 16);
+    bulk_load(slot, w.rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
+    bulk_load(slot + D * 4, w.colsum + row * D, D * 4, FEM_BAR(kBarSide + ss));
+    if (GATED) bulk_load(slot + 2 * D * 4, gate.colsum0 + row * D, D * 4, FEM_BAR(kBarSide + ss));
+    bulk_load(slot + Lay::kSideMask, w.colmask + row * 4, 16, FEM_BAR(kBarSide + ss));
   };
   // E item e (key tile e / kNB; bank e % kNB, the mean's first when GATED)
   // into E slot e % kSlotsE
@@ -224,13 +251,13 @@ __global__ void __launch_bounds__(384, 1)
     for (int e = 0; e < min(ne, kPreE); ++e) load_e(e);
   }
   for (int j = tid; j < D; j += 384) {
-    const ChanInfo ci = chan[bh * D + j];
+    const ChanInfo ci = w.chan[bh * D + j];
     const float bj = beta[h * D + j];
     const bool lin = ci.linear != 0.f;
     if (lin) {
       c_coef[j] = make_float4(bj, ci.c_lin, bj != 0.f ? kLn2 / bj : 0.f, 0.f);
     } else {
-      const float c = shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j];
+      const float c = w.shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j];
       c_coef[j] = make_float4(0.f, c - kBankOffset / bj, kLn2 / bj, 1.f);
     }
     // the mean's anchor: its bank holds v - c, so mu = c + acc/L
@@ -241,16 +268,22 @@ __global__ void __launch_bounds__(384, 1)
     const int t = base + tid;
     bool moved = false;
     if (t < nk) {
-      const uint4 m = reinterpret_cast<const uint4 *>(colmask)[static_cast<size_t>(bh) * n_kt_all + t];
+      const uint4 m = reinterpret_cast<const uint4 *>(w.colmask)[static_cast<size_t>(bh) * n_kt_all + t];
       moved = (m.x | m.y | m.z | m.w) != 0u;
     }
     const unsigned bits = __ballot_sync(0xffffffffu, moved);
     if (lane == 0) move_bits[(base >> 5) + warp] = bits;
   }
+  if (tid == 0) {
+    reinterpret_cast<float *>(smem + Lay::kMisc)[4] = 0.f;        // the mean bank's largest guard bound
+  }
+  if (tid < 128) reinterpret_cast<unsigned *>(smem + Lay::kBad)[tid] = 0u;
+  if (tid < 4) reinterpret_cast<unsigned *>(smem + Lay::kMisc)[16 + tid] = 0u;  // rows with listed entries
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem + Lay::kTmemSlot);
+  const uint32_t tDiag = tmem + static_cast<uint32_t>((nk % kBufS) * 128);
 
   // Every warp keeps the launch's register count: moving registers from the
   // producer warps to the softmax (setmaxnreg) made the compiled code spill
@@ -312,17 +345,25 @@ __global__ void __launch_bounds__(384, 1)
       for (int kt = 0; ok && kt < nk; ++kt) {
         const int b = kt % kBufS;
         if (!(ok = wait_or_abort(FEM_BAR(kBarPFull + b), (kt / kBufS) & 1, err, kErrWaitMma, abort_flag))) break;
-        // each bank of the tile into its accumulator, D columns apart
+        // each bank of the tile into its accumulator, D columns apart; the
+        // beta bank of a split diagonal tile into its own buffer
 #pragma unroll
         for (int part = 0; part < kNB; ++part) {
           const int e = kt * kNB + part, st = e % kSlotsE;
           if (!(ok = wait_or_abort(FEM_BAR(kBarEFull + st), (e / kSlotsE) & 1, err, kErrWaitTma, abort_flag))) break;
           tc_fence_after_sync();
           const uint32_t sE = sbase + Lay::kE + st * Lay::kTile;
+          const bool to_diag = split && kt == nk - 1 && part == kNB - 1;
+          // the diagonal tile's buffer was last read by the P E of tile nk - kBufS
+          if (to_diag && nk >= kBufS &&
+              !(ok = wait_or_abort(FEM_BAR(kBarPvDone + nk % kBufS), ((nk - kBufS) / kBufS) & 1, err, kErrWaitMma,
+                                   abort_flag)))
+            break;
+          const uint32_t dst = to_diag ? tDiag : tAcc + part * D;
 #pragma unroll
           for (int kk = 0; kk < kBlockK / 16; ++kk)
-            mma_f16_ts(tAcc + part * D, tmem + b * 128 + kk * 8, smem_desc_sw128(sE + kk * 2048, 16384, 1024),
-                       idesc_pv, (kt > 0 || kk > 0) ? 1u : 0u);
+            mma_f16_ts(dst, tmem + b * 128 + kk * 8, smem_desc_sw128(sE + kk * 2048, 16384, 1024), idesc_pv,
+                       ((kt > 0 && !to_diag) || kk > 0) ? 1u : 0u);
           mma_commit(FEM_BAR(kBarEEmpty + st));
         }
         if (!ok) break;
@@ -340,23 +381,14 @@ __global__ void __launch_bounds__(384, 1)
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t tAcc = tmem + Lay::kAccCol + lane_off;  // every accumulator column
     const uint32_t tAccB = tmem + Lay::kAccB + lane_off;   // the beta read's
+    const uint32_t tDiagL = tDiag + lane_off;
     float *s_alpha = reinterpret_cast<float *>(smem + Lay::kAlpha);
     float *s_invL = reinterpret_cast<float *>(smem + Lay::kInvL);
-    // Rows 0 .. hz_rows-1 of a causal diagonal tile may have fix-up entries
-    // (entry hz_base + r): for them the accumulator before the diagonal tile is
-    // kept in a free score buffer (the stash) and written out in place of the
-    // listed channels' outputs, and (m, L) before it go into the entry.
-    int hz_base = 0, hz_rows = 0;
-    if (causal) {
-      const int2 tf = tilefix[static_cast<size_t>(bh) * n_kt_all + qt];
-      hz_base = tf.x;
-      hz_rows = tf.y;
-    }
-    const bool hz_warp = hz_rows > 32 * (warp & 3);  // warp-uniform
-    const bool hz_row = r < hz_rows;
-    // the score buffer no tile after the diagonal one uses; its last P E
-    // completed before the correction of the diagonal tile fills it
-    const uint32_t tStash = tmem + (nk % kBufS) * 128 + lane_off;
+    float2 *s_pre = reinterpret_cast<float2 *>(smem + Lay::kPre);
+    float4 *s_gco = reinterpret_cast<float4 *>(smem + Lay::kGco);
+    unsigned *s_flag = reinterpret_cast<unsigned *>(smem + Lay::kFlag);  // [128][4]
+    unsigned *s_bad = reinterpret_cast<unsigned *>(smem + Lay::kBad);
+    int *s_misc = reinterpret_cast<int *>(smem + Lay::kMisc);
     float m_row = -INFINITY, L_row = 0.f;
     bool ok = true;
     if (is_sm) {
@@ -402,11 +434,7 @@ __global__ void __launch_bounds__(384, 1)
         }
         s_alpha[b * 128 + r] = alpha;
         mbar_arrive(FEM_BAR(kBarAlpha + b));
-        if (hz_row && kt == nk - 1) {
-          // diagonal tile: the row's state before it, for the fix-up
-          fixups[hz_base + r].m_pre = m_old;
-          fixups[hz_base + r].l_pre = L_row;
-        }
+        if (kt == nk - 1) s_pre[r] = make_float2(m_old, L_row);  // the row's state before its last key tile
         // P = exp2(s * scale - m) as fp16 over the first 64 columns of the buffer; L from the fp32 values
         const float2 scale2 = make_float2(qk_scale, qk_scale), negm2 = make_float2(-m_row, -m_row);
         float2 ls[4];
@@ -435,6 +463,11 @@ __global__ void __launch_bounds__(384, 1)
     }
     else {
       // ------------------------------------------------------------ correction
+      // thread j < D: channel j's sum of |bank| over the key tiles read so far,
+      // in the units of the current shift (and the mean bank's, GATED), and
+      // the same before the diagonal tile
+      float ecol = 0.f, ecol_pre = 0.f, ecol0 = 0.f;
+      const float beta_r = r < D ? beta[h * D + r] : 0.f;  // for the guard's coefficients after the loop
       for (int kt = 0; kt < nk; ++kt) {
         const int b = kt % kBufS;
         ok = __all_sync(0xffffffffu,
@@ -443,20 +476,28 @@ __global__ void __launch_bounds__(384, 1)
         const float alpha = s_alpha[b * 128 + r];
         const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
         const bool rowmv = __any_sync(0xffffffffu, alpha != 1.f);
-        const bool stash = hz_warp && kt == nk - 1;  // diagonal tile of rows with fix-up entries
-        if (kt > 0 && (rowmv || colmv || stash)) {
-          // this tile's rescale factors exp(beta_j (c_old - c_new)), 1 for unmoved
-          // channels, and its moved-channel mask, loaded tiles ahead with K
-          const float *rf =
-              reinterpret_cast<const float *>(smem + Lay::kSide + (kt % Lay::kSideStages) * Lay::kSideStride);
+        const bool last_split = split && kt == nk - 1;  // acc keeps its state; the epilogue rescales
+        // this tile's rescale factors exp(beta_j (c_old - c_new)), 1 for unmoved
+        // channels, its column sums and its moved-channel mask, loaded tiles
+        // ahead with K
+        const float *rf =
+            reinterpret_cast<const float *>(smem + Lay::kSide + (kt % Lay::kSideStages) * Lay::kSideStride);
+        ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSide + kt % Lay::kSideStages),
+                                                   (kt / Lay::kSideStages) & 1, err, kErrWaitTma, abort_flag));
+        if (!ok) break;
+        if (r < D) {
+          if (last_split) ecol_pre = ecol;
+          ecol = fmaf(ecol, rf[r], rf[D + r]);
+          if (GATED) ecol0 += rf[2 * D + r];
+        }
+        const bool do_b = !last_split && (rowmv || colmv);  // the beta accumulator needs a rescale
+        const bool do_m = GATED && rowmv;                    // the mean's accumulator
+        if (kt > 0 && (do_b || do_m)) {
           unsigned gm = 0;  // 32-column groups holding a moved channel
           int g0 = 0;
           float f0[32];  // factors of the first such group, read before acc is ready
-          if (colmv) {
-            ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSide + kt % Lay::kSideStages),
-                                                       (kt / Lay::kSideStages) & 1, err, kErrWaitTma, abort_flag));
-            if (!ok) break;
-            const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + D);
+          if (colmv && do_b) {
+            const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + Lay::kSideMask / 4);
             gm = (m4.x ? 1u : 0u) | (m4.y ? 2u : 0u) | (m4.z ? 4u : 0u) | (m4.w ? 8u : 0u);
             g0 = __ffs(gm) - 1;
 #pragma unroll
@@ -468,28 +509,19 @@ __global__ void __launch_bounds__(384, 1)
                                                      kErrWaitMma, abort_flag));
           if (!ok) break;
           tc_fence_after_sync();
-          if (stash) {
+          if (do_m) {
+            // the mean's accumulator: the row maximum's factor only
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
               uint32_t v[32];
-              tmem_ld32(tAccB + c * 32, v);
+              tmem_ld32(tAcc + c * 32, v);
               tmem_ld_wait();
-              tmem_st32(tStash + c * 32, v);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+              tmem_st32(tAcc + c * 32, v);
             }
           }
-          if (rowmv) {
-            if (GATED) {
-              // the mean's accumulator: the row maximum's factor only
-#pragma unroll 1
-              for (int c = 0; c < D / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld32(tAcc + c * 32, v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-                tmem_st32(tAcc + c * 32, v);
-              }
-            }
+          if (do_b && rowmv) {
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
               uint32_t v[32];
@@ -504,7 +536,7 @@ __global__ void __launch_bounds__(384, 1)
               }
               tmem_st32(tAccB + c * 32, v);
             }
-          } else if (colmv) {
+          } else if (do_b && colmv) {
             {
               uint32_t v[32];
               tmem_ld32(tAccB + g0 * 32, v);
@@ -532,13 +564,32 @@ __global__ void __launch_bounds__(384, 1)
         tc_fence_before_sync();
         mbar_arrive(FEM_BAR(kBarPFull + b));
       }
+      // the guard's coefficients of channel j: an entry is rejected when
+      //   X a + Z / L < Y          (final state, a = acc / L)
+      //   X a_pre + Zp < Y L_pre   (state before the diagonal tile)
+      // with X = tau beta, Z = -2^-25 Ecol, Zp = -2^-25 Ecol_pre and Y = 2^-25
+      // (shifted bank) or -tau (linear bank); see kGuardTau
+      if (r < D) {
+        const bool lin = c_coef[r].w == 0.f;
+        const float4 g = make_float4(kGuardTau * beta_r, -kGuardUlp * ecol, lin ? -kGuardTau : kGuardUlp, -kGuardUlp * ecol_pre);
+        s_gco[r] = g;
+        // the same test on the final state as a < A + B / L: A = Y / X, B = -Z / X for
+        // X > 0; at beta = 0 (X = 0, linear) it holds for no L >= 1 unless -Z > tau,
+        // in which case every entry of the channel goes to the exact test
+        reinterpret_cast<float2 *>(smem + Lay::kThr)[r] =
+            g.x > 0.f ? make_float2(g.z / g.x, -g.y / g.x) : make_float2(-g.y > kGuardTau ? INFINITY : -INFINITY, 0.f);
+        // the mean bank (linear, beta = 0): rejected when 2^-25 Ecol0 / L > tau;
+        // the CTA keeps the largest 2^-25 Ecol0 (positive floats order as integers)
+        if (GATED) atomicMax(reinterpret_cast<int *>(smem + Lay::kMisc) + 4, __float_as_int(kGuardUlp * ecol0));
+      }
     }
     // ---- epilogue, half the channels per warpgroup.  acc/L is staged in
     // shared memory (the K and E rings are idle once every contraction
-    // completed) as 32-column boxes, row r by thread r; the transform then
-    // runs column-parallel and writes each row's 32 columns of a box as one
-    // coalesced 128-byte store.  GATED: boxes 0 .. D/32-1 hold the mean's
-    // accumulator, boxes D/32 .. 2D/32-1 the beta_max read's.
+    // completed) as 32-column boxes, row r by thread r, and checked by the
+    // underflow guard; the transform then runs column-parallel and writes each
+    // row's 32 columns of a box as one coalesced 128-byte store.  GATED: boxes
+    // 0 .. D/32-1 hold the mean's accumulator, boxes D/32 .. 2D/32-1 the
+    // beta_max read's.
     if (ok) ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarAccDone), 0, err, kErrWaitMma, abort_flag));
     ok = bar_and(1, 256, ok);  // both warpgroups went through every key tile
     if (ok) {
@@ -547,18 +598,24 @@ __global__ void __launch_bounds__(384, 1)
       constexpr int NC = D / 64;             // 32-column chunks of this warpgroup
       constexpr int kBoxB = (kNB - 1) * (D / 32);  // first box of the beta read
       const int c_lo = is_sm ? 0 : NC;
-      // (row, chunk) masks of the channels a fix-up row lists, in the idle
-      // rings behind the staging boxes
-      unsigned *s_hzm = reinterpret_cast<unsigned *>(smem + Lay::kK + kNB * (D / 32) * 16384);
-#pragma unroll 1
-      for (int part = 0; part < kNB; ++part) {
+      const bool row_ok = t_row < T;
+      // GATED: the mean bank's guard for the whole row (its bound is per channel;
+      // the largest one stands for all)
+      const bool mean_bad = GATED && reinterpret_cast<const float *>(smem + Lay::kMisc)[4] * invL > kGuardTau;
+      const float2 pre = s_pre[r];  // (m, L) before the last key tile
+      const float alpha_last = split ? s_alpha[((nk - 1) % kBufS) * 128 + r] : 1.f;
+      const float *rf_last =
+          reinterpret_cast<const float *>(smem + Lay::kSide + ((nk - 1) % Lay::kSideStages) * Lay::kSideStride);
+      unsigned bad = 0;  // a rejected entry whose state before the diagonal tile is rejected too
+      const float2 *s_ab = reinterpret_cast<const float2 *>(smem + Lay::kThr);
+      if (GATED) {
         uint32_t v[NC][32];
 #pragma unroll
-        for (int c = 0; c < NC; ++c) tmem_ld32(tAcc + part * D + (c_lo + c) * 32, v[c]);
+        for (int c = 0; c < NC; ++c) tmem_ld32(tAcc + (c_lo + c) * 32, v[c]);
         tmem_ld_wait();
 #pragma unroll
         for (int c = 0; c < NC; ++c) {
-          uint8_t *box = smem + Lay::kK + (part * (D / 32) + c_lo + c) * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
+          uint8_t *box = smem + Lay::kK + (c_lo + c) * 16384;  // 128 rows x 32 fp32, 128-byte swizzle
 #pragma unroll
           for (int i4 = 0; i4 < 8; ++i4)
             *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) =
@@ -566,26 +623,106 @@ __global__ void __launch_bounds__(384, 1)
                             __uint_as_float(v[c][4 * i4 + 2]) * invL, __uint_as_float(v[c][4 * i4 + 3]) * invL);
         }
       }
-      if (hz_warp) {
-        // listed channels of fix-up rows: the beta read's accumulator before
-        // the diagonal tile, staged in place of acc/L and written out untransformed
+      // the diagonal tile's factors: alpha of the row, exp(beta (c_old - c_new)) of the channel
+      const bool scale_last =
+          split && (__any_sync(0xffffffffu, alpha_last != 1.f) || ((move_bits[(nk - 1) >> 5] >> ((nk - 1) & 31)) & 1u));
+      {
+        // chunk by chunk: acc (before the diagonal tile when split) plus the
+        // diagonal tile's P E, the guard's test, staged
+        bool cand = false;
 #pragma unroll 1
         for (int c = c_lo; c < c_lo + NC; ++c) {
-          uint32_t w[32];
-          if (qt > 0) {
-            tmem_ld32(tStash + c * 32, w);
-            tmem_ld_wait();
-          }
-          const unsigned mc = hz_row ? fixups[hz_base + r].mask[c] : 0u;
-          s_hzm[r * 4 + c] = mc;
-          uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
+          uint32_t va[32], vd[32];
+          tmem_ld32(tAccB + c * 32, va);
+          if (split) tmem_ld32(tDiagL + c * 32, vd);
+          tmem_ld_wait();
+          if (!split) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if ((mc >> i) & 1u)
-              reinterpret_cast<float *>(box + sw128_offset(r, i >> 2))[i & 3] = qt > 0 ? __uint_as_float(w[i]) : 0.f;
+            for (int i = 0; i < 32; ++i) vd[i] = va[i];
+          } else if (scale_last) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              vd[i] = __float_as_uint(fmaf(__uint_as_float(va[i]), alpha_last * rf_last[c * 32 + i], __uint_as_float(vd[i])));
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) vd[i] = __float_as_uint(__uint_as_float(va[i]) + __uint_as_float(vd[i]));
+          }
+          uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
+          const float4 *ab = reinterpret_cast<const float4 *>(s_ab + c * 32);
+#pragma unroll
+          for (int i4 = 0; i4 < 8; ++i4) {
+            const float4 p = ab[2 * i4], q = ab[2 * i4 + 1];  // {A, B} of four channels
+            const float a0 = __uint_as_float(vd[4 * i4]) * invL, a1 = __uint_as_float(vd[4 * i4 + 1]) * invL,
+                        a2 = __uint_as_float(vd[4 * i4 + 2]) * invL, a3 = __uint_as_float(vd[4 * i4 + 3]) * invL;
+            cand |= (a0 < fmaf(p.y, invL, p.x)) | (a1 < fmaf(p.w, invL, p.z)) | (a2 < fmaf(q.y, invL, q.x)) |
+                    (a3 < fmaf(q.w, invL, q.z));
+            *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(a0, a1, a2, a3);
+          }
+        }
+        cand = (cand || mean_bad) && row_ok;
+        if (__any_sync(0xffffffffu, cand)) {
+          // the exact guard on the candidate rows; a rejected entry's accumulator
+          // before the diagonal tile goes out in place of the output (the
+          // fix-up's starting state), and whether that state passes the guard
+          // decides where the fix-up starts
+#pragma unroll 1
+          for (int c = c_lo; c < c_lo + NC; ++c) {
+            uint32_t vp[32];
+            tmem_ld32(tAccB + c * 32, vp);
+            tmem_ld_wait();
+            unsigned fm = 0;
+            if (cand) {
+              uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
+              const float4 *gco = s_gco + c * 32;
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                float *cell = reinterpret_cast<float *>(box + sw128_offset(r, i >> 2)) + (i & 3);
+                const float4 g = gco[i];
+                const float2 t = s_ab[c * 32 + i];
+                if (!(mean_bad || *cell < fmaf(t.y, invL, t.x))) continue;
+                fm |= 1u << i;
+                const float a_pre = split ? __uint_as_float(vp[i]) : 0.f;
+                if (split && fmaf(g.x, a_pre, g.w) < g.z * pre.y) bad = 1;
+                *cell = a_pre;
+              }
+            }
+            s_flag[r * 4 + c] = fm;
+            if (fm) atomicOr(reinterpret_cast<unsigned *>(smem + Lay::kMisc) + 16 + (r >> 5), 1u << (r & 31));
+          }
+        } else {
+#pragma unroll
+          for (int c = c_lo; c < c_lo + NC; ++c) s_flag[r * 4 + c] = 0u;
         }
       }
-      bar_sync(is_sm ? 2 : 3, 128);
+      if (bad) atomicOr(s_bad + r, 1u);
+      bar_sync(4, 256);
+      // ---- list the rejected rows: one block of entries that restart from the
+      // diagonal tile, one of entries recomputed over every key tile, each padded
+      // to a multiple of kFixChunk rows (rows -1) for the fix-up's chunks.  The slots are
+      // reserved now and written after the transform, which hides the atomic.
+      const unsigned *rowflags = reinterpret_cast<const unsigned *>(smem + Lay::kMisc) + 16;
+      const bool any_listed = (rowflags[0] | rowflags[1] | rowflags[2] | rowflags[3]) != 0u;
+      int base = 0;  // thread 0 of the softmax warpgroup: the first reserved slot
+      if (any_listed && is_sm) {
+        const bool listed = (rowflags[r >> 5] >> (r & 31)) & 1u;
+        const bool diag = listed && split && s_bad[r] == 0u;
+        const unsigned bd = __ballot_sync(0xffffffffu, diag), bf = __ballot_sync(0xffffffffu, listed && !diag);
+        if (lane == 0) {
+          s_misc[8 + (warp & 3)] = __popc(bd);
+          s_misc[12 + (warp & 3)] = __popc(bf);
+        }
+        bar_sync(2, 128);
+        if (r == 0) {
+          int nd = 0, nf = 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            nd += s_misc[8 + q];
+            nf += s_misc[12 + q];
+          }
+          base = atomicAdd(w.fixup_count, pad_chunk(nd) + pad_chunk(nf));
+          atomicAdd(w.fixup_rows, nd + nf);
+        }
+      }
       // Thread r takes column r % 32 of a chunk and rows r / 32 + 4k, so its
       // channel's coefficients stay in registers, each warp access is one
       // 128-byte row of the box, and 8 loads at a time are in flight before the math.
@@ -594,8 +731,9 @@ __global__ void __launch_bounds__(384, 1)
       //                 or, for |x| < 2^-6 (also beta = 0), as c + a times the
       //                 series of log1p(x)/x
       // GATED: mu = c_mean + a_mean, F the beta_max read as above, and
-      // o = g (mu + lambda (F - mu)); a listed fix-up entry gets the stashed
-      // accumulator in out and mu in the gate's side buffer instead.
+      // o = g (mu + lambda (F - mu)).  A listed entry gets the staged value
+      // itself (the accumulator before its diagonal tile) and, GATED, its mu in
+      // the gate's side buffer.
       const int col = r & 31, row0 = r >> 5;
       const int rows_left = T - qt * kBlockQ;
       const size_t tile_off = (static_cast<size_t>(bh) * T + static_cast<size_t>(qt) * kBlockQ) * D + col;
@@ -629,6 +767,8 @@ __global__ void __launch_bounds__(384, 1)
               gv[k] = __ldcs(gate.g + oi);
             }
           }
+          // rows of this batch with listed entries (row0 + 4 (k0 + k) lies in word k0 / 8, bit row0 + 4 k)
+          const unsigned rw = any_listed ? reinterpret_cast<const unsigned *>(smem + Lay::kMisc)[16 + (k0 >> 3)] : 0u;
           float o[8];
 #pragma unroll
           for (int k = 0; k < 8; k += 2) {
@@ -650,18 +790,18 @@ __global__ void __launch_bounds__(384, 1)
               const int row = row0 + 4 * (k0 + k);
               const float mu =
                   c_mean + *reinterpret_cast<const float *>(box_m + sw128_offset(row0 + 4 * (k0 + k), col >> 2));
-              if (row < hz_rows && ((s_hzm[row * 4 + c] >> col) & 1u)) {
+              if (((rw >> (row0 + 4 * k)) & 1u) && ((s_flag[row * 4 + c] >> col) & 1u)) {
                 o[k] = a[k];
-                gate.mu_side[tile_off + static_cast<size_t>(row) * D + c * 32] = mu;
+                if (row < rows_left) gate.mu_side[tile_off + static_cast<size_t>(row) * D + c * 32] = mu;
               } else {
                 o[k] = gv[k] * fmaf(lamv[k], o[k] - mu, mu);
               }
             }
-          } else if (hz_rows > 0) {
+          } else if (rw) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
               const int row = row0 + 4 * (k0 + k);
-              if (row < hz_rows && ((s_hzm[row * 4 + c] >> col) & 1u)) o[k] = a[k];
+              if (((rw >> (row0 + 4 * k)) & 1u) && ((s_flag[row * 4 + c] >> col) & 1u)) o[k] = a[k];
             }
           }
 #pragma unroll
@@ -669,6 +809,55 @@ __global__ void __launch_bounds__(384, 1)
             const int row = row0 + 4 * (k0 + k);
             if (row < rows_left) __stcs(out_tile + static_cast<size_t>(row) * D + c * 32, o[k]);
           }
+        }
+      }
+      // ---- the listed rows' entries, in the slots reserved before the transform
+      if (any_listed && is_sm) {
+        if (r == 0) s_misc[0] = base;
+        bar_sync(2, 128);
+        const int b0 = s_misc[0], wq = warp & 3;
+        int nd = 0, nf = 0, pd = 0, pf = 0;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int a = s_misc[8 + q], b = s_misc[12 + q];
+          nd += a;
+          nf += b;
+          pd += q < wq ? a : 0;
+          pf += q < wq ? b : 0;
+        }
+        const int sd = pad_chunk(nd), sf = pad_chunk(nf);
+        const bool listed = (rowflags[r >> 5] >> (r & 31)) & 1u;
+        const bool diag = listed && split && s_bad[r] == 0u;
+        const unsigned bd = __ballot_sync(0xffffffffu, diag), bf = __ballot_sync(0xffffffffu, listed && !diag);
+        const unsigned below = (1u << lane) - 1u;
+        if (listed) {
+          const float2 pr = s_pre[r];
+          FixupEntry e;
+          e.row = bh * T + t_row;
+#pragma unroll
+          for (int g = 0; g < 4; ++g) e.mask[g] = g < D / 32 ? s_flag[r * 4 + g] : 0u;
+          e.m_pre = pr.x;
+          e.l_pre = pr.y;
+          e.kt0 = diag ? nk - 1 : 0;
+          // a recomputation from the first key tile keeps the mean the kernel
+          // left aside unless the mean bank's own guard rejected it (l_pre = 1)
+          if (!diag)
+            e.l_pre = (GATED && reinterpret_cast<const float *>(smem + Lay::kMisc)[4] * s_invL[r] > kGuardTau) ? 1.f
+                                                                                                                : 0.f;
+          w.fixups[diag ? b0 + pd + __popc(bd & below) : b0 + sd + pf + __popc(bf & below)] = e;
+        }
+        FixupEntry padding;
+        padding.row = -1;
+        padding.mask[0] = padding.mask[1] = padding.mask[2] = padding.mask[3] = 0u;
+        padding.m_pre = -INFINITY;
+        padding.l_pre = 0.f;
+        if (r < sd - nd) {
+          padding.kt0 = nk - 1;
+          w.fixups[b0 + nd + r] = padding;
+        }
+        if (r < sf - nf) {
+          padding.kt0 = 0;
+          w.fixups[b0 + sd + nf + r] = padding;
         }
       }
     }
@@ -685,10 +874,9 @@ __global__ void __launch_bounds__(384, 1)
 
 template <int D, bool GATED>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
-                               const CUtensorMap &te0, float *out, const float *beta, const ChanInfo *chan,
-                               const float *shift, const float *rfac, const unsigned *colmask, const int2 *tilefix,
-                               FixupEntry *fixups, float *lse, int BH, int H, int T, int causal, const TcGate &gate,
-                               unsigned *err, cudaStream_t stream) {
+                               const CUtensorMap &te0, float *out, const float *beta, const BankWorkspace &w,
+                               float *lse, int BH, int H, int T, int causal, const TcGate &gate, unsigned *err,
+                               cudaStream_t stream) {
   using Lay = TcLayout<D, GATED>;
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   if (n_qt > Lay::kMaxKeyTiles || BH > 65535) return cudaErrorInvalidValue;
@@ -696,32 +884,23 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
   cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D, GATED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const dim3 grid(n_qt, BH);
-  fem_tc_kernel<D, GATED><<<grid, 384, smem, stream>>>(tq, tk, te, te0, out, beta, chan, shift, rfac, colmask, tilefix,
-                                                       fixups, lse, H, T, causal, gate, err);
+  fem_tc_kernel<D, GATED><<<grid, 384, smem, stream>>>(tq, tk, te, te0, out, beta, w, lse, H, T, causal, gate, err);
   return cudaGetLastError();
 }
 
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
-                      const CUtensorMap *te0, float *out, const float *beta, const ChanInfo *chan, const float *shift,
-                      const float *rfac, const unsigned *colmask, const int2 *tilefix, FixupEntry *fixups, float *lse,
+                      const CUtensorMap *te0, float *out, const float *beta, const BankWorkspace &w, float *lse,
                       int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream) {
-  const TcGate none = {nullptr, nullptr, nullptr, nullptr};
+  const TcGate none = {nullptr, nullptr, nullptr, nullptr, nullptr};
   if ((te0 != nullptr) != (gate != nullptr)) return cudaErrorInvalidValue;
   if (gate) {
-    if (d == 64)
-      return launch_tc_d<64, true>(tq, tk, te, *te0, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH,
-                                   H, T, causal, *gate, err, stream);
+    if (d == 64) return launch_tc_d<64, true>(tq, tk, te, *te0, out, beta, w, lse, BH, H, T, causal, *gate, err, stream);
     if (d == 128)
-      return launch_tc_d<128, true>(tq, tk, te, *te0, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH,
-                                    H, T, causal, *gate, err, stream);
+      return launch_tc_d<128, true>(tq, tk, te, *te0, out, beta, w, lse, BH, H, T, causal, *gate, err, stream);
     return cudaErrorInvalidValue;
   }
-  if (d == 64)
-    return launch_tc_d<64, false>(tq, tk, te, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H,
-                                  T, causal, none, err, stream);
-  if (d == 128)
-    return launch_tc_d<128, false>(tq, tk, te, te, out, beta, chan, shift, rfac, colmask, tilefix, fixups, lse, BH, H,
-                                   T, causal, none, err, stream);
+  if (d == 64) return launch_tc_d<64, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream);
+  if (d == 128) return launch_tc_d<128, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream);
   return cudaErrorInvalidValue;
 }
 

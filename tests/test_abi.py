@@ -44,7 +44,9 @@ def test_workspace_bytes(lib):
     assert lib.fem_fwd_workspace_bytes(1, 1, -3, 64, 1) == 0
     a = lib.fem_fwd_workspace_bytes(4, 16, 8192, 128, 1)
     b = lib.fem_fwd_workspace_bytes(4, 16, 8192, 128, 0)
-    assert a > b > 0 and a % 256 == 0 and b % 256 == 0
+    # both forms of the read keep the same arrays (the guard's fix-up list serves both)
+    assert a == b > 0 and a % 256 == 0
+    assert lib.fem_fwd_workspace_bytes(4, 16, 8192, 64, 1) < a
 
 
 def _call(lib, fn, q=16, k=16, v=16, beta=16, out=16, lse=0, B=1, H=1, T=8, d=64, causal=1):
@@ -71,6 +73,19 @@ def test_unsupported_head_dim(lib):
     assert _call(lib, "fem_fwd_f32", d=300) == 2
 
 
+@pytest.mark.parametrize("fn", ["fem_fwd", "fem_fwd_host", "fem_fwd_noalloc"])
+def test_sequence_beyond_the_tensor_core_limit_is_refused_synchronously(lib, fn):
+    """T above 2^20 keys (the tensor-core kernel's bitmap of key tiles) is refused on the host
+    with FEM_ERR_UNSUPPORTED before any CUDA call (the pointers are fakes)."""
+    assert _call(lib, fn, T=(1 << 20) + 1) == 2
+
+
+def test_workspace_variant_refuses_long_sequence_synchronously(lib):
+    p = lambda x: ctypes.c_void_p(x) if x else None  # noqa: E731  fake, never dereferenced
+    T = (1 << 20) + 1
+    assert lib.fem_fwd_ws(p(16), p(16), p(16), p(16), p(16), None, 1, 1, T, 64, 1, p(256), 1 << 40, None) == 2
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError):
         fem.load(str(tmp_path / "missing.so"))
@@ -92,6 +107,7 @@ def test_gated_argument_errors_are_synchronous(lib):
     assert call(lam=24) == 1  # not 16-byte aligned
     assert call(b=0) == 1
     assert call(d=32) == 2
+    assert f(p(16), p(16), p(16), p(16), p(16), p(16), p(16), None, 1, 1, (1 << 20) + 1, 64, 1, None) == 2
 
 
 def test_decode_argument_errors_are_synchronous(lib):
