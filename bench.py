@@ -53,7 +53,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle CPU-baseline budget")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-context", action="store_true", help="skip the torch SDPA context timing")
+    ap.add_argument("--no-context", action="store_true", help="skip the context timings (SDPA, secondary reads)")
+    ap.add_argument("--no-workloads", action="store_true", help="skip the per-workload records")
+    ap.add_argument("--workload-seconds", type=float, default=2.0, help="oracle budget per workload record")
     ap.add_argument("--shape", default=None,
                     help="B,H,T override of the workload sizes (profiling aid; the JSON config reports them)")
     return ap.parse_args()
@@ -274,6 +276,83 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def time_cuda(fn, stream, warmup, iters):
+    """Mean ms per call of fn() over iters calls after warmup calls (CUDA events on stream)."""
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(iters):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / iters
+
+
+def workload_records(args, device, stream):
+    """One record per synthetic workload at 1 GPU: the read's time and throughput against
+    its roofline, the attention-mode comparator on the same inputs (bf16 workloads), the
+    fix-up's row count, and the oracle on a bounded sample of the workload on the host."""
+    import numpy as np
+    import torch
+
+    from paper_2602_07160_gb300 import fem
+    from paper_2602_07160_gb300 import workloads as W
+
+    peak, _ = bf16_peak()
+    hbm = hbm_peak()
+    recs = {}
+    for name, w in W.WORKLOADS.items():
+        q, k, v, beta = W.make_inputs(w)
+        qd, kd, vd, bd = (x.to(device) for x in (q, k, v, beta))
+        out = torch.empty(q.shape, dtype=torch.float32, device=device)
+        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=device)
+        elem = q.element_size()
+        io_bytes = 3 * q.numel() * elem + out.numel() * 4 + lse.numel() * 4
+        rec = {"config": w.describe(), "flops": w.flops, "algorithmic_bytes": io_bytes}
+        if w.dtype == "f32":
+            def call():
+                fem.fem_fwd_f32(qd, kd, vd, bd, causal=w.causal, out=out, lse=lse, stream=stream)
+            ms = time_cuda(call, stream, 5, 200)
+            rec.update({"path": "fem_fwd_f32 (CUDA cores, fp32)", "ms": ms, "us": ms * 1e3,
+                        "tflops": w.flops / (ms * 1e-3) / 1e12,
+                        "roofline": {"bound": "latency", "note": "a few microseconds of launch and one "
+                                     "dependent key loop per row; no throughput roofline applies"}})
+        else:
+            def call():
+                fem.fem_fwd(qd, kd, vd, bd, causal=w.causal, out=out, lse=lse, stream=stream)
+            iters = max(5, min(200, int(2000 / max(1.0, w.flops / 1e9))))
+            ms = time_cuda(call, stream, 3, iters)
+            fem.check_device_error(stream)
+            tf = w.flops / (ms * 1e-3) / 1e12
+            rec.update({"path": "fem_fwd (pre-pass, tcgen05 read, exact fix-up)", "ms": ms, "tflops": tf,
+                        "fixup_rows": fem.last_fixup_rows(stream)})
+            if name == "vit_s_full_prior":
+                gbs = io_bytes / (ms * 1e-3) / 1e9
+                rec["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
+                                   "note": "algorithmic bytes Q, K, V in, out and lse out; tensor fraction "
+                                           f"{tf / peak:.3f} of the bf16 peak"}
+            else:
+                rec["roofline"] = {"bound": "tensor", "achieved": tf, "peak": peak, "unit": "TFLOP/s",
+                                   "frac": tf / peak}
+
+            def attn():
+                fem.fem_attn_fwd(qd, kd, vd, causal=w.causal, out=out, lse=lse, stream=stream)
+            ams = time_cuda(attn, stream, 3, iters)
+            rec["attn_mode"] = {"ms": ams, "tflops": w.flops / (ams * 1e-3) / 1e12, "fem_over_attn": ms / ams}
+        # the oracle on the host cores, a bounded sample of the same workload
+        s = OracleSampler(w, q, k, v, beta)
+        val, n, dt = s.measure(args.workload_seconds)
+        rec["cpu_oracle"] = {"value": val, "unit": UNIT, "cores": s.threads, "rows": n, "seconds": dt,
+                             "rows_per_s": n / dt}
+        recs[name] = rec
+        del qd, kd, vd, bd, out, lse
+        torch.cuda.empty_cache()
+    return recs
+
+
 def run_fem(args):
     import numpy as np
     import torch
@@ -372,6 +451,18 @@ def run_fem(args):
                                         "(plain softmax attention: no value bank, no shifts)"}}
         except Exception as exc:  # context only; the FEM numbers stand without it
             context = {"sdpa": {"unavailable": str(exc)[:200]}}
+        # the build's own attention mode: the same tensor-core kernel with V in place of the bank
+        aout = torch.empty(q.shape, dtype=torch.float32, device=device)
+
+        def attn():
+            fem.fem_attn_fwd(qd, kd, vd, causal=w.causal, out=aout, lse=False, stream=stream)
+        attn_ms = time_cuda(attn, stream, 3, 20)
+        fem.check_device_error(stream)
+        context["attn_mode"] = {"ms": attn_ms, "tflops": w.flops / (attn_ms * 1e-3) / 1e12,
+                                "fem_overhead": ms_step / attn_ms - 1.0,
+                                "what": "fem_attn_fwd: plain softmax attention on the read's tcgen05 kernel (V in "
+                                        "place of the value bank, bf16 P; no pre-pass, shifts or guard)"}
+        del aout
         # the two-level gated read (one pass over the beta = 0 and beta_max banks)
         lam = torch.rand(q.shape, device=device)
         gate = torch.ones(q.shape, device=device)
@@ -497,6 +588,11 @@ def run_fem(args):
         e2e = {"value": job_throughput(w.flops, world, e2e_s * 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "steps": args.e2e_steps}
 
+    # ---- every synthetic workload at 1 GPU (rank 0, N = 1 only)
+    workloads = None
+    if rank == 0 and world == 1 and not args.no_workloads:
+        workloads = workload_records(args, device, stream)
+
     # ---- the oracle on the host cores (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -521,7 +617,8 @@ def run_fem(args):
             "cpu_baseline": cpu,
             "clocks": clk,
             "context": context,
-            "gpu_launches": K * (5 if w.causal else 4),  # stats, plan, bank, tensor-core read (+ fix-up)
+            "workloads": workloads,
+            "gpu_launches": K * 5,  # stats, plan, bank, tensor-core read, fix-up per step
         }
         print(json.dumps(line), flush=True)
     if dist is not None:

@@ -150,7 +150,7 @@ int fem_fwd_noalloc(const void *q, const void *k, const void *v,
  * the same prior weights mix two value banks, the mean's and beta_max's,
  * into two accumulators, and the epilogue applies the gates.  Allocates its
  * workspace stream-ordered on `stream`: fem_fwd's workspace twice (one per
- * bank) and, when causal, 4 B*H*T*d bytes written only at fix-up rows.
+ * bank) and 4 B*H*T*d bytes written only at the fix-up's entries.
  * Errors as fem_fwd; a null or misaligned lam or gate is
  * FEM_ERR_INVALID_ARG.
  */
@@ -242,6 +242,32 @@ int fem_bwd_f32(const float *q, const float *k, const float *v, const float *bet
  * FEM_ERR_CUDA if the synchronisation failed.
  */
 int fem_check_device_error(void *stream);
+
+/*
+ * fem_attn_fwd -- diagnostic comparator: plain softmax attention on the same
+ * tensor-core kernel, o_t = sum_i softmax(s_t)_i v_i (the read's beta -> 0
+ * limit, Prop. "app-baseline", and the prior mean of the two-level gated read,
+ * Sec. 3), with V itself (bf16) in place of the value bank: no pre-pass, no
+ * shifts, no underflow guard, P rounded to bf16 for the second contraction.
+ * It measures the cost of the free-energy read over attention at the same
+ * shapes.  Layout and rules as fem_fwd (no beta); lse as fem_fwd.  No
+ * workspace.
+ */
+int fem_attn_fwd(const void *q, const void *k, const void *v, float *out, float *lse, int B,
+                 int H, int T, int d, int causal, void *stream);
+
+/*
+ * fem_probe_wait_timeout -- diagnostic of the failure path; the paper has no
+ * counterpart.  Enqueues on `stream` one kernel whose single thread waits,
+ * with the same bounded-wait helper every kernel of the library uses, on a
+ * shared-memory mbarrier that nothing completes.  After limit_us
+ * microseconds (1 .. 1,000,000) the wait gives up, records the fact in the
+ * per-device error word and the kernel returns; fem_check_device_error()
+ * then reports FEM_ERR_TIMEOUT (and clears the word).  The kernel issues no
+ * copy and no tensor-core operation, so the context stays usable.  A
+ * limit_us of 0 or above 1,000,000 is FEM_ERR_INVALID_ARG.
+ */
+int fem_probe_wait_timeout(unsigned limit_us, void *stream);
 
 /*
  * fem_last_fixup_rows -- synchronises `stream` and returns the number of rows

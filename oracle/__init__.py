@@ -140,6 +140,21 @@ def gated_read(q, k, v, beta_max, lam, gate, causal: bool, nthreads: int = 0, li
     return gate * ((1.0 - lam) * mu + lam * fmax), lse
 
 
+def gated_read_rows(q, k, v, beta_max, lam, gate, causal: bool, rows, nthreads: int = 0, lib=None):
+    """gated_read on selected rows (flat indices (b*H + h)*T + t): the same
+    composition of the beta = 0 and beta_max reads of those rows.
+
+    lam, gate: [B, H, T, d].  Returns (out [n, d], lse [n]) as float64 numpy arrays."""
+    rows = np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+    beta_max = _f64(beta_max)
+    d = beta_max.shape[-1]
+    lam = _f64(lam).reshape(-1, d)[rows]
+    gate = _f64(gate).reshape(-1, d)[rows]
+    mu, lse = fem_read_rows(q, k, v, np.zeros_like(beta_max), causal, rows, nthreads=nthreads, lib=lib)
+    fmax, _ = fem_read_rows(q, k, v, beta_max, causal, rows, nthreads=nthreads, lib=lib)
+    return gate * ((1.0 - lam) * mu + lam * fmax), lse
+
+
 def decode_read(q, k, v, beta, nthreads: int = 0, lib=None):
     """Decode read: one query per (b, h) against a cache of T keys and values
     holding the query's own key and value, i.e. row T - 1 of the causal read

@@ -204,6 +204,19 @@ int static_scratch(void **out) {
   return FEM_OK;
 }
 
+// The error path of the bounded waits, exercised on purpose: one thread waits
+// on an mbarrier of its own that nothing arrives on, with the library's wait
+// helper and a short limit; the helper gives up, records kErrWaitProbe in the
+// error word and the kernel returns.  No copy or tensor-core operation is
+// issued, so nothing is left in flight.
+__global__ void wait_probe_kernel(unsigned *err, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(smem_u32(&bar), 1);
+  fence_mbar_init();
+  mbar_wait_for(smem_u32(&bar), 0, err, kErrWaitProbe, limit_ns);
+}
+
 }  // namespace
 }  // namespace fem
 
@@ -248,7 +261,7 @@ static BankWorkspace bank_workspace(uint8_t *ws, const WsLayout &w) {
 }
 
 // Gated part of a read: the mean's pre-pass workspace (ws_layout, non-causal)
-// and its zero beta, the gates, and mu_side (causal only).
+// and its zero beta, the gates, and mu_side (the mean at the fix-up entries).
 struct GatedArgs {
   uint8_t *ws0;
   const float *zero_beta, *lam, *g;
@@ -342,12 +355,13 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
   // workspace: the beta_max read's, the mean's pre-pass (non-causal layout),
-  // a zero beta [H, d], and mu_side [B, H, T, d] fp32 for causal fix-ups
+  // a zero beta [H, d], and mu_side [B, H, T, d] fp32 for the fix-up's entries
+  // (the guard can list entries of either mask)
   const size_t n = static_cast<size_t>(B) * H * T * d;
   const size_t ws_bytes = round256(fem_fwd_workspace_bytes(B, H, T, d, causal));
   const size_t ws0_bytes = round256(fem_fwd_workspace_bytes(B, H, T, d, 0));
   const size_t zb_bytes = round256(static_cast<size_t>(H) * d * sizeof(float));
-  const size_t mu_bytes = causal ? round256(n * sizeof(float)) : 0;
+  const size_t mu_bytes = round256(n * sizeof(float));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *buf = nullptr;
   cudaError_t e = ws_alloc(ds, &buf, ws_bytes + ws0_bytes + zb_bytes + mu_bytes, s);
@@ -358,7 +372,7 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   ga.zero_beta = reinterpret_cast<const float *>(p + ws_bytes + ws0_bytes);
   ga.lam = lam;
   ga.g = gate;
-  ga.mu_side = causal ? reinterpret_cast<float *>(p + ws_bytes + ws0_bytes + zb_bytes) : nullptr;
+  ga.mu_side = reinterpret_cast<float *>(p + ws_bytes + ws0_bytes + zb_bytes);
   e = cudaMemsetAsync(const_cast<float *>(ga.zero_beta), 0, static_cast<size_t>(H) * d * sizeof(float), s);
   rc = map_cuda(e);
   if (rc == FEM_OK) rc = fwd_impl(q, k, v, beta_max, out, lse, B, H, T, d, causal, p, &ga, ds, s);
@@ -575,6 +589,36 @@ int fem_set_kernel_events(void *start, void *stop) {
     t_ev_start = t_ev_stop = nullptr;
   }
   return FEM_OK;
+}
+
+int fem_attn_fwd(const void *q, const void *k, const void *v, float *out, float *lse, int B, int H, int T, int d,
+                 int causal, void *stream) {
+  int rc = check_common(q, k, v, out, out, lse, B, H, T, d, causal);  // out stands in for beta (unused)
+  if (rc != FEM_OK) return rc;
+  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
+  DeviceState *ds = nullptr;
+  if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  const int BH = B * H;
+  CUtensorMap tq, tk, tv;
+  if ((rc = make_map(&tq, q, BH, T, d)) != FEM_OK) return rc;
+  if ((rc = make_map(&tk, k, BH, T, d)) != FEM_OK) return rc;
+  if ((rc = make_map(&tv, v, BH, T, d)) != FEM_OK) return rc;
+  const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
+  t_ev_start = t_ev_stop = nullptr;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = ev0 ? cudaEventRecord(ev0, s) : cudaSuccess;
+  if (e == cudaSuccess) e = launch_attn(d, tq, tk, tv, out, lse, BH, H, T, causal, ds->err, s);
+  if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
+  return map_cuda(e);
+}
+
+int fem_probe_wait_timeout(unsigned limit_us, void *stream) {
+  if (limit_us == 0 || limit_us > 1000000u) return FEM_ERR_INVALID_ARG;
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  wait_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(ds->err, 1000ull * limit_us);
+  return map_cuda(cudaGetLastError());
 }
 
 int fem_check_device_error(void *stream) {

@@ -71,6 +71,7 @@ constexpr int kFixChunk = 8;  // fix-up entries per chunk: rows scored together,
 constexpr unsigned kErrWaitTma = 1u;
 constexpr unsigned kErrWaitMma = 2u;
 constexpr unsigned kErrTmemAlloc = 4u;
+constexpr unsigned kErrWaitProbe = 8u;  // the diagnostic wait probe gave up (fem_probe_wait_timeout)
 
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // 1 s per wait
 
@@ -181,18 +182,24 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
 
 
 // Waits for the phase with the given parity to complete.  Gives up after
-// kWaitLimitNs, records `code` in the error word and returns false.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned *err, unsigned code) {
+// limit_ns, records `code` in the error word and returns false.
+__device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, unsigned *err, unsigned code,
+                                              unsigned long long limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_timer_ns();
   while (true) {
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
+    if (global_timer_ns() - t0 > limit_ns) {
       atomicOr(err, code);
       return false;
     }
   }
+}
+
+// mbar_wait_for with the kernels' limit, kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned *err, unsigned code) {
+  return mbar_wait_for(bar, parity, err, code, kWaitLimitNs);
 }
 
 // ---------------------------------------------------------------------------

@@ -70,6 +70,11 @@ cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const
                       const CUtensorMap *te0, float *out, const float *beta, const BankWorkspace &w, float *lse,
                       int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream);
 
+// The attention-mode comparator on the same kernel: o = softmax(q k^T / sqrt(d)) v
+// with bf16 P and V on the tensor cores (tv maps V like the bank).
+cudaError_t launch_attn(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, float *out,
+                        float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream);
+
 // Largest sequence length launch_tc takes (its shared-memory bitmap of moved key tiles).
 constexpr int kMaxSeqLen = 8192 * kBlockK;
 

@@ -146,7 +146,15 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t *>(&v);
 }
 
-template <int D, bool GATED>
+__device__ __forceinline__ uint32_t pack_bf162(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// ATTN: the attention-mode comparator -- plain softmax attention
+// o = sum_i p_t(i) v_i, the same kernel with V itself (bf16) as the second
+// operand and P in bf16: no value bank, no shifts, no guard.
+template <int D, bool GATED, bool ATTN = false>
 __global__ void __launch_bounds__(384, 1)
     fem_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_e0,
@@ -184,7 +192,7 @@ __global__ void __launch_bounds__(384, 1)
   // causal with earlier key tiles: the diagonal tile's P E (of the beta bank)
   // goes to the score buffer no other tile uses from then on, so acc keeps
   // the state before it
-  const bool split = causal && nk > 1;
+  const bool split = !ATTN && causal && nk > 1;
 
   // K tile kt into K stage kt % kStagesK, with its side data into side slot
   // kt % 8.  Side slot kt % 8 was last read by the correction of tile kt - 8,
@@ -197,6 +205,7 @@ __global__ void __launch_bounds__(384, 1)
       tma_load_3d(sbase + Lay::kK + st * Lay::kTile + b * 16384, &tmap_k, FEM_BAR(kBarKFull + st), b * 64,
                   kt * kBlockK, bh);
     const size_t row = static_cast<size_t>(bh) * n_kt_all + kt;
+    if (ATTN) return;  // no bank, no side data
     const uint32_t slot = sbase + Lay::kSide + ss * Lay::kSideStride;
     mbar_arrive_expect_tx(FEM_BAR(kBarSide + ss), Lay::kSideMask + 16);
     bulk_load(slot, w.rfac + row * D, D * 4, FEM_BAR(kBarSide + ss));
@@ -251,6 +260,10 @@ __global__ void __launch_bounds__(384, 1)
     for (int e = 0; e < min(ne, kPreE); ++e) load_e(e);
   }
   for (int j = tid; j < D; j += 384) {
+    if (ATTN) {  // o = acc / L: the linear form at beta = 0 around 0
+      c_coef[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+      continue;
+    }
     const ChanInfo ci = w.chan[bh * D + j];
     const float bj = beta[h * D + j];
     const bool lin = ci.linear != 0.f;
@@ -267,7 +280,7 @@ __global__ void __launch_bounds__(384, 1)
   for (int base = 0; base < nk; base += 384) {
     const int t = base + tid;
     bool moved = false;
-    if (t < nk) {
+    if (!ATTN && t < nk) {
       const uint4 m = reinterpret_cast<const uint4 *>(w.colmask)[static_cast<size_t>(bh) * n_kt_all + t];
       moved = (m.x | m.y | m.z | m.w) != 0u;
     }
@@ -339,7 +352,7 @@ __global__ void __launch_bounds__(384, 1)
   } else if (warp == 2) {
     // ---------------------------------------------------------------- PV issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_pv = idesc_f16(128, D, false, true);
+      constexpr uint32_t idesc_pv = idesc_f16(128, D, ATTN, true);  // fp16 P and bank, or bf16 P and V
       const uint32_t tAcc = tmem + Lay::kAccCol;
       bool ok = true;
       for (int kt = 0; ok && kt < nk; ++kt) {
@@ -448,7 +461,7 @@ __global__ void __launch_bounds__(384, 1)
             const float2 x = __ffma2_rn(make_float2(s[c * 32 + 2 * i], s[c * 32 + 2 * i + 1]), scale2, negm2);
             const float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
             ls[i & 3] = __fadd2_rn(ls[i & 3], e);
-            p[i] = pack_half2(e.x, e.y);
+            p[i] = ATTN ? pack_bf162(e.x, e.y) : pack_half2(e.x, e.y);
           }
           tmem_st16(tS + c * 16, p);
         }
@@ -467,7 +480,7 @@ __global__ void __launch_bounds__(384, 1)
       // in the units of the current shift (and the mean bank's, GATED), and
       // the same before the diagonal tile
       float ecol = 0.f, ecol_pre = 0.f, ecol0 = 0.f;
-      const float beta_r = r < D ? beta[h * D + r] : 0.f;  // for the guard's coefficients after the loop
+      const float beta_r = (!ATTN && r < D) ? beta[h * D + r] : 0.f;  // for the guard's coefficients after the loop
       for (int kt = 0; kt < nk; ++kt) {
         const int b = kt % kBufS;
         ok = __all_sync(0xffffffffu,
@@ -482,10 +495,12 @@ __global__ void __launch_bounds__(384, 1)
         // ahead with K
         const float *rf =
             reinterpret_cast<const float *>(smem + Lay::kSide + (kt % Lay::kSideStages) * Lay::kSideStride);
-        ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSide + kt % Lay::kSideStages),
-                                                   (kt / Lay::kSideStages) & 1, err, kErrWaitTma, abort_flag));
+        if (!ATTN) {
+          ok = __all_sync(0xffffffffu, wait_or_abort(FEM_BAR(kBarSide + kt % Lay::kSideStages),
+                                                     (kt / Lay::kSideStages) & 1, err, kErrWaitTma, abort_flag));
+        }
         if (!ok) break;
-        if (r < D) {
+        if (!ATTN && r < D) {
           if (last_split) ecol_pre = ecol;
           ecol = fmaf(ecol, rf[r], rf[D + r]);
           if (GATED) ecol0 += rf[2 * D + r];
@@ -569,7 +584,7 @@ __global__ void __launch_bounds__(384, 1)
       //   X a_pre + Zp < Y L_pre   (state before the diagonal tile)
       // with X = tau beta, Z = -2^-25 Ecol, Zp = -2^-25 Ecol_pre and Y = 2^-25
       // (shifted bank) or -tau (linear bank); see kGuardTau
-      if (r < D) {
+      if (!ATTN && r < D) {
         const bool lin = c_coef[r].w == 0.f;
         const float4 g = make_float4(kGuardTau * beta_r, -kGuardUlp * ecol, lin ? -kGuardTau : kGuardUlp, -kGuardUlp * ecol_pre);
         s_gco[r] = g;
@@ -654,8 +669,9 @@ __global__ void __launch_bounds__(384, 1)
             const float4 p = ab[2 * i4], q = ab[2 * i4 + 1];  // {A, B} of four channels
             const float a0 = __uint_as_float(vd[4 * i4]) * invL, a1 = __uint_as_float(vd[4 * i4 + 1]) * invL,
                         a2 = __uint_as_float(vd[4 * i4 + 2]) * invL, a3 = __uint_as_float(vd[4 * i4 + 3]) * invL;
-            cand |= (a0 < fmaf(p.y, invL, p.x)) | (a1 < fmaf(p.w, invL, p.z)) | (a2 < fmaf(q.y, invL, q.x)) |
-                    (a3 < fmaf(q.w, invL, q.z));
+            if (!ATTN)
+              cand |= (a0 < fmaf(p.y, invL, p.x)) | (a1 < fmaf(p.w, invL, p.z)) | (a2 < fmaf(q.y, invL, q.x)) |
+                      (a3 < fmaf(q.w, invL, q.z));
             *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(a0, a1, a2, a3);
           }
         }
@@ -872,7 +888,7 @@ __global__ void __launch_bounds__(384, 1)
 #undef FEM_BAR
 }
 
-template <int D, bool GATED>
+template <int D, bool GATED, bool ATTN = false>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
                                const CUtensorMap &te0, float *out, const float *beta, const BankWorkspace &w,
                                float *lse, int BH, int H, int T, int causal, const TcGate &gate, unsigned *err,
@@ -881,10 +897,12 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   if (n_qt > Lay::kMaxKeyTiles || BH > 65535) return cudaErrorInvalidValue;
   const uint32_t smem = Lay::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(fem_tc_kernel<D, GATED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e =
+      cudaFuncSetAttribute(fem_tc_kernel<D, GATED, ATTN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const dim3 grid(n_qt, BH);
-  fem_tc_kernel<D, GATED><<<grid, 384, smem, stream>>>(tq, tk, te, te0, out, beta, w, lse, H, T, causal, gate, err);
+  fem_tc_kernel<D, GATED, ATTN>
+      <<<grid, 384, smem, stream>>>(tq, tk, te, te0, out, beta, w, lse, H, T, causal, gate, err);
   return cudaGetLastError();
 }
 
@@ -901,6 +919,17 @@ cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const
   }
   if (d == 64) return launch_tc_d<64, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream);
   if (d == 128) return launch_tc_d<128, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_attn(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, float *out,
+                        float *lse, int BH, int H, int T, int causal, unsigned *err, cudaStream_t stream) {
+  const TcGate none = {nullptr, nullptr, nullptr, nullptr, nullptr};
+  const BankWorkspace w = {};
+  if (d == 64)
+    return launch_tc_d<64, false, true>(tq, tk, tv, tv, out, nullptr, w, lse, BH, H, T, causal, none, err, stream);
+  if (d == 128)
+    return launch_tc_d<128, false, true>(tq, tk, tv, tv, out, nullptr, w, lse, BH, H, T, causal, none, err, stream);
   return cudaErrorInvalidValue;
 }
 

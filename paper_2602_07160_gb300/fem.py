@@ -23,7 +23,8 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
-           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd", "fem_tdc_conv", "fem_bwd_f32"]
+           "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd", "fem_tdc_conv", "fem_bwd_f32",
+           "fem_probe_wait_timeout", "fem_attn_fwd"]
 
 
 class FemError(RuntimeError):
@@ -67,6 +68,10 @@ def load(path: str | None = None):
         lib.fem_fwd_workspace_bytes.argtypes = [i, i, i, i, i]
         lib.fem_fwd_workspace_bytes.restype = sz
         lib.fem_check_device_error.argtypes = [vp]
+        lib.fem_attn_fwd.argtypes = [vp, vp, vp, vp, vp, i, i, i, i, i, vp]
+        lib.fem_attn_fwd.restype = i
+        lib.fem_probe_wait_timeout.argtypes = [ctypes.c_uint, vp]
+        lib.fem_probe_wait_timeout.restype = i
         lib.fem_last_fixup_rows.argtypes = [vp]
         lib.fem_set_kernel_events.argtypes = [vp, vp]
         lib.fem_set_kernel_events.restype = i
@@ -129,6 +134,19 @@ def fem_fwd(q, k, v, beta, causal: bool = True, out=None, lse=None, stream=None)
                         B, H, T, d, int(bool(causal)), _stream(stream, q.device))
     if rc != 0:
         raise FemError("fem_fwd", rc)
+    return out, (None if lse is False else lse)
+
+
+def fem_attn_fwd(q, k, v, causal: bool = True, out=None, lse=None, stream=None):
+    """Plain softmax attention on the same tensor-core kernel (the comparator; bf16 CUDA
+    tensors).  Returns (out, lse)."""
+    beta = torch.zeros((q.shape[1], q.shape[3]), dtype=torch.float32, device=q.device)  # shape check only
+    B, H, T, d = _check_qkvb(q, k, v, beta, torch.bfloat16, "cuda")
+    out, lse = _outputs(q, out, lse, q.device)
+    rc = load().fem_attn_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(out), None if lse is False else _ptr(lse),
+                             B, H, T, d, int(bool(causal)), _stream(stream, q.device))
+    if rc != 0:
+        raise FemError("fem_attn_fwd", rc)
     return out, (None if lse is False else lse)
 
 
@@ -290,6 +308,15 @@ def fem_fwd_noalloc(q, k, v, beta, causal: bool = True, out=None, lse=None, stre
     if rc != 0:
         raise FemError("fem_fwd_noalloc", rc)
     return out, (None if lse is False else lse)
+
+
+def probe_wait_timeout(limit_us: int, stream=None, device=None):
+    """Enqueue the library's wait probe: a bounded wait on an mbarrier nothing completes,
+    which gives up after limit_us microseconds and records a timeout in the error word."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    rc = load().fem_probe_wait_timeout(int(limit_us), _stream(stream, dev))
+    if rc != 0:
+        raise FemError("fem_probe_wait_timeout", rc)
 
 
 def check_device_error(stream=None, device=None):

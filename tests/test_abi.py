@@ -156,3 +156,9 @@ def test_backward_argument_errors_are_synchronous(lib):
     assert call(dq=0) == 1
     assert call(dq=8) == 1
     assert call(d=300) == 2
+
+
+def test_wait_probe_argument_errors_are_synchronous(lib):
+    """fem_probe_wait_timeout rejects a limit of 0 or above one second before any CUDA call."""
+    assert lib.fem_probe_wait_timeout(0, None) == 1
+    assert lib.fem_probe_wait_timeout(1_000_001, None) == 1

@@ -105,3 +105,46 @@ def test_gated_read_fixup_rows(d):
     scale = max(1.0, float(gate.abs().max()))
     assert err.max() <= BF16_MAX * scale and err.mean() <= BF16_MEAN, (err.max(), err.mean())
     assert np.abs(lse.cpu().double().numpy() - ref_lse).max() <= 2e-3
+
+
+def test_gated_read_headline_shape_sampled():
+    """The one-pass gated kernel (its own TMEM and shared-memory layout at d = 128: two score
+    buffers, two K stages, two accumulators) at B4 H16 T8192 causal with the paper's gate
+    parameterisation, checked on sampled rows that include the first and last key tiles."""
+    w = W.WORKLOADS["lm_causal_d128"]
+    q, k, v, bmax = W.make_inputs(w)
+    lam, gate = _gates(17, q.shape)
+    dev = torch.device("cuda", 0)
+    out, lse = fem.fem_fwd_gated(*(x.to(dev) for x in (q, k, v, bmax, lam, gate)), causal=True)
+    fem.check_device_error()
+    r = np.random.default_rng(4)
+    rows = np.unique(np.concatenate([np.arange(384), (w.B * w.H - 1) * w.T + np.arange(w.T - 128, w.T),
+                                     r.choice(w.B * w.H * w.T, 1200, replace=False)]))
+    ref, ref_lse = oracle.gated_read_rows(q, k, v, bmax, lam, gate, True, rows)
+    got = out.reshape(-1, w.d)[torch.from_numpy(rows).to(dev)].cpu().double().numpy()
+    assert np.isfinite(got).all()
+    err = np.abs(got - ref)
+    scale = max(1.0, float(gate.abs().max()))
+    assert err.max() <= BF16_MAX * scale and err.mean() <= BF16_MEAN, (err.max(), err.mean())
+    assert np.abs(lse.reshape(-1)[torch.from_numpy(rows).to(dev)].cpu().double().numpy() - ref_lse).max() <= 2e-3
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_gated_read_peaked_prior(d):
+    """Q and K scaled by 2 (score spread of about 30 nats) with beta_max up to 1e3: the gated
+    kernel's guard routes the entries its 16-bit operands cannot hold to the exact fix-up."""
+    q, k, v, _ = W.make_custom(1, 2, 400, d, seed=31)
+    q = (q.float() * 2).to(torch.bfloat16)
+    k = (k.float() * 2).to(torch.bfloat16)
+    bmax = W.beta_grid(2, d, [0.05, 1.0, 5.0, 20.0, 100.0, 1e3])
+    lam, gate = _gates(5, q.shape)
+    dev = torch.device("cuda", 0)
+    for causal in (True, False):
+        out, _ = fem.fem_fwd_gated(*(x.to(dev) for x in (q, k, v, bmax, lam, gate)), causal=causal)
+        fem.check_device_error()
+        ref, _ = oracle.gated_read(q, k, v, bmax, lam, gate, causal)
+        o = out.cpu().double().numpy()
+        assert np.isfinite(o).all()
+        err = np.abs(o - ref)
+        scale = max(1.0, float(gate.abs().max()))
+        assert err.max() <= BF16_MAX * scale and err.mean() <= BF16_MEAN, (causal, err.max(), err.mean())
