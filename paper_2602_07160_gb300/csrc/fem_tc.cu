@@ -77,14 +77,14 @@ struct TcLayout {
   static constexpr uint32_t kTmemSlot = kBar + kNumBars * 8;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kChan = kBar + 512;               // per-channel epilogue coefficients
-  static constexpr uint32_t kMoveBits = kChan + 4 * D * 4 + (GATED ? 4 * D : 0);  // 1 bit per key tile: a shift moved
+  static constexpr uint32_t kMoveBits = kChan + 4 * D * 4 + (GATED ? 4 * D : 0);
   static constexpr int kMaxKeyTiles = kMaxSeqLen / kBlockK;  // T <= 1M keys
   // side ring: per key tile its rescale factors exp(beta_j (c_old - c_new)) [D],
   // the bank's column sums [D] (GATED: also the mean bank's [D]) and the
   // moved-channel mask [4], loaded with the K tile, kSideStages tiles deep
   static constexpr int kSideStages = 8;
   static constexpr int kSideArrays = GATED ? 3 : 2;
-  static constexpr uint32_t kSide = kMoveBits + kMaxKeyTiles / 8;
+  static constexpr uint32_t kSide = kMoveBits;
   static constexpr uint32_t kSideMask = kSideArrays * D * 4;  // offset of the mask in a slot
   static constexpr uint32_t kSideStride = kSideMask + 128;
   static constexpr uint32_t kAlpha = kSide + kSideStages * kSideStride;  // alpha per row, per score buffer
@@ -170,7 +170,6 @@ __global__ void __launch_bounds__(384, 1)
   // with c the last shift; linear bank {beta, c, ln2/beta (0 at beta = 0), 0}
   // with c the anchor
   float4 *c_coef = reinterpret_cast<float4 *>(smem + Lay::kChan);
-  unsigned *move_bits = reinterpret_cast<unsigned *>(smem + Lay::kMoveBits);
   const uint32_t bars = sbase + Lay::kBar;
 #define FEM_BAR(i) (bars + 8u * static_cast<uint32_t>(i))
 
@@ -258,34 +257,6 @@ __global__ void __launch_bounds__(384, 1)
       tma_load_3d(sbase + Lay::kQ + b * 16384, &tmap_q, FEM_BAR(kBarQ), b * 64, qt * kBlockQ, bh);
     for (int kt = 0; kt < min(nk, kPreK); ++kt) load_k(kt);
     for (int e = 0; e < min(ne, kPreE); ++e) load_e(e);
-  }
-  for (int j = tid; j < D; j += 384) {
-    if (ATTN) {  // o = acc / L: the linear form at beta = 0 around 0
-      c_coef[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-      continue;
-    }
-    const ChanInfo ci = w.chan[bh * D + j];
-    const float bj = beta[h * D + j];
-    const bool lin = ci.linear != 0.f;
-    if (lin) {
-      c_coef[j] = make_float4(bj, ci.c_lin, bj != 0.f ? kLn2 / bj : 0.f, 0.f);
-    } else {
-      const float c = w.shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + j];
-      c_coef[j] = make_float4(0.f, c - kBankOffset / bj, kLn2 / bj, 1.f);
-    }
-    // the mean's anchor: its bank holds v - c, so mu = c + acc/L
-    if (GATED) reinterpret_cast<float *>(c_coef + D)[j] = gate.chan0[bh * D + j].c_lin;
-  }
-  // one bit per key tile: set when some channel's shift moved there
-  for (int base = 0; base < nk; base += 384) {
-    const int t = base + tid;
-    bool moved = false;
-    if (!ATTN && t < nk) {
-      const uint4 m = reinterpret_cast<const uint4 *>(w.colmask)[static_cast<size_t>(bh) * n_kt_all + t];
-      moved = (m.x | m.y | m.z | m.w) != 0u;
-    }
-    const unsigned bits = __ballot_sync(0xffffffffu, moved);
-    if (lane == 0) move_bits[(base >> 5) + warp] = bits;
   }
   if (tid == 0) {
     reinterpret_cast<float *>(smem + Lay::kMisc)[4] = 0.f;        // the mean bank's largest guard bound
@@ -480,14 +451,24 @@ __global__ void __launch_bounds__(384, 1)
       // in the units of the current shift (and the mean bank's, GATED), and
       // the same before the diagonal tile
       float ecol = 0.f, ecol_pre = 0.f, ecol0 = 0.f;
-      const float beta_r = (!ATTN && r < D) ? beta[h * D + r] : 0.f;  // for the guard's coefficients after the loop
+      // channel r's epilogue coefficients, loaded now and stored after the loop
+      // (the epilogue is the first reader): the bank's mode and anchor, the last
+      // shift, beta and, GATED, the mean's anchor
+      ChanInfo ci_r = {0.f, 1.f};
+      float beta_r = 0.f, shift_r = 0.f, c0_r = 0.f;
+      if (!ATTN && r < D) {
+        ci_r = w.chan[bh * D + r];
+        beta_r = beta[h * D + r];
+        shift_r = w.shift[(static_cast<size_t>(bh) * n_kt_all + nk - 1) * D + r];
+        if (GATED) c0_r = gate.chan0[bh * D + r].c_lin;
+      }
       for (int kt = 0; kt < nk; ++kt) {
         const int b = kt % kBufS;
         ok = __all_sync(0xffffffffu,
                         wait_or_abort(FEM_BAR(kBarAlpha + b), (kt / kBufS) & 1, err, kErrWaitMma, abort_flag));
         if (!ok) break;
         const float alpha = s_alpha[b * 128 + r];
-        const bool colmv = (move_bits[kt >> 5] >> (kt & 31)) & 1u;  // some channel's shift moved
+        // (colmv, some channel's shift moved at this tile, comes with the side data below)
         const bool rowmv = __any_sync(0xffffffffu, alpha != 1.f);
         const bool last_split = split && kt == nk - 1;  // acc keeps its state; the epilogue rescales
         // this tile's rescale factors exp(beta_j (c_old - c_new)), 1 for unmoved
@@ -500,6 +481,11 @@ __global__ void __launch_bounds__(384, 1)
                                                      (kt / Lay::kSideStages) & 1, err, kErrWaitTma, abort_flag));
         }
         if (!ok) break;
+        bool colmv = false;
+        if (!ATTN) {
+          const uint4 m4 = *reinterpret_cast<const uint4 *>(rf + Lay::kSideMask / 4);
+          colmv = (m4.x | m4.y | m4.z | m4.w) != 0u;
+        }
         if (!ATTN && r < D) {
           if (last_split) ecol_pre = ecol;
           ecol = fmaf(ecol, rf[r], rf[D + r]);
@@ -584,8 +570,19 @@ __global__ void __launch_bounds__(384, 1)
       //   X a_pre + Zp < Y L_pre   (state before the diagonal tile)
       // with X = tau beta, Z = -2^-25 Ecol, Zp = -2^-25 Ecol_pre and Y = 2^-25
       // (shifted bank) or -tau (linear bank); see kGuardTau
+      if (r < D) {
+        if (ATTN) {
+          c_coef[r] = make_float4(0.f, 0.f, 0.f, 0.f);  // o = acc / L: the linear form at beta = 0 around 0
+        } else if (ci_r.linear != 0.f) {
+          c_coef[r] = make_float4(beta_r, ci_r.c_lin, beta_r != 0.f ? kLn2 / beta_r : 0.f, 0.f);
+        } else {
+          c_coef[r] = make_float4(0.f, shift_r - kBankOffset / beta_r, kLn2 / beta_r, 1.f);
+        }
+        // the mean's anchor: its bank holds v - c, so mu = c + acc/L
+        if (GATED) reinterpret_cast<float *>(c_coef + D)[r] = c0_r;
+      }
       if (!ATTN && r < D) {
-        const bool lin = c_coef[r].w == 0.f;
+        const bool lin = ci_r.linear != 0.f;
         const float4 g = make_float4(kGuardTau * beta_r, -kGuardUlp * ecol, lin ? -kGuardTau : kGuardUlp, -kGuardUlp * ecol_pre);
         s_gco[r] = g;
         // the same test on the final state as a < A + B / L: A = Y / X, B = -Z / X for
@@ -640,7 +637,11 @@ __global__ void __launch_bounds__(384, 1)
       }
       // the diagonal tile's factors: alpha of the row, exp(beta (c_old - c_new)) of the channel
       const bool scale_last =
-          split && (__any_sync(0xffffffffu, alpha_last != 1.f) || ((move_bits[(nk - 1) >> 5] >> ((nk - 1) & 31)) & 1u));
+          split && (__any_sync(0xffffffffu, alpha_last != 1.f) ||
+                    (reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->x |
+                     reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->y |
+                     reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->z |
+                     reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->w) != 0u);
       {
         // chunk by chunk: acc (before the diagonal tile when split) plus the
         // diagonal tile's P E, the guard's test, staged
