@@ -95,7 +95,9 @@ struct TcLayout {
   static constexpr uint32_t kFlag = kThr + D * 8;    // per row and 32-channel group: entries the guard rejects
   static constexpr uint32_t kBad = kFlag + 128 * 16;  // per row: restart from the diagonal tile not possible
   static constexpr uint32_t kMisc = kBad + 128 * 4;   // entry counts and bases, guard bounds, row flags
-  static constexpr uint32_t kBytes = kMisc + 128;
+  // 1/L of row 4 k + q at [32 q + k]: the transform's batch of 8 rows in two 16-byte loads
+  static constexpr uint32_t kInvLT = kMisc + 128;
+  static constexpr uint32_t kBytes = kInvLT + 128 * 4;
   static constexpr uint32_t kAlloc = kBytes + 1024;
   static constexpr uint32_t kAccCol = kBufS * 128;
   static constexpr uint32_t kAccB = kAccCol + (GATED ? D : 0);  // the beta (or beta_max) read's accumulator
@@ -262,7 +264,8 @@ __global__ void __launch_bounds__(384, 1)
     reinterpret_cast<float *>(smem + Lay::kMisc)[4] = 0.f;        // the mean bank's largest guard bound
   }
   if (tid < 128) reinterpret_cast<unsigned *>(smem + Lay::kBad)[tid] = 0u;
-  if (tid < 4) reinterpret_cast<unsigned *>(smem + Lay::kMisc)[16 + tid] = 0u;  // rows with listed entries
+  // rows with listed entries [16..19], rows with candidate entries [20..23]
+  if (tid < 8) reinterpret_cast<unsigned *>(smem + Lay::kMisc)[16 + tid] = 0u;
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
@@ -443,6 +446,7 @@ __global__ void __launch_bounds__(384, 1)
         mbar_arrive(FEM_BAR(kBarPFull + b));
       }
       s_invL[r] = 1.f / L_row;
+      reinterpret_cast<float *>(smem + Lay::kInvLT)[(r & 3) * 32 + (r >> 2)] = 1.f / L_row;
       if (ok && lse && t_row < T) lse[static_cast<size_t>(bh) * T + t_row] = (m_row + lg2_approx(L_row)) * kLn2;
     }
     else {
@@ -610,10 +614,10 @@ __global__ void __launch_bounds__(384, 1)
       constexpr int NC = D / 64;             // 32-column chunks of this warpgroup
       constexpr int kBoxB = (kNB - 1) * (D / 32);  // first box of the beta read
       const int c_lo = is_sm ? 0 : NC;
-      const bool row_ok = t_row < T;
       // GATED: the mean bank's guard for the whole row (its bound is per channel;
       // the largest one stands for all)
-      const bool mean_bad = GATED && reinterpret_cast<const float *>(smem + Lay::kMisc)[4] * invL > kGuardTau;
+      const float mean_bound = GATED ? reinterpret_cast<const float *>(smem + Lay::kMisc)[4] : 0.f;
+      const bool mean_bad = GATED && mean_bound * invL > kGuardTau;
       const float2 pre = s_pre[r];  // (m, L) before the last key tile
       const float alpha_last = split ? s_alpha[((nk - 1) % kBufS) * 128 + r] : 1.f;
       const float *rf_last =
@@ -635,111 +639,33 @@ __global__ void __launch_bounds__(384, 1)
                             __uint_as_float(v[c][4 * i4 + 2]) * invL, __uint_as_float(v[c][4 * i4 + 3]) * invL);
         }
       }
-      // the diagonal tile's factors: alpha of the row, exp(beta (c_old - c_new)) of the channel
-      const bool scale_last =
-          split && (__any_sync(0xffffffffu, alpha_last != 1.f) ||
-                    (reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->x |
-                     reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->y |
-                     reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->z |
-                     reinterpret_cast<const uint4 *>(rf_last + Lay::kSideMask / 4)->w) != 0u);
-      {
-        // chunk by chunk: acc (before the diagonal tile when split) plus the
-        // diagonal tile's P E, the guard's test, staged
-        bool cand = false;
+      // chunk by chunk: acc (before the diagonal tile when split) times the
+      // diagonal tile's factors, alpha of the row and exp(beta (c_old - c_new))
+      // of the channel (both exactly 1 unless the row maximum or the channel's
+      // shift moved on it), plus the diagonal tile's P E, over L, staged
 #pragma unroll 1
-        for (int c = c_lo; c < c_lo + NC; ++c) {
-          uint32_t va[32], vd[32];
-          tmem_ld32(tAccB + c * 32, va);
-          if (split) tmem_ld32(tDiagL + c * 32, vd);
+      for (int c = c_lo; c < c_lo + NC; ++c) {
+        uint32_t va[32], vd[32];
+        tmem_ld32(tAccB + c * 32, va);
+        if (split) {
+          tmem_ld32(tDiagL + c * 32, vd);
           tmem_ld_wait();
-          if (!split) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) vd[i] = va[i];
-          } else if (scale_last) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              vd[i] = __float_as_uint(fmaf(__uint_as_float(va[i]), alpha_last * rf_last[c * 32 + i], __uint_as_float(vd[i])));
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) vd[i] = __float_as_uint(__uint_as_float(va[i]) + __uint_as_float(vd[i]));
-          }
-          uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
-          const float4 *ab = reinterpret_cast<const float4 *>(s_ab + c * 32);
-#pragma unroll
-          for (int i4 = 0; i4 < 8; ++i4) {
-            const float4 p = ab[2 * i4], q = ab[2 * i4 + 1];  // {A, B} of four channels
-            const float a0 = __uint_as_float(vd[4 * i4]) * invL, a1 = __uint_as_float(vd[4 * i4 + 1]) * invL,
-                        a2 = __uint_as_float(vd[4 * i4 + 2]) * invL, a3 = __uint_as_float(vd[4 * i4 + 3]) * invL;
-            if (!ATTN)
-              cand |= (a0 < fmaf(p.y, invL, p.x)) | (a1 < fmaf(p.w, invL, p.z)) | (a2 < fmaf(q.y, invL, q.x)) |
-                      (a3 < fmaf(q.w, invL, q.z));
-            *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) = make_float4(a0, a1, a2, a3);
-          }
-        }
-        cand = (cand || mean_bad) && row_ok;
-        if (__any_sync(0xffffffffu, cand)) {
-          // the exact guard on the candidate rows; a rejected entry's accumulator
-          // before the diagonal tile goes out in place of the output (the
-          // fix-up's starting state), and whether that state passes the guard
-          // decides where the fix-up starts
-#pragma unroll 1
-          for (int c = c_lo; c < c_lo + NC; ++c) {
-            uint32_t vp[32];
-            tmem_ld32(tAccB + c * 32, vp);
-            tmem_ld_wait();
-            unsigned fm = 0;
-            if (cand) {
-              uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
-              const float4 *gco = s_gco + c * 32;
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                float *cell = reinterpret_cast<float *>(box + sw128_offset(r, i >> 2)) + (i & 3);
-                const float4 g = gco[i];
-                const float2 t = s_ab[c * 32 + i];
-                if (!(mean_bad || *cell < fmaf(t.y, invL, t.x))) continue;
-                fm |= 1u << i;
-                const float a_pre = split ? __uint_as_float(vp[i]) : 0.f;
-                if (split && fmaf(g.x, a_pre, g.w) < g.z * pre.y) bad = 1;
-                *cell = a_pre;
-              }
-            }
-            s_flag[r * 4 + c] = fm;
-            if (fm) atomicOr(reinterpret_cast<unsigned *>(smem + Lay::kMisc) + 16 + (r >> 5), 1u << (r & 31));
-          }
+          for (int i = 0; i < 32; ++i)
+            vd[i] = __float_as_uint(fmaf(__uint_as_float(va[i]), alpha_last * rf_last[c * 32 + i], __uint_as_float(vd[i])));
         } else {
+          tmem_ld_wait();
 #pragma unroll
-          for (int c = c_lo; c < c_lo + NC; ++c) s_flag[r * 4 + c] = 0u;
+          for (int i = 0; i < 32; ++i) vd[i] = va[i];
         }
-      }
-      if (bad) atomicOr(s_bad + r, 1u);
-      bar_sync(4, 256);
-      // ---- list the rejected rows: one block of entries that restart from the
-      // diagonal tile, one of entries recomputed over every key tile, each padded
-      // to a multiple of kFixChunk rows (rows -1) for the fix-up's chunks.  The slots are
-      // reserved now and written after the transform, which hides the atomic.
-      const unsigned *rowflags = reinterpret_cast<const unsigned *>(smem + Lay::kMisc) + 16;
-      const bool any_listed = (rowflags[0] | rowflags[1] | rowflags[2] | rowflags[3]) != 0u;
-      int base = 0;  // thread 0 of the softmax warpgroup: the first reserved slot
-      if (any_listed && is_sm) {
-        const bool listed = (rowflags[r >> 5] >> (r & 31)) & 1u;
-        const bool diag = listed && split && s_bad[r] == 0u;
-        const unsigned bd = __ballot_sync(0xffffffffu, diag), bf = __ballot_sync(0xffffffffu, listed && !diag);
-        if (lane == 0) {
-          s_misc[8 + (warp & 3)] = __popc(bd);
-          s_misc[12 + (warp & 3)] = __popc(bf);
-        }
-        bar_sync(2, 128);
-        if (r == 0) {
-          int nd = 0, nf = 0;
+        uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            nd += s_misc[8 + q];
-            nf += s_misc[12 + q];
-          }
-          base = atomicAdd(w.fixup_count, pad_chunk(nd) + pad_chunk(nf));
-          atomicAdd(w.fixup_rows, nd + nf);
-        }
+        for (int i4 = 0; i4 < 8; ++i4)
+          *reinterpret_cast<float4 *>(box + sw128_offset(r, i4)) =
+              make_float4(__uint_as_float(vd[4 * i4]) * invL, __uint_as_float(vd[4 * i4 + 1]) * invL,
+                          __uint_as_float(vd[4 * i4 + 2]) * invL, __uint_as_float(vd[4 * i4 + 3]) * invL);
       }
+      bar_sync(4, 256);  // every box is staged
       // Thread r takes column r % 32 of a chunk and rows r / 32 + 4k, so its
       // channel's coefficients stay in registers, each warp access is one
       // 128-byte row of the box, and 8 loads at a time are in flight before the math.
@@ -748,9 +674,9 @@ __global__ void __launch_bounds__(384, 1)
       //                 or, for |x| < 2^-6 (also beta = 0), as c + a times the
       //                 series of log1p(x)/x
       // GATED: mu = c_mean + a_mean, F the beta_max read as above, and
-      // o = g (mu + lambda (F - mu)).  A listed entry gets the staged value
-      // itself (the accumulator before its diagonal tile) and, GATED, its mu in
-      // the gate's side buffer.
+      // o = g (mu + lambda (F - mu)).  The underflow guard's test a < A + B / L
+      // runs here too, thread per channel with A, B in registers; rows with a
+      // candidate entry are marked for the exact test after the transform.
       const int col = r & 31, row0 = r >> 5;
       const int rows_left = T - qt * kBlockQ;
       const size_t tile_off = (static_cast<size_t>(bh) * T + static_cast<size_t>(qt) * kBlockQ) * D + col;
@@ -759,6 +685,7 @@ __global__ void __launch_bounds__(384, 1)
       for (int c = c_lo; c < c_lo + NC; ++c) {
         const float4 cf = c_coef[c * 32 + col];
         const float c_mean = GATED ? reinterpret_cast<const float *>(c_coef + D)[c * 32 + col] : 0.f;
+        const float2 thr = ATTN ? make_float2(0.f, 0.f) : s_ab[c * 32 + col];
         const bool lin = cf.w == 0.f;
         // pairs of rows go through the packed fp32x2 pipe; the lg2 argument is
         // a (shifted) or 1 + beta a (linear)
@@ -784,8 +711,21 @@ __global__ void __launch_bounds__(384, 1)
               gv[k] = __ldcs(gate.g + oi);
             }
           }
-          // rows of this batch with listed entries (row0 + 4 (k0 + k) lies in word k0 / 8, bit row0 + 4 k)
-          const unsigned rw = any_listed ? reinterpret_cast<const unsigned *>(smem + Lay::kMisc)[16 + (k0 >> 3)] : 0u;
+          // the guard's quick test on the 8 rows (row0 + 4 (k0 + k) lies in word k0 / 8, bit row0 + 4 k)
+          if (!ATTN) {
+            const float4 il0 = *reinterpret_cast<const float4 *>(smem + Lay::kInvLT + (row0 * 32 + k0) * 4);
+            const float4 il1 = *reinterpret_cast<const float4 *>(smem + Lay::kInvLT + (row0 * 32 + k0 + 4) * 4);
+            const float il[8] = {il0.x, il0.y, il0.z, il0.w, il1.x, il1.y, il1.z, il1.w};
+            unsigned cm = 0;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              bool cnd = a[k] < fmaf(thr.y, il[k], thr.x);
+              if (GATED) cnd = cnd || mean_bound * il[k] > kGuardTau;
+              cm |= (cnd && row0 + 4 * (k0 + k) < rows_left) ? 1u << (row0 + 4 * k) : 0u;
+            }
+            cm = __reduce_or_sync(0xffffffffu, cm);
+            if (cm && lane == 0) atomicOr(reinterpret_cast<unsigned *>(smem + Lay::kMisc) + 20 + (k0 >> 3), cm);
+          }
           float o[8];
 #pragma unroll
           for (int k = 0; k < 8; k += 2) {
@@ -804,21 +744,9 @@ __global__ void __launch_bounds__(384, 1)
           if (GATED) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-              const int row = row0 + 4 * (k0 + k);
               const float mu =
                   c_mean + *reinterpret_cast<const float *>(box_m + sw128_offset(row0 + 4 * (k0 + k), col >> 2));
-              if (((rw >> (row0 + 4 * k)) & 1u) && ((s_flag[row * 4 + c] >> col) & 1u)) {
-                o[k] = a[k];
-                if (row < rows_left) gate.mu_side[tile_off + static_cast<size_t>(row) * D + c * 32] = mu;
-              } else {
-                o[k] = gv[k] * fmaf(lamv[k], o[k] - mu, mu);
-              }
-            }
-          } else if (rw) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const int row = row0 + 4 * (k0 + k);
-              if (((rw >> (row0 + 4 * k)) & 1u) && ((s_flag[row * 4 + c] >> col) & 1u)) o[k] = a[k];
+              o[k] = gv[k] * fmaf(lamv[k], o[k] - mu, mu);
             }
           }
 #pragma unroll
@@ -828,7 +756,78 @@ __global__ void __launch_bounds__(384, 1)
           }
         }
       }
-      // ---- the listed rows' entries, in the slots reserved before the transform
+      // ---- the exact guard on the marked rows, row r by thread r: a rejected
+      // entry's accumulator before the diagonal tile replaces its output (the
+      // fix-up's starting state; GATED: its mu goes to the gate's side buffer),
+      // and whether that state passes the guard too decides where the fix-up starts
+      bar_sync(4, 256);  // the transform's stores and marks are complete
+      const unsigned *rowcand = reinterpret_cast<const unsigned *>(smem + Lay::kMisc) + 20;
+      if ((rowcand[0] | rowcand[1] | rowcand[2] | rowcand[3]) != 0u) {
+        const bool cand = (rowcand[r >> 5] >> (r & 31)) & 1u;
+        if (__any_sync(0xffffffffu, cand)) {
+#pragma unroll 1
+          for (int c = c_lo; c < c_lo + NC; ++c) {
+            uint32_t vp[32];
+            tmem_ld32(tAccB + c * 32, vp);
+            tmem_ld_wait();
+            unsigned fm = 0;
+            if (cand) {
+              const uint8_t *box = smem + Lay::kK + (kBoxB + c) * 16384;
+              const float4 *gco = s_gco + c * 32;
+              const size_t orow = (static_cast<size_t>(bh) * T + t_row) * D + c * 32;
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const float cell = *(reinterpret_cast<const float *>(box + sw128_offset(r, i >> 2)) + (i & 3));
+                const float4 g = gco[i];
+                const float2 t = s_ab[c * 32 + i];
+                if (!(mean_bad || cell < fmaf(t.y, invL, t.x))) continue;
+                fm |= 1u << i;
+                const float a_pre = split ? __uint_as_float(vp[i]) : 0.f;
+                if (split && fmaf(g.x, a_pre, g.w) < g.z * pre.y) bad = 1;
+                out[orow + i] = a_pre;
+                if (GATED)
+                  gate.mu_side[orow + i] =
+                      reinterpret_cast<const float *>(c_coef + D)[c * 32 + i] +
+                      *(reinterpret_cast<const float *>(smem + Lay::kK + c * 16384 + sw128_offset(r, i >> 2)) + (i & 3));
+              }
+            }
+            s_flag[r * 4 + c] = fm;
+            if (fm) atomicOr(reinterpret_cast<unsigned *>(smem + Lay::kMisc) + 16 + (r >> 5), 1u << (r & 31));
+          }
+        } else {
+#pragma unroll
+          for (int c = c_lo; c < c_lo + NC; ++c) s_flag[r * 4 + c] = 0u;
+        }
+        if (bad) atomicOr(s_bad + r, 1u);
+        bar_sync(4, 256);
+      }
+      // ---- list the rejected rows: one block of entries that restart from the
+      // diagonal tile, one of entries recomputed over every key tile, each padded
+      // to a multiple of kFixChunk rows (rows -1) for the fix-up's chunks
+      const unsigned *rowflags = reinterpret_cast<const unsigned *>(smem + Lay::kMisc) + 16;
+      const bool any_listed = (rowflags[0] | rowflags[1] | rowflags[2] | rowflags[3]) != 0u;
+      int base = 0;  // thread 0 of the softmax warpgroup: the first reserved slot
+      if (any_listed && is_sm) {
+        const bool listed = (rowflags[r >> 5] >> (r & 31)) & 1u;
+        const bool diag = listed && split && s_bad[r] == 0u;
+        const unsigned bd = __ballot_sync(0xffffffffu, diag), bf = __ballot_sync(0xffffffffu, listed && !diag);
+        if (lane == 0) {
+          s_misc[8 + (warp & 3)] = __popc(bd);
+          s_misc[12 + (warp & 3)] = __popc(bf);
+        }
+        bar_sync(2, 128);
+        if (r == 0) {
+          int nd = 0, nf = 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            nd += s_misc[8 + q];
+            nf += s_misc[12 + q];
+          }
+          base = atomicAdd(w.fixup_count, pad_chunk(nd) + pad_chunk(nf));
+          atomicAdd(w.fixup_rows, nd + nf);
+        }
+      }
+      // ---- the listed rows' entries, in the reserved slots
       if (any_listed && is_sm) {
         if (r == 0) s_misc[0] = base;
         bar_sync(2, 128);
