@@ -716,15 +716,26 @@ __global__ void __launch_bounds__(384, 1)
             const float4 il0 = *reinterpret_cast<const float4 *>(smem + Lay::kInvLT + (row0 * 32 + k0) * 4);
             const float4 il1 = *reinterpret_cast<const float4 *>(smem + Lay::kInvLT + (row0 * 32 + k0 + 4) * 4);
             const float il[8] = {il0.x, il0.y, il0.z, il0.w, il1.x, il1.y, il1.z, il1.w};
-            unsigned cm = 0;
+            // two rows per packed fma; the rows' own marks only when some entry of the batch is a candidate
+            bool anyc = false;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              bool cnd = a[k] < fmaf(thr.y, il[k], thr.x);
-              if (GATED) cnd = cnd || mean_bound * il[k] > kGuardTau;
-              cm |= (cnd && row0 + 4 * (k0 + k) < rows_left) ? 1u << (row0 + 4 * k) : 0u;
+            for (int k = 0; k < 8; k += 2) {
+              const float2 t2 = __ffma2_rn(make_float2(thr.y, thr.y), make_float2(il[k], il[k + 1]),
+                                           make_float2(thr.x, thr.x));
+              anyc = anyc || a[k] < t2.x || a[k + 1] < t2.y;
+              if (GATED) anyc = anyc || mean_bound * fmaxf(il[k], il[k + 1]) > kGuardTau;
             }
-            cm = __reduce_or_sync(0xffffffffu, cm);
-            if (cm && lane == 0) atomicOr(reinterpret_cast<unsigned *>(smem + Lay::kMisc) + 20 + (k0 >> 3), cm);
+            if (__any_sync(0xffffffffu, anyc)) {
+              unsigned cm = 0;
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                bool cnd = a[k] < fmaf(thr.y, il[k], thr.x);
+                if (GATED) cnd = cnd || mean_bound * il[k] > kGuardTau;
+                cm |= (cnd && row0 + 4 * (k0 + k) < rows_left) ? 1u << (row0 + 4 * k) : 0u;
+              }
+              cm = __reduce_or_sync(0xffffffffu, cm);
+              if (cm && lane == 0) atomicOr(reinterpret_cast<unsigned *>(smem + Lay::kMisc) + 20 + (k0 >> 3), cm);
+            }
           }
           float o[8];
 #pragma unroll
