@@ -86,6 +86,18 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
     const int bh = g / n_kt, kt = g % n_kt, rows = min(kBlockK, T - kt * kBlockK);
     if (!mbar_wait(smem_u32(&s_full[st]), (i / kStages) & 1, err, kErrWaitTma)) return;
     const uint8_t *tile = ring + st * M::kTileBytes;
+    // the thread's rows into registers, then the slot goes back to the copy engine
+    // before the reductions (rows past T are not read)
+    uint4 rawv[M::RPG];
+#pragma unroll
+    for (int r = 0; r < M::RPG; ++r) {
+      const int row = rg * M::RPG + r;
+      rawv[r] = row < rows ? *reinterpret_cast<const uint4 *>(tile + (row * D + cc * 8) * 2) : make_uint4(0u, 0u, 0u, 0u);
+    }
+    __syncthreads();  // every read of the slot is done
+    if (tid == 0 && i + kStages < my_n)
+      stats_issue<D>(v, T, n_kt, blockIdx.x + (i + kStages) * gridDim.x, smem_u32(ring + st * M::kTileBytes),
+                     smem_u32(&s_full[st]));
     float mx[8], mn[8], sm[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
@@ -97,7 +109,7 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
     for (int r = 0; r < M::RPG; ++r) {
       const int row = rg * M::RPG + r;
       if (row < rows) {
-        const uint4 raw = *reinterpret_cast<const uint4 *>(tile + (row * D + cc * 8) * 2);
+        const uint4 raw = rawv[r];
         const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
@@ -129,10 +141,7 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
         s_part[buf][2][warp][cc * 8 + u] = sm[u];
       }
     }
-    __syncthreads();  // every read of the slot and every partial of this tile are done
-    if (tid == 0 && i + kStages < my_n)
-      stats_issue<D>(v, T, n_kt, blockIdx.x + (i + kStages) * gridDim.x, smem_u32(ring + st * M::kTileBytes),
-                     smem_u32(&s_full[st]));
+    __syncthreads();  // every partial of this tile is written
     for (int j = tid; j < D; j += 128) {
       float a = s_part[buf][0][0][j], b = s_part[buf][1][0][j], c = s_part[buf][2][0][j];
 #pragma unroll
