@@ -56,7 +56,11 @@ typedef enum {
  *   beta    : device, float32 [H, d], beta >= 0
  *   out     : device, float32 [B, H, T, d]
  *   lse     : device, float32 [B, H, T], or NULL
- *   B, H, T : >= 1;  d in {64, 128};  causal: 0 (full prior) or 1
+ *   B, H, T : >= 1;  d in {16, 32, 64, 128};  causal: 0 (full prior) or 1
+ * d = 64 and 128 run on the tensor cores as below.  d = 16 and 32, too narrow
+ * for 64-channel tiles to pay, run on CUDA cores (fem_fwd_f32's kernel reading
+ * bf16): every product and sum in fp32, no workspace beyond 256 bytes, no
+ * fix-up rows.  Any other d is FEM_ERR_UNSUPPORTED.
  * Allocates its workspace stream-ordered on `stream` from a memory pool the
  * library keeps per device (freed memory stays in the pool for the next
  * call; the entry points that allocate all use it).  Accuracy: the score contraction takes bf16 q, k; the second

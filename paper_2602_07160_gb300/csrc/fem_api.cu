@@ -124,9 +124,18 @@ struct WsLayout {
   size_t tstat, chan, bcoef, shift, rfac, colsum, colmask, bank, fixups, count, total;
 };
 
+// Head dimensions of the bf16 read that run on CUDA cores (no workspace but the counters).
+bool small_d(int d) { return d == 16 || d == 32; }
+
 bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   (void)causal;  // the guard's fix-up list serves both forms of the read
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0) return false;
+  if (small_d(d)) {
+    *w = WsLayout{};
+    w->count = 0;
+    w->total = 256;
+    return true;
+  }
   const size_t BH = static_cast<size_t>(B) * H;
   const size_t n_kt = (static_cast<size_t>(T) + kBlockK - 1) / kBlockK;
   size_t off = 0;
@@ -173,6 +182,9 @@ int check_tc_sizes(int T, int d) {
   if (T > kMaxSeqLen) return FEM_ERR_UNSUPPORTED;
   return FEM_OK;
 }
+
+// Sizes the plain bf16 read takes: the tensor-core sizes, and d in {16, 32} on CUDA cores.
+int check_read_sizes(int T, int d) { return small_d(d) ? FEM_OK : check_tc_sizes(T, d); }
 
 // ---------------------------------------------------------------------------
 // Fixed scratch for fem_fwd_noalloc.  Some callers may not allocate device
@@ -274,6 +286,16 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
                     int H, int T, int d, int causal, uint8_t *ws, const GatedArgs *ga, DeviceState *ds,
                     cudaStream_t s) {
   const int BH = B * H;
+  if (small_d(d) && !ga) {
+    // CUDA cores, exact to fp32 rounding: no bank, no guard, no fix-up rows
+    cudaError_t e = cudaMemsetAsync(ds->last_fixup, 0, sizeof(int), s);
+    const cudaEvent_t ev0 = t_ev_start, ev1 = t_ev_stop;
+    t_ev_start = t_ev_stop = nullptr;
+    if (e == cudaSuccess && ev0) e = cudaEventRecord(ev0, s);
+    if (e == cudaSuccess) e = launch_simt_bf16(q, k, v, beta, out, lse, B, H, T, d, causal, s);
+    if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
+    return map_cuda(e);
+  }
   WsLayout w;
   ws_layout(B, H, T, d, causal, &w);
   BankWorkspace bw = bank_workspace(ws, w);
@@ -317,7 +339,7 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
                int T, int d, int causal, void *workspace, size_t workspace_bytes, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
-  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
+  if ((rc = check_read_sizes(T, d)) != FEM_OK) return rc;
   WsLayout w;
   ws_layout(B, H, T, d, causal, &w);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return FEM_ERR_INVALID_ARG;
@@ -332,7 +354,7 @@ int fem_fwd(const void *q, const void *k, const void *v, const float *beta, floa
             int T, int d, int causal, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
-  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
+  if ((rc = check_read_sizes(T, d)) != FEM_OK) return rc;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
   const size_t bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
@@ -487,7 +509,7 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
                  int H, int T, int d, int causal, void *stream) {
   if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0 || (causal != 0 && causal != 1)) return FEM_ERR_INVALID_ARG;
-  if (check_tc_sizes(T, d) != FEM_OK) return FEM_ERR_UNSUPPORTED;
+  if (check_read_sizes(T, d) != FEM_OK) return FEM_ERR_UNSUPPORTED;
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
@@ -573,7 +595,7 @@ int fem_fwd_noalloc(const void *q, const void *k, const void *v, const float *be
                     int H, int T, int d, int causal, void *stream) {
   int rc = check_common(q, k, v, beta, out, lse, B, H, T, d, causal);
   if (rc != FEM_OK) return rc;
-  if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
+  if ((rc = check_read_sizes(T, d)) != FEM_OK) return rc;
   const size_t need = fem_fwd_workspace_bytes(B, H, T, d, causal);
   if (need == 0 || need > kStaticScratchBytes) return FEM_ERR_NO_MEMORY;
   void *scratch = nullptr;

@@ -120,5 +120,8 @@ cudaError_t launch_bwd_f32(const float *q, const float *k, const float *v, const
 // fp32-input read on CUDA cores.
 cudaError_t launch_f32(const float *q, const float *k, const float *v, const float *beta, float *out, float *lse,
                        int B, int H, int T, int d, int causal, cudaStream_t stream);
+// bf16 inputs of head dimension 16 or 32 on the same CUDA-core kernel (fp32 arithmetic).
+cudaError_t launch_simt_bf16(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse,
+                             int B, int H, int T, int d, int causal, cudaStream_t stream);
 
 }  // namespace fem

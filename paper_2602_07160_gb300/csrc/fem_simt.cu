@@ -1,4 +1,7 @@
-// The FEM read for fp32 inputs on CUDA cores, exact to fp32 rounding.
+// The FEM read on CUDA cores, exact to fp32 rounding: fp32 inputs of any head
+// dimension up to 256, and bf16 inputs of head dimension 16 or 32 (too narrow
+// for the tensor-core read's 64-channel tiles to pay; here every product and
+// sum is fp32).
 //
 // One warp per output row t; lane l owns channels l, l+32, ...  For every key
 // i in the support the warp forms s_{t,i} = q_t . k_i / sqrt(d) (lane-partial
@@ -27,10 +30,14 @@ __device__ __forceinline__ float expm1_over_beta(float b, float x) {
   return b != 0.f ? expm1f(b * x) / b : x;
 }
 
-__global__ void __launch_bounds__(128) fem_f32_kernel(const float *__restrict__ q, const float *__restrict__ k,
-                                                       const float *__restrict__ v, const float *__restrict__ beta,
-                                                       float *__restrict__ out, float *__restrict__ lse, int H,
-                                                       int T, int d, int causal, long long n_rows) {
+__device__ __forceinline__ float ld_in(const float *p) { return *p; }
+__device__ __forceinline__ float ld_in(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
+
+template <typename In>
+__global__ void __launch_bounds__(128) fem_simt_kernel(const In *__restrict__ q, const In *__restrict__ k,
+                                                        const In *__restrict__ v, const float *__restrict__ beta,
+                                                        float *__restrict__ out, float *__restrict__ lse, int H,
+                                                        int T, int d, int causal, long long n_rows) {
   const int lane = threadIdx.x & 31;
   const long long row = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -40,15 +47,15 @@ __global__ void __launch_bounds__(128) fem_f32_kernel(const float *__restrict__ 
   const int n = causal ? t + 1 : T;
   const int per = (d + 31) / 32;
   const float inv_sqrt_d = rsqrtf(static_cast<float>(d));
-  const float *kb = k + bh * T * d;
-  const float *vb = v + bh * T * d;
+  const In *kb = k + bh * T * d;
+  const In *vb = v + bh * T * d;
 
   float qv[kSimtMaxPerLane], bj[kSimtMaxPerLane], c[kSimtMaxPerLane], A[kSimtMaxPerLane], W[kSimtMaxPerLane];
 #pragma unroll
   for (int u = 0; u < kSimtMaxPerLane; ++u) {
     const int j = lane + 32 * u;
     const bool ok = u < per && j < d;
-    qv[u] = ok ? q[row * d + j] : 0.f;
+    qv[u] = ok ? ld_in(q + row * d + j) : 0.f;
     bj[u] = ok ? beta[h * d + j] : 0.f;
     c[u] = -INFINITY;
     A[u] = 0.f;
@@ -57,12 +64,12 @@ __global__ void __launch_bounds__(128) fem_f32_kernel(const float *__restrict__ 
   float m = -INFINITY, L = 0.f;
 
   for (int i = 0; i < n; ++i) {
-    const float *kr = kb + static_cast<long long>(i) * d;
+    const In *kr = kb + static_cast<long long>(i) * d;
     float part = 0.f;
 #pragma unroll
     for (int u = 0; u < kSimtMaxPerLane; ++u) {
       const int j = lane + 32 * u;
-      if (u < per && j < d) part = fmaf(qv[u], kr[j], part);
+      if (u < per && j < d) part = fmaf(qv[u], ld_in(kr + j), part);
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
@@ -78,12 +85,12 @@ __global__ void __launch_bounds__(128) fem_f32_kernel(const float *__restrict__ 
       m = s;
     }
     const float p = expf(s - m);
-    const float *vr = vb + static_cast<long long>(i) * d;
+    const In *vr = vb + static_cast<long long>(i) * d;
 #pragma unroll
     for (int u = 0; u < kSimtMaxPerLane; ++u) {
       const int j = lane + 32 * u;
       if (!(u < per && j < d)) continue;
-      const float x = vr[j];
+      const float x = ld_in(vr + j);
       const float b = bj[u];
       if (x > c[u]) {
         if (c[u] != -INFINITY) {
@@ -120,8 +127,18 @@ cudaError_t launch_f32(const float *q, const float *k, const float *v, const flo
                        int B, int H, int T, int d, int causal, cudaStream_t stream) {
   const long long n_rows = static_cast<long long>(B) * H * T;
   const long long blocks = (n_rows + 3) / 4;
-  fem_f32_kernel<<<static_cast<unsigned>(blocks), 128, 0, stream>>>(q, k, v, beta, out, lse, H, T, d, causal,
-                                                                    n_rows);
+  fem_simt_kernel<float><<<static_cast<unsigned>(blocks), 128, 0, stream>>>(q, k, v, beta, out, lse, H, T, d,
+                                                                            causal, n_rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_simt_bf16(const void *q, const void *k, const void *v, const float *beta, float *out, float *lse,
+                             int B, int H, int T, int d, int causal, cudaStream_t stream) {
+  const long long n_rows = static_cast<long long>(B) * H * T;
+  const long long blocks = (n_rows + 3) / 4;
+  fem_simt_kernel<__nv_bfloat16><<<static_cast<unsigned>(blocks), 128, 0, stream>>>(
+      static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
+      static_cast<const __nv_bfloat16 *>(v), beta, out, lse, H, T, d, causal, n_rows);
   return cudaGetLastError();
 }
 

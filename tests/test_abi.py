@@ -69,8 +69,17 @@ def test_argument_errors_are_synchronous(lib, fn):
 
 def test_unsupported_head_dim(lib):
     assert _call(lib, "fem_fwd", d=96) == 2
-    assert _call(lib, "fem_fwd_host", d=32) == 2
+    assert _call(lib, "fem_fwd", d=8) == 2
+    assert _call(lib, "fem_fwd_host", d=48) == 2
     assert _call(lib, "fem_fwd_f32", d=300) == 2
+
+
+def test_small_head_dims_take_no_workspace(lib):
+    """bf16 d in {16, 32} runs on CUDA cores: only the fix-up counters' 256 bytes."""
+    lib.fem_fwd_workspace_bytes.restype = ctypes.c_size_t
+    for d in (16, 32):
+        assert lib.fem_fwd_workspace_bytes(4, 16, 8192, d, 1) == 256
+    assert lib.fem_fwd_workspace_bytes(4, 16, 8192, 64, 1) > (1 << 20)
 
 
 @pytest.mark.parametrize("fn", ["fem_fwd", "fem_fwd_host", "fem_fwd_noalloc"])
