@@ -527,6 +527,25 @@ def run_fem(args):
                                "shape": {"B": Bg, "H": Hg, "T": Tg, "m": mg, "d": dg},
                                "what": "fem_gla_fwd: FEM over a GLA prior, O(T) recurrent fp32 scan on CUDA cores; "
                                        "FLOPs 4 m (d + 1) per step and head"}
+        # the same read chunked on the tensor cores (bf16 operands, fp32 state), same inputs
+        fem.fem_gla_fwd_tc(qf, kf, vg, lg, bg, out=go, logz=False, stream=stream)
+        a0.record(stream)
+        for _ in range(3):
+            fem.fem_gla_fwd_tc(qf, kf, vg, lg, bg, out=go, logz=False, stream=stream)
+        a1.record(stream)
+        torch.cuda.synchronize(device)
+        fem.check_device_error(stream)
+        glt_ms = a0.elapsed_time(a1) / 3
+        # per 128-step chunk: Qf Kf^T (128 x 128 x m), the masked A E^T (128 x 80 x 128), Qf Shat^T
+        # (128 x 80 x m) and the state's K^T E^T (128 x 80 x 128, half of its rows padding), 2 FLOP per MAC
+        n_chunks = Bg * Hg * ((Tg + 127) // 128)
+        glt_flops = 2.0 * n_chunks * (128 * 128 * mg + 128 * 80 * 128 + 128 * 80 * mg + 128 * 80 * 128)
+        context["gla_read_tc"] = {"ms": glt_ms, "tflops": glt_flops / (glt_ms * 1e-3) / 1e12,
+                                  "peak_tflops": peak, "frac": glt_flops / (glt_ms * 1e-3) / 1e12 / peak,
+                                  "speedup_over_scan": gla_ms / glt_ms,
+                                  "what": "fem_gla_fwd_tc: the GLA-prior read in 128-step chunks, four tcgen05 "
+                                          "contractions per chunk (bf16 operands, fp32 accumulation and state), "
+                                          "one CTA per (b, h); FLOPs those of the four contractions"}
         del qf, kf, vg, lg, bg, go
         # the time-decay conditioner's convolution, H_c = 64 channels over the same B and T (HBM-bound)
         Hc = 64

@@ -205,6 +205,26 @@ int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *l
                 void *stream);
 
 /*
+ * fem_gla_fwd_tc -- the same read (fem_gla_fwd's definition and arguments)
+ * chunked on the tensor cores, for m = d = 64 (FEM_ERR_UNSUPPORTED
+ * otherwise).  One CTA per (b, h) walks 128-step chunks: the decay-masked
+ * qf kf^T of the chunk against the chunk's value bank, qf against the state
+ * of the earlier chunks, and the state's update, as bf16 contractions with
+ * fp32 accumulation (tcgen05); the state itself is kept in fp32.  Channels
+ * with beta < 1/4 use the bank expm1(beta (v - c)) / beta anchored at the
+ * smallest value so far, the others exp(beta v - lambda) with a log-scaled
+ * state.  Accuracy is the bf16 read's for values of unit spread (max abs 2e-2,
+ * mean abs 2e-3 against the float64 definition); per entry the bound is about
+ * 2^-8 |v - c| (linear) or 2^-8 / beta (shifted), so it scales with the
+ * values' spread.  Entries whose in-chunk part could be carried by terms
+ * under fp32's range are recomputed exactly.  No workspace; qf, kf, v, out
+ * 16-byte aligned.
+ */
+int fem_gla_fwd_tc(const float *qf, const float *kf, const float *v, const float *logdecay,
+                   const float *beta, float *out, float *logz, int B, int H, int T, int m, int d,
+                   void *stream);
+
+/*
  * fem_tdc_conv -- the time-decay conditioner's convolution (App. "Low-rank
  * Convolution: Time-Decay Conditioner (TDC)", Eq. "tdc-conv", streaming form
  * of Prop. "tdc-lowrank"):

@@ -21,7 +21,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libfem.so")
-SOURCES = ["fem_api.cu", "fem_tc.cu", "fem_bank.cu", "fem_fixup.cu", "fem_simt.cu", "fem_decode.cu", "fem_gla.cu", "fem_tdc.cu", "fem_bwd.cu"]
+SOURCES = ["fem_api.cu", "fem_tc.cu", "fem_bank.cu", "fem_fixup.cu", "fem_simt.cu", "fem_decode.cu", "fem_gla.cu", "fem_gla_tc.cu", "fem_tdc.cu", "fem_bwd.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

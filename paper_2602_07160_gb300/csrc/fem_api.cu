@@ -439,6 +439,24 @@ int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc,
   return map_cuda(e);
 }
 
+int fem_gla_fwd_tc(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta,
+                   float *out, float *logz, int B, int H, int T, int m, int d, void *stream) {
+  if (!qf || !kf || !v || !logdecay || !beta || !out) return FEM_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || T <= 0 || m <= 0 || d <= 0) return FEM_ERR_INVALID_ARG;
+  if (!aligned16(qf) || !aligned16(kf) || !aligned16(v) || !aligned16(out)) return FEM_ERR_INVALID_ARG;
+  for (const void *p : {static_cast<const void *>(logdecay), static_cast<const void *>(beta),
+                        static_cast<const void *>(logz)})
+    if (p && (reinterpret_cast<uintptr_t>(p) & 3u)) return FEM_ERR_INVALID_ARG;
+  if (m != 64 || d != 64) return FEM_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * H > 2147483647ll || static_cast<long long>(B) * H * T * 64 >= (1ll << 40))
+    return FEM_ERR_UNSUPPORTED;
+  DeviceState *ds = nullptr;
+  int rc = device_state(&ds);
+  if (rc != FEM_OK) return rc;
+  return map_cuda(launch_gla_tc(qf, kf, v, logdecay, beta, out, logz, B, H, T, ds->err,
+                                static_cast<cudaStream_t>(stream)));
+}
+
 int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta, float *out,
                 float *logz, int B, int H, int T, int m, int d, void *stream) {
   if (!qf || !kf || !v || !logdecay || !beta || !out) return FEM_ERR_INVALID_ARG;

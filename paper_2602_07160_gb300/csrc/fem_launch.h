@@ -107,6 +107,10 @@ cudaError_t launch_gla(const float *qf, const float *kf, const float *v, const f
                        float *out, float *logz, int BH, int H, int T, int m, int d, void *ws, int num_sms,
                        cudaStream_t stream);
 
+// The GLA-prior read chunked on the tensor cores (m = d = 64), one CTA per (b, h).
+cudaError_t launch_gla_tc(const float *qf, const float *kf, const float *v, const float *logdecay, const float *beta,
+                          float *out, float *logz, int B, int H, int T, unsigned *err, cudaStream_t stream);
+
 // Time-decay conditioner convolution h_t = exp(-s_t) h_{t-1} + u_t over [B, T, Hc]
 // (segmented scan); `ws` holds tdc_workspace_bytes() bytes.
 size_t tdc_workspace_bytes(int B, int T, int Hc);

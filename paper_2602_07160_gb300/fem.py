@@ -24,7 +24,7 @@ STATUS = {0: "FEM_OK", 1: "FEM_ERR_INVALID_ARG", 2: "FEM_ERR_UNSUPPORTED", 3: "F
 EXPORTS = ["fem_fwd", "fem_fwd_ws", "fem_fwd_workspace_bytes", "fem_fwd_f32", "fem_fwd_host",
            "fem_check_device_error", "fem_last_fixup_rows", "fem_set_kernel_events", "fem_status_str",
            "fem_fwd_noalloc", "fem_fwd_gated", "fem_decode", "fem_gla_fwd", "fem_tdc_conv", "fem_bwd_f32",
-           "fem_probe_wait_timeout", "fem_attn_fwd"]
+           "fem_probe_wait_timeout", "fem_attn_fwd", "fem_gla_fwd_tc"]
 
 
 class FemError(RuntimeError):
@@ -61,6 +61,8 @@ def load(path: str | None = None):
         lib.fem_decode.restype = i
         lib.fem_gla_fwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
         lib.fem_gla_fwd.restype = i
+        lib.fem_gla_fwd_tc.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
+        lib.fem_gla_fwd_tc.restype = i
         lib.fem_tdc_conv.argtypes = [vp, vp, vp, i, i, i, vp]
         lib.fem_tdc_conv.restype = i
         lib.fem_bwd_f32.argtypes = [vp] * 11 + [i, i, i, i, i, vp]
@@ -207,7 +209,12 @@ def fem_decode(q, k, v, beta, out=None, lse=None, stream=None):
     return out, (None if lse is False else lse)
 
 
-def fem_gla_fwd(qf, kf, v, logdecay, beta, out=None, logz=None, stream=None):
+def fem_gla_fwd_tc(qf, kf, v, logdecay, beta, out=None, logz=None, stream=None):
+    """fem_gla_fwd chunked on the tensor cores (m = d = 64; bf16 operands, fp32 state)."""
+    return fem_gla_fwd(qf, kf, v, logdecay, beta, out=out, logz=logz, stream=stream, _entry="fem_gla_fwd_tc")
+
+
+def fem_gla_fwd(qf, kf, v, logdecay, beta, out=None, logz=None, stream=None, _entry="fem_gla_fwd"):
     """The read over a GLA prior on fp32 CUDA tensors.
 
     qf, kf: [B, H, T, m] nonnegative features; v: [B, H, T, d]; logdecay: [B, H, T] (<= 0);
@@ -225,10 +232,10 @@ def fem_gla_fwd(qf, kf, v, logdecay, beta, out=None, logz=None, stream=None):
         out = torch.empty((B, H, T, d), dtype=torch.float32, device=qf.device)
     if logz is None:
         logz = torch.empty((B, H, T), dtype=torch.float32, device=qf.device)
-    rc = load().fem_gla_fwd(_ptr(qf), _ptr(kf), _ptr(v), _ptr(logdecay), _ptr(beta), _ptr(out),
-                            None if logz is False else _ptr(logz), B, H, T, m, d, _stream(stream, qf.device))
+    rc = getattr(load(), _entry)(_ptr(qf), _ptr(kf), _ptr(v), _ptr(logdecay), _ptr(beta), _ptr(out),
+                                 None if logz is False else _ptr(logz), B, H, T, m, d, _stream(stream, qf.device))
     if rc != 0:
-        raise FemError("fem_gla_fwd", rc)
+        raise FemError(_entry, rc)
     return out, (None if logz is False else logz)
 
 
