@@ -87,28 +87,24 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // (truncation below 4e-6 relative), (e^y - 1) / beta beyond (ex2.approx: the result
 // is rounded to bf16); x itself at beta = 0.
 __device__ __forceinline__ float em1_beta_fast(float x, float y, float rb) {
-  if (fabsf(y) < 0.5f) {
-    float p = fmaf(y, 1.f / 720.f, 1.f / 120.f);
-    p = fmaf(y, p, 1.f / 24.f);
-    p = fmaf(y, p, 1.f / 6.f);
-    p = fmaf(y, p, 0.5f);
-    p = fmaf(y, p, 1.f);
-    return x * p;
-  }
-  return (__expf(y) - 1.f) * rb;
+  float p = fmaf(y, 1.f / 720.f, 1.f / 120.f);  // both forms, then a select: no branch per element
+  p = fmaf(y, p, 1.f / 24.f);
+  p = fmaf(y, p, 1.f / 6.f);
+  p = fmaf(y, p, 0.5f);
+  p = fmaf(y, p, 1.f);
+  const float far = (__expf(y) - 1.f) * rb;
+  return fabsf(y) < 0.5f ? x * p : far;
 }
 
 // log1p(x) for x > -1: the series to x^5 for |x| < 2^-6 (truncation below 2^-36
 // relative), lg2.approx of 1 + x beyond.
 __device__ __forceinline__ float log1p_fast(float x) {
-  if (fabsf(x) < 0.015625f) {
-    float p = fmaf(x, 0.2f, -0.25f);
-    p = fmaf(x, p, 1.f / 3.f);
-    p = fmaf(x, p, -0.5f);
-    p = fmaf(x, p, 1.f);
-    return x * p;
-  }
-  return __logf(1.f + x);
+  float p = fmaf(x, 0.2f, -0.25f);  // both forms, then a select
+  p = fmaf(x, p, 1.f / 3.f);
+  p = fmaf(x, p, -0.5f);
+  p = fmaf(x, p, 1.f);
+  const float far = __logf(1.f + x);
+  return fabsf(x) < 0.015625f ? x * p : far;
 }
 
 // 8 consecutive fp32 as bf16 into a 16-byte chunk of a 128-byte-swizzled row.
@@ -264,6 +260,8 @@ __global__ void __launch_bounds__(256, 1)
       const float mn = fminf(fminf(pmin[j], pmin[kGD + j]), fminf(pmin[2 * kGD + j], pmin[3 * kGD + j]));
       if (b >= kGlaLinBeta) {
         c_lam[j] = b * mx;
+        pmax[j] = 1.f;  // no move of the state (see below)
+        pmin[j] = 0.f;
       } else {
         // the anchor: the mean of the values so far, at most 1/beta above their minimum (so that
         // 1 + beta num / Z >= 1/e); the state moves with it (either way)
@@ -273,12 +271,23 @@ __global__ void __launch_bounds__(256, 1)
         c_rsum[j] = rsum;
         const float mean = rsum / static_cast<float>(c * kGC + rows);
         const float cn = b > 0.f ? fminf(mean, rmin + 1.f / b) : mean, co = c_anc[j];
+        // the state's move with the anchor: factors here, the transform by every thread below
+        float e = 1.f, w = 0.f;
         if (co != INFINITY && cn != co) {
-          const float x = co - cn, e = expf(b * x), w = b != 0.f ? expm1f(b * x) / b : x;
-          for (int f = 0; f < kGM; ++f) Sf[j * kGM + f] = fmaf(e, Sf[j * kGM + f], w * Sf[kGD * kGM + f]);
+          const float x = co - cn;
+          e = expf(b * x);
+          w = b != 0.f ? expm1f(b * x) / b : x;
         }
+        pmax[j] = e;  // the chunk's extremes are consumed; their space holds the factors
+        pmin[j] = w;
         c_anc[j] = cn;
       }
+    }
+    __syncthreads();
+    for (int i = tid; i < kGD * kGM; i += 256) {
+      const int j = i >> 6, f = i & 63;
+      const float e = pmax[j], w = pmin[j];
+      if (e != 1.f || w != 0.f) Sf[i] = fmaf(e, Sf[i], w * Sf[kGD * kGM + f]);
     }
     __syncthreads();
     // the chunk's bank (channels x keys, K-major) and the state's bf16 copy (channels x features)
@@ -394,17 +403,16 @@ __global__ void __launch_bounds__(256, 1)
       for (int u = 0; u < 32; ++u) {
         const int j = q * 32 + u;
         const float b = c_beta[j], rb = c_rb[j], in = __uint_as_float(ai[u]), ix = __uint_as_float(ax[u]);
-        if (b < kGlaLinBeta) {
-          const float num = fmaf(et, ix, in);
-          o[u] = b != 0.f ? c_anc[j] + log1p_fast(b * num * rZ) * rb : c_anc[j] + num * rZ;
-        } else {
-          if (!(in >= 0x1p-100f * zi)) flag |= 1u << u;
-          const float la = in > 0.f ? c_lam[j] + __logf(in) : -INFINITY;
-          const float lb = ix > 0.f ? c_mu[j] + gt + __logf(ix) : -INFINITY;
-          const float hi = fmaxf(la, lb), lo = fminf(la, lb);
-          const float ln = hi == -INFINITY ? -INFINITY : hi + __logf(1.f + __expf(lo - hi));
-          o[u] = (ln - lz) * rb;
-        }
+        // both forms, then a select (the form is the channel's; no branch per element)
+        const bool lin = b < kGlaLinBeta;
+        const float num = fmaf(et, ix, in), x = b * num * rZ;
+        const float o_lin = b != 0.f ? fmaf(log1p_fast(x), rb, c_anc[j]) : fmaf(num, rZ, c_anc[j]);
+        const float la = in > 0.f ? c_lam[j] + __logf(in) : -INFINITY;
+        const float lb = ix > 0.f ? c_mu[j] + gt + __logf(ix) : -INFINITY;
+        const float hi = fmaxf(la, lb), lo = fminf(la, lb);
+        const float ln = hi == -INFINITY ? -INFINITY : hi + __logf(1.f + __expf(lo - hi));
+        o[u] = lin ? o_lin : (ln - lz) * rb;
+        flag |= (!lin && !(in >= 0x1p-100f * zi)) ? 1u << u : 0u;
       }
       if (t < rows) {
         float *orow = out + (r0 + t) * kGD + q * 32;
