@@ -159,9 +159,10 @@ __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__
 // plan: one block per (b, h) and group of 32 channels, four threads per
 // channel, each holding a quarter of a window of 64 key tiles in registers so
 // every load of a window is in flight at once.  The lazy shift is a sequential
-// recurrence over tiles: the four quarters run it in turn, handing the running
-// (max, shift) on by warp shuffles.  Besides the schedule it writes the bank's
-// per-tile coefficients (BankCoef) and the moved-channel word of its group.
+// recurrence over tiles: one lane per channel walks it over the window's tile
+// maxima in shared memory, then the four lanes write the window's schedule in
+// parallel.  Besides the schedule it writes the bank's per-tile coefficients
+// (BankCoef) and the moved-channel word of its group.
 // ---------------------------------------------------------------------------
 template <int D>
 __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ tstat, const float *__restrict__ beta,
@@ -170,6 +171,8 @@ __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ ts
                                                    unsigned *__restrict__ colmask, float4 *__restrict__ bcoef) {
   constexpr int kParts = 4, kPer = 16, kWin = kParts * kPer;
   __shared__ unsigned s_mask[kWin];
+  __shared__ float s_tm[kWin][33];      // the window's tile maxima per channel of the block
+  __shared__ float s_cl[kWin + 1][33];  // the shift before the window and after each of its tiles
   const int tid = threadIdx.x, part = tid % kParts, lane = tid & 31;
   const int grp = blockIdx.y, j = grp * 32 + tid / kParts;
   const int bh = blockIdx.x, h = bh % H;
@@ -210,43 +213,47 @@ __global__ void __launch_bounds__(128) plan_kernel(const float4 *__restrict__ ts
   }
   if (part == 0) chan[bh * D + j] = ci;
   const bool lin = ci.linear != 0.f;
-  // pass 2: running maximum, lazy shift, rescale factors, moved-channel masks
-  float cp = -INFINITY, cl = -INFINITY;
+  // pass 2, per window of 64 key tiles: the running maximum and the lazy shift are a
+  // sequential recurrence, walked by one lane per channel over the window's tile maxima in
+  // shared memory; then the four lanes of the channel write their quarter of the tiles'
+  // shift, rescale factor, bank coefficients and moved-channel bits in parallel
+  const int jl = tid / kParts;
+  float cp = -INFINITY, cl = -INFINITY;  // carried across windows by the walking lane
   for (int w0 = 0; w0 < n_kt; w0 += kWin) {
-    float tmx[kPer];
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
       const int kt = w0 + part * kPer + u;
-      tmx[u] = kt < n_kt ? ts[static_cast<size_t>(kt) * D].x : -INFINITY;
+      s_tm[part * kPer + u][jl] = kt < n_kt ? ts[static_cast<size_t>(kt) * D].x : -INFINITY;
     }
     for (int i = tid; i < kWin; i += 128) s_mask[i] = 0u;
     __syncthreads();
-    for (int stage = 0; stage < kParts; ++stage) {
-      if (part == stage) {
-#pragma unroll
-        for (int u = 0; u < kPer; ++u) {
-          const int kt = w0 + stage * kPer + u;
-          if (kt < n_kt) {
-            cp = fmaxf(cp, tmx[u]);
-            const float prev = cl;
-            if (lin) {
-              cl = ci.c_lin;
-            } else if (cl == -INFINITY || b * (cp - cl) > kShiftLag) {
-              cl = cp;
-            }
-            const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
-            shift[o] = cl;
-            const bool moved = !lin && kt > 0 && cl != prev;
-            rfac[o] = moved ? expf(b * (prev - cl)) : 1.f;
-            if (moved) atomicOr(&s_mask[stage * kPer + u], 1u << (j & 31));
-            bcoef[o] = lin ? make_float4(b > 0.f ? 1.f / b : 0.f, b, cl, __int_as_float(0x7fc00000))
-                           : make_float4(b * kLog2e, (kBankOffset - b * cl) * kLog2e, cl, 0.f);
-          }
+    if (part == 0) {
+      s_cl[0][jl] = cl;
+#pragma unroll 16
+      for (int u = 0; u < kWin; ++u) {
+        cp = fmaxf(cp, s_tm[u][jl]);
+        if (lin) {
+          cl = ci.c_lin;
+        } else if (cl == -INFINITY || b * (cp - cl) > kShiftLag) {
+          cl = cp;
         }
+        s_cl[u + 1][jl] = cl;
       }
-      // the quarter that ran hands its state on to the channel's other lanes
-      cp = __shfl_sync(0xffffffffu, cp, (lane & ~(kParts - 1)) | stage);
-      cl = __shfl_sync(0xffffffffu, cl, (lane & ~(kParts - 1)) | stage);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int w = part * kPer + u, kt = w0 + w;
+      if (kt < n_kt) {
+        const float c = s_cl[w + 1][jl], prev = s_cl[w][jl];
+        const size_t o = (static_cast<size_t>(bh) * n_kt + kt) * D + j;
+        shift[o] = c;
+        const bool moved = !lin && kt > 0 && c != prev;
+        rfac[o] = moved ? expf(b * (prev - c)) : 1.f;
+        if (moved) atomicOr(&s_mask[w], 1u << (j & 31));
+        bcoef[o] = lin ? make_float4(b > 0.f ? 1.f / b : 0.f, b, c, __int_as_float(0x7fc00000))
+                       : make_float4(b * kLog2e, (kBankOffset - b * c) * kLog2e, c, 0.f);
+      }
     }
     __syncthreads();
     for (int i = tid; i < kWin; i += 128) {
