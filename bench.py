@@ -536,16 +536,18 @@ def run_fem(args):
         torch.cuda.synchronize(device)
         fem.check_device_error(stream)
         glt_ms = a0.elapsed_time(a1) / 3
-        # per 128-step chunk: Qf Kf^T (128 x 128 x m), the masked A E^T (128 x 80 x 128), Qf Shat^T
-        # (128 x 80 x m) and the state's K^T E^T (128 x 80 x 128, half of its rows padding), 2 FLOP per MAC
-        n_chunks = Bg * Hg * ((Tg + 127) // 128)
-        glt_flops = 2.0 * n_chunks * (128 * 128 * mg + 128 * 80 * 128 + 128 * 80 * mg + 128 * 80 * 128)
+        # per 128-step chunk and CTA (two per head, 32 channels each): Qf Kf^T (128 x 128 x m), the masked
+        # A E^T (128 x 48 x 128), Qf Shat^T (128 x 48 x m) and the state's K^T E^T (128 x 48 x 128, half of
+        # its rows padding), 2 FLOP per MAC: the contractions the kernel issues
+        n_chunks = 2 * Bg * Hg * ((Tg + 127) // 128)
+        glt_flops = 2.0 * n_chunks * (128 * 128 * mg + 128 * 48 * 128 + 128 * 48 * mg + 128 * 48 * 128)
         context["gla_read_tc"] = {"ms": glt_ms, "tflops": glt_flops / (glt_ms * 1e-3) / 1e12,
                                   "peak_tflops": peak, "frac": glt_flops / (glt_ms * 1e-3) / 1e12 / peak,
                                   "speedup_over_scan": gla_ms / glt_ms,
                                   "what": "fem_gla_fwd_tc: the GLA-prior read in 128-step chunks, four tcgen05 "
                                           "contractions per chunk (bf16 operands, fp32 accumulation and state), "
-                                          "one CTA per (b, h); FLOPs those of the four contractions"}
+                                          "two CTAs per (b, h) of 32 channels each; FLOPs those of the "
+                                          "contractions issued"}
         del qf, kf, vg, lg, bg, go
         # the time-decay conditioner's convolution, H_c = 64 channels over the same B and T (HBM-bound)
         Hc = 64

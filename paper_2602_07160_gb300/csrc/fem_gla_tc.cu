@@ -5,17 +5,18 @@
 //   s_t(i) = K_{t,i} <qf_t, kf_i> (i <= t),  K_{t,i} = exp(g_{i+1} + ... + g_t),
 //   p_t = s_t / Z_t,  o_{t,j} = (1/beta_j) log sum_i p_t(i) exp(beta_j v_{i,j}).
 //
-// One CTA per (b, h) walks the sequence in chunks of 128 steps.  With gamma_t
+// Two CTAs per (b, h), 32 value channels each, walk the sequence in chunks of
+// 128 steps (the score and mask work is repeated in both).  With gamma_t
 // the running sum of g inside the chunk (so K_{t,i} = exp(gamma_t - gamma_i) for
 // i, t in the chunk and exp(gamma_t) from the chunk start), a chunk is four
 // contractions on tcgen05 (kind::f16, bf16 operands, fp32 accumulation in TMEM):
 //
 //   S     = Qf Kf^T                                  [128 x 128], K = m
-//   intra = (S o decay-mask) E^T                     [128 x 80],  K = 128 keys
-//   inter = Qf Shat^T                                [128 x 80],  K = m
-//   U     = (Kf o exp(gamma_last - gamma_i))^T E^T   [m x 80],    K = 128 keys
+//   intra = (S o decay-mask) E^T                     [128 x 48],  K = 128 keys
+//   inter = Qf Shat^T                                [128 x 48],  K = m
+//   U     = (Kf o exp(gamma_last - gamma_i))^T E^T   [m x 48],    K = 128 keys
 //
-// E holds, per channel j and key i, the value bank of the chunk; channel 64 is
+// E holds, per channel j and key i, the value bank of the chunk; channel 32 is
 // the constant 1 that gives the normaliser Z ("A one-pass implementation
 // appends a constant channel to values").  Shat is the state, sum over earlier
 // keys of K_{.,i} kf_i E_ij, kept in fp32 (the bf16 copy only feeds the
@@ -24,7 +25,7 @@
 //   beta_j <  1/4: linear, E = expm1(beta (v - c)) / beta with the anchor c the
 //     mean of the values so far, at most 1/beta above their minimum; when c moves
 //     to c', the state becomes e^{beta (c - c')} Shat_j + expm1(beta (c - c')) / beta
-//     Shat_64, and the read is o = c + log1p(beta num / Z) / beta (c + num / Z at
+//     Shat_Z (the constant channel's state), and the read is o = c + log1p(beta num / Z) / beta (c + num / Z at
 //     beta = 0);
 //   beta_j >= 1/4: shifted, E = exp(beta v - lambda) with lambda the chunk's
 //     largest beta v, the state carried as e^{mu} Shat with mu the log of its
@@ -46,8 +47,11 @@ namespace {
 
 constexpr int kGC = 128;        // steps per chunk (rows of S, TMEM lanes)
 constexpr int kGM = 64;         // feature width
-constexpr int kGD = 64;         // value channels
-constexpr int kGN = 80;         // channels, the constant channel, zero padding to a multiple of 16
+constexpr int kVD = 64;         // value channels of a head (the row width of v and out)
+constexpr int kGD = 32;         // value channels of a CTA: two CTAs share a head
+constexpr int kGN = 48;         // the CTA's channels, the constant channel, zero padding to a multiple of 16
+constexpr int kQtr = 256 / kGD;  // groups of keys in the per-channel passes (thread = channel and group)
+constexpr int kKg = kGC / kQtr;  // keys per group
 constexpr float kGlaLinBeta = 0.25f;
 
 struct GLay {
@@ -58,16 +62,16 @@ struct GLay {
   static constexpr uint32_t kQ16 = 103424;                         // 1024-aligned operands from here
   static constexpr uint32_t kK16 = kQ16 + 16384;
   static constexpr uint32_t kKT16 = kK16 + 16384;  // two boxes of 128 rows (64 features, 64 zero) x 64 keys
-  static constexpr uint32_t kE16 = kKT16 + 32768;  // two boxes of 80 channels x 64 keys
-  static constexpr uint32_t kEBox = 10240;
-  static constexpr uint32_t kS16 = kE16 + 2 * kEBox;    // 80 channels x 64 features
-  static constexpr uint32_t kSf = kS16 + 10240;         // fp32 state [channel][feature]
+  static constexpr uint32_t kE16 = kKT16 + 32768;  // two boxes of kGN channels x 64 keys
+  static constexpr uint32_t kEBox = kGN * 128;
+  static constexpr uint32_t kS16 = kE16 + 2 * kEBox;    // kGN channels x 64 features
+  static constexpr uint32_t kSf = kS16 + kGN * 128;     // fp32 state [channel][feature]
   static constexpr uint32_t kChan = kSf + kGN * kGM * 4;  // per channel: beta, anchor, mu, lambda, running min and sum, 1/beta
   static constexpr uint32_t kBar = kChan + 7 * kGN * 4;
   static constexpr uint32_t kTmemSlot = kBar + 32;
   static constexpr uint32_t kBytes = kTmemSlot + 32;
   static constexpr uint32_t kAlloc = kBytes + 1024;
-  static_assert(kPart + 3 * 4 * kGD * 4 <= kQ16, "partials fit below the operands");
+  static_assert(kPart + 3 * kQtr * kGD * 4 <= kQ16, "partials fit below the operands");
   static_assert(kQ16 % 1024 == 0 && kK16 % 1024 == 0 && kKT16 % 1024 == 0 && kE16 % 1024 == 0 &&
                     kEBox % 1024 == 0 && kS16 % 1024 == 0,
                 "swizzled operands on 1024-byte boundaries");
@@ -122,12 +126,12 @@ __global__ void __launch_bounds__(256, 1)
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int bh = blockIdx.x, h = bh % H;
+  const int bh = blockIdx.x, h = bh % H, jo = blockIdx.y * kGD;  // the head, its first channel here
   const int n_ch = (T + kGC - 1) / kGC;
   float *q32 = reinterpret_cast<float *>(smem + GLay::kQ32), *k32 = reinterpret_cast<float *>(smem + GLay::kK32),
         *v32 = reinterpret_cast<float *>(smem + GLay::kV32);
   float *gam = reinterpret_cast<float *>(smem + GLay::kGam), *dk = reinterpret_cast<float *>(smem + GLay::kDk);
-  float *pmax = reinterpret_cast<float *>(smem + GLay::kPart), *pmin = pmax + 4 * kGD, *psum = pmin + 4 * kGD;
+  float *pmax = reinterpret_cast<float *>(smem + GLay::kPart), *pmin = pmax + kQtr * kGD, *psum = pmin + kQtr * kGD;
   float *Sf = reinterpret_cast<float *>(smem + GLay::kSf);
   float *c_beta = reinterpret_cast<float *>(smem + GLay::kChan), *c_anc = c_beta + kGN, *c_mu = c_anc + kGN,
         *c_lam = c_mu + kGN, *c_rmin = c_lam + kGN, *c_rsum = c_rmin + kGN, *c_rb = c_rsum + kGN;
@@ -137,11 +141,11 @@ __global__ void __launch_bounds__(256, 1)
   auto issue_inputs = [&](int c) {  // the chunk's rows of qf, kf and v (contiguous in [B, H, T, .])
     const int rows = min(kGC, T - c * kGC);
     const size_t r0 = base_row + static_cast<size_t>(c) * kGC;
-    const uint32_t bytes = static_cast<uint32_t>(rows) * kGM * 4;
-    mbar_arrive_expect_tx(bar_in, 3 * bytes);
+    const uint32_t bytes = static_cast<uint32_t>(rows) * kGM * 4, vbytes = static_cast<uint32_t>(rows) * kVD * 4;
+    mbar_arrive_expect_tx(bar_in, 2 * bytes + vbytes);
     bulk_load(sbase + GLay::kQ32, qf + r0 * kGM, bytes, bar_in);
     bulk_load(sbase + GLay::kK32, kf + r0 * kGM, bytes, bar_in);
-    bulk_load(sbase + GLay::kV32, v + r0 * kGD, bytes, bar_in);
+    bulk_load(sbase + GLay::kV32, v + r0 * kVD, vbytes, bar_in);  // whole rows: both CTAs' channels
   };
 
   if (tid == 0) {
@@ -161,16 +165,16 @@ __global__ void __launch_bounds__(256, 1)
     const int bx = i >> 9, r = 64 + ((i >> 3) & 63), ch = i & 7;
     *reinterpret_cast<uint4 *>(smem + GLay::kKT16 + bx * 16384 + sw128_offset(r, ch)) = make_uint4(0u, 0u, 0u, 0u);
   }
-  for (int i = tid; i < 2 * 16 * 8; i += 256) {
-    const int bx = i >> 7, r = 64 + ((i >> 3) & 15), ch = i & 7;
-    const uint32_t one = r == 64 ? pack_bf16x2(1.f, 1.f) : 0u;
+  for (int i = tid; i < 2 * (kGN - kGD) * 8; i += 256) {
+    const int bx = i / ((kGN - kGD) * 8), r = kGD + (i >> 3) % (kGN - kGD), ch = i & 7;
+    const uint32_t one = r == kGD ? pack_bf16x2(1.f, 1.f) : 0u;
     *reinterpret_cast<uint4 *>(smem + GLay::kE16 + bx * GLay::kEBox + sw128_offset(r, ch)) = make_uint4(one, one, one, one);
   }
   for (int i = tid; i < kGN * kGM; i += 256) Sf[i] = 0.f;
   for (int i = tid; i < kGN * 8; i += 256)
     *reinterpret_cast<uint4 *>(smem + GLay::kS16 + sw128_offset(i >> 3, i & 7)) = make_uint4(0u, 0u, 0u, 0u);
   for (int j = tid; j < kGN; j += 256) {
-    c_beta[j] = j < kGD ? beta[h * kGD + j] : 0.f;
+    c_beta[j] = j < kGD ? beta[h * kVD + jo + j] : 0.f;
     c_anc[j] = INFINITY;
     c_mu[j] = -INFINITY;
     c_lam[j] = 0.f;
@@ -199,7 +203,7 @@ __global__ void __launch_bounds__(256, 1)
         const int rr = i >> 4, cc = (i & 15) * 4;
         *reinterpret_cast<float4 *>(q32 + rr * kGM + cc) = make_float4(0.f, 0.f, 0.f, 0.f);
         *reinterpret_cast<float4 *>(k32 + rr * kGM + cc) = make_float4(0.f, 0.f, 0.f, 0.f);
-        *reinterpret_cast<float4 *>(v32 + rr * kGD + cc) = make_float4(0.f, 0.f, 0.f, 0.f);
+        *reinterpret_cast<float4 *>(v32 + rr * kVD + cc) = make_float4(0.f, 0.f, 0.f, 0.f);
       }
     }
     // ---- gamma_t = g_0 + ... + g_t over the chunk (warps 0-3, one step each)
@@ -229,10 +233,10 @@ __global__ void __launch_bounds__(256, 1)
       st_bf16x8(smem + GLay::kK16 + sw128_offset(rr, ch), k32 + rr * kGM + ch * 8, 1.f);
     }
     {
-      const int j = tid & 63, qtr = tid >> 6;
+      const int j = tid % kGD, qtr = tid / kGD;
       float mx = -INFINITY, mn = INFINITY, sm = 0.f;
-      for (int i = qtr * 32; i < min(qtr * 32 + 32, rows); ++i) {
-        const float x = v32[i * kGD + j];
+      for (int i = qtr * kKg; i < min(qtr * kKg + kKg, rows); ++i) {
+        const float x = v32[i * kVD + jo + j];
         mx = fmaxf(mx, x);
         mn = fminf(mn, x);
         sm += x;
@@ -256,8 +260,13 @@ __global__ void __launch_bounds__(256, 1)
     if (tid < kGD) {
       const int j = tid;
       const float b = c_beta[j];
-      const float mx = fmaxf(fmaxf(pmax[j], pmax[kGD + j]), fmaxf(pmax[2 * kGD + j], pmax[3 * kGD + j]));
-      const float mn = fminf(fminf(pmin[j], pmin[kGD + j]), fminf(pmin[2 * kGD + j], pmin[3 * kGD + j]));
+      float mx = pmax[j], mn = pmin[j], sm = psum[j];
+#pragma unroll
+      for (int g = 1; g < kQtr; ++g) {
+        mx = fmaxf(mx, pmax[g * kGD + j]);
+        mn = fminf(mn, pmin[g * kGD + j]);
+        sm += psum[g * kGD + j];
+      }
       if (b >= kGlaLinBeta) {
         c_lam[j] = b * mx;
         pmax[j] = 1.f;  // no move of the state (see below)
@@ -266,7 +275,7 @@ __global__ void __launch_bounds__(256, 1)
         // the anchor: the mean of the values so far, at most 1/beta above their minimum (so that
         // 1 + beta num / Z >= 1/e); the state moves with it (either way)
         const float rmin = fminf(c_rmin[j], mn);
-        const float rsum = c_rsum[j] + ((psum[j] + psum[kGD + j]) + (psum[2 * kGD + j] + psum[3 * kGD + j]));
+        const float rsum = c_rsum[j] + sm;
         c_rmin[j] = rmin;
         c_rsum[j] = rsum;
         const float mean = rsum / static_cast<float>(c * kGC + rows);
@@ -285,24 +294,24 @@ __global__ void __launch_bounds__(256, 1)
     }
     __syncthreads();
     for (int i = tid; i < kGD * kGM; i += 256) {
-      const int j = i >> 6, f = i & 63;
+      const int j = i / kGM, f = i % kGM;
       const float e = pmax[j], w = pmin[j];
       if (e != 1.f || w != 0.f) Sf[i] = fmaf(e, Sf[i], w * Sf[kGD * kGM + f]);
     }
     __syncthreads();
     // the chunk's bank (channels x keys, K-major) and the state's bf16 copy (channels x features)
     {
-      const int j = tid & 63, qtr = tid >> 6;
+      const int j = tid % kGD, qtr = tid / kGD;
       const float b = c_beta[j];
       const bool lin = b < kGlaLinBeta;
       const float sh = lin ? c_anc[j] : c_lam[j], rb = c_rb[j];
 #pragma unroll 1
-      for (int kc = qtr * 4; kc < qtr * 4 + 4; ++kc) {
+      for (int kc = qtr * (kKg / 8); kc < (qtr + 1) * (kKg / 8); ++kc) {
         float e[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
           const int i = kc * 8 + u;
-          const float x = v32[i * kGD + j];
+          const float x = v32[i * kVD + jo + j];
           float val;
           if (lin) val = em1_beta_fast(x - sh, b * (x - sh), rb);
           else val = __expf(b * x - sh);
@@ -378,8 +387,8 @@ __global__ void __launch_bounds__(256, 1)
                    kk > 0 ? 1u : 0u);
       mma_commit(bar_a);
     }
-    // ---- the outputs (thread = row of its warp's lane quarter; warps 4-7 take channels 0..31,
-    // warps 0-3 channels 32..63) and then the state (warps 0, 1, 4, 5, thread = feature)
+    // ---- the outputs (thread = row of its warp's lane quarter; warps 4-7 take the CTA's channels
+    // 0..15, warps 0-3 channels 16..31) and then the state (warps 0, 1, 4, 5, thread = feature)
     const bool state_warp = (warp & 3) < 2;
     ok = __all_sync(0xffffffffu, mbar_wait(bar_a, par, err, kErrWaitMma));
     if (ok) {
@@ -389,20 +398,18 @@ __global__ void __launch_bounds__(256, 1)
       const float zi = __uint_as_float(tmem_ld1(tmem + kColIntra + lane_off + kGD));
       const float zx = __uint_as_float(tmem_ld1(tmem + kColInter + lane_off + kGD));
       uint32_t ai[32], ax[32];
-      tmem_ld32(tmem + kColIntra + lane_off + q * 32, ai);
-      tmem_ld32(tmem + kColInter + lane_off + q * 32, ax);
+      tmem_ld32(tmem + kColIntra + lane_off, ai);
+      tmem_ld32(tmem + kColInter + lane_off, ax);
       tmem_ld_wait();
       const float Z = fmaf(et, zx, zi), lz = __logf(Z), rZ = 1.f / Z;
-      if (q == 0 && t < rows && logz) logz[r0 + t] = lz;
+      if (q == 0 && blockIdx.y == 0 && t < rows && logz) logz[r0 + t] = lz;
       // shifted channels whose in-chunk sum fell below 2^-100 of the row's in-chunk prior mass:
       // the chunk's shift may lie far above every key the row sees (the largest value came
       // later in the chunk), so terms under fp32's range may carry the sum; recomputed below
       unsigned flag = 0;
-      float o[32];
-#pragma unroll
-      for (int u = 0; u < 32; ++u) {
-        const int j = q * 32 + u;
-        const float b = c_beta[j], rb = c_rb[j], in = __uint_as_float(ai[u]), ix = __uint_as_float(ax[u]);
+      float o[16];
+      auto read = [&](int j, float in, float ix) {  // j: the CTA's channel
+        const float b = c_beta[j], rb = c_rb[j];
         // both forms, then a select (the form is the channel's; no branch per element)
         const bool lin = b < kGlaLinBeta;
         const float num = fmaf(et, ix, in), x = b * num * rZ;
@@ -411,13 +418,20 @@ __global__ void __launch_bounds__(256, 1)
         const float lb = ix > 0.f ? c_mu[j] + gt + __logf(ix) : -INFINITY;
         const float hi = fmaxf(la, lb), lo = fminf(la, lb);
         const float ln = hi == -INFINITY ? -INFINITY : hi + __logf(1.f + __expf(lo - hi));
-        o[u] = lin ? o_lin : (ln - lz) * rb;
-        flag |= (!lin && !(in >= 0x1p-100f * zi)) ? 1u << u : 0u;
+        flag |= (!lin && !(in >= 0x1p-100f * zi)) ? 1u << j : 0u;
+        return lin ? o_lin : (ln - lz) * rb;
+      };
+      if (q == 0) {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) o[u] = read(u, __uint_as_float(ai[u]), __uint_as_float(ax[u]));
+      } else {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) o[u] = read(16 + u, __uint_as_float(ai[16 + u]), __uint_as_float(ax[16 + u]));
       }
       if (t < rows) {
-        float *orow = out + (r0 + t) * kGD + q * 32;
+        float *orow = out + (r0 + t) * kVD + jo + q * 16;
 #pragma unroll
-        for (int u = 0; u < 32; u += 4) *reinterpret_cast<float4 *>(orow + u) = make_float4(o[u], o[u + 1], o[u + 2], o[u + 3]);
+        for (int u = 0; u < 16; u += 4) *reinterpret_cast<float4 *>(orow + u) = make_float4(o[u], o[u + 1], o[u + 2], o[u + 3]);
       }
       // the flagged entries exactly: the row's fp32 scores (still in TMEM) and the chunk's values,
       // one pass over the visible keys with the running maximum of beta v as the shift
@@ -428,15 +442,15 @@ __global__ void __launch_bounds__(256, 1)
         tmem_ld_wait();
         unsigned fm = t < rows ? flag : 0u;
         while (fm) {
-          const int j = q * 32 + __ffs(fm) - 1;
+          const int j = __ffs(fm) - 1;  // the CTA's channel
           fm &= fm - 1;
           const float b = c_beta[j];
-          const float *vcol = v + r0 * kGD + j;
+          const float *vcol = v + r0 * kVD + jo + j;
           float m = -INFINITY, acc = 0.f;
 #pragma unroll
           for (int i = 0; i < kGC; ++i) {
             if (i <= t) {
-              const float x = b * __ldg(vcol + static_cast<size_t>(i) * kGD);
+              const float x = b * __ldg(vcol + static_cast<size_t>(i) * kVD);
               const float a = __uint_as_float(sr[i >> 5][i & 31]) * expf(gt - gam[i]);
               if (x > m) {
                 acc = fmaf(acc, expf(m - x), a);
@@ -455,14 +469,14 @@ __global__ void __launch_bounds__(256, 1)
           const float lb = ix > 0.f ? c_mu[j] + gt + logf(ix) : -INFINITY;
           const float hi = fmaxf(la, lb), lo = fminf(la, lb);
           const float ln = hi == -INFINITY ? -INFINITY : hi + log1pf(expf(lo - hi));
-          out[(r0 + t) * kGD + j] = (ln - lz) / b;
+          out[(r0 + t) * kVD + jo + j] = (ln - lz) / b;
         }
       }
     }
     __syncthreads();  // the exact entries read the state before its update
     if (ok && state_warp) {
-      // feature f = the warp's TMEM lane; warps 0, 1 take channels 0..39 (columns 0..63
-      // loaded), warps 4, 5 channels 40..79 (columns 32..95 loaded)
+      // feature f = the warp's TMEM lane; warps 0, 1 take channels 0 .. kGN/2 - 1, warps 4, 5
+      // the rest (columns 0..63 loaded)
       const int f = (warp & 1) * 32 + lane;
       const float eg = __expf(glast);
       uint32_t uu[2][32];
@@ -476,18 +490,15 @@ __global__ void __launch_bounds__(256, 1)
           st = fmaf(__expf(mo + glast - mn), st, __expf(lam - mn) * uv);
         }
       };
+      tmem_ld32(tmem + kColU + lane_off, uu[0]);
+      tmem_ld32(tmem + kColU + lane_off + 32, uu[1]);
+      tmem_ld_wait();
       if (warp < 4) {
-        tmem_ld32(tmem + kColU + lane_off, uu[0]);
-        tmem_ld32(tmem + kColU + lane_off + 32, uu[1]);
-        tmem_ld_wait();
 #pragma unroll
-        for (int u = 0; u < 40; ++u) update(u, __uint_as_float(uu[u >> 5][u & 31]));
+        for (int u = 0; u < kGN / 2; ++u) update(u, __uint_as_float(uu[u >> 5][u & 31]));
       } else {
-        tmem_ld32(tmem + kColU + lane_off + 32, uu[0]);
-        tmem_ld32(tmem + kColU + lane_off + 64, uu[1]);
-        tmem_ld_wait();
 #pragma unroll
-        for (int u = 0; u < 40; ++u) update(40 + u, __uint_as_float(uu[(u + 8) >> 5][(u + 8) & 31]));
+        for (int u = kGN / 2; u < kGN; ++u) update(u, __uint_as_float(uu[u >> 5][u & 31]));
       }
     }
     tc_fence_before_sync();
@@ -509,7 +520,8 @@ cudaError_t launch_gla_tc(const float *qf, const float *kf, const float *v, cons
                           float *out, float *logz, int B, int H, int T, unsigned *err, cudaStream_t stream) {
   cudaError_t e = cudaFuncSetAttribute(gla_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, GLay::kAlloc);
   if (e != cudaSuccess) return e;
-  gla_tc_kernel<<<B * H, 256, GLay::kAlloc, stream>>>(qf, kf, v, logdecay, beta, out, logz, H, T, err);
+  gla_tc_kernel<<<dim3(B * H, kVD / kGD), 256, GLay::kAlloc, stream>>>(qf, kf, v, logdecay, beta, out, logz, H, T,
+                                                                      err);
   return cudaGetLastError();
 }
 
