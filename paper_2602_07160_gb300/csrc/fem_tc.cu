@@ -48,7 +48,7 @@
 //
 // TMEM (512 columns): score buffers [0,128) [128,256) [256,384), acc
 // [384, 384 + D); the diagonal tile's P E goes to score buffer nk mod 3.
-// Shared memory: Q, K[3], E[2] tiles of [128 x D] 16-bit
+// Shared memory: Q, K[kStagesK], E[kSlotsE] tiles of [128 x D] 16-bit
 // elements in the 128-byte-swizzle layout TMA writes (64-element column
 // blocks of 128 rows x 128 bytes, chunk c of row r at chunk c ^ (r & 7)),
 // then barriers and per-channel state.  Every mbarrier completes once per use
@@ -67,8 +67,11 @@ struct TcLayout {
   static constexpr uint32_t kTile = D * 128 * 2;
   // 512 TMEM columns: kBufS score buffers of 128 and kNB * D accumulator columns
   static constexpr int kBufS = (GATED && D == 128) ? 2 : 3;
-  static constexpr int kStagesK = (GATED && D == 128) ? 2 : 3;
-  static constexpr int kSlotsE = GATED ? (D == 128 ? 3 : 6) : 2;  // one bank tile per slot
+  // at d = 128 the bank ring takes the third 32 KB slot: the score contractions run up to two key
+  // tiles ahead of the P E, so a bank tile is needed later than its K tile and waits on its load
+  // more often (three K stages and two bank slots ran 0.5 % slower per step)
+  static constexpr int kStagesK = D == 128 ? 2 : 3;
+  static constexpr int kSlotsE = GATED ? (D == 128 ? 3 : 6) : (D == 128 ? 3 : 2);  // one bank tile per slot
   static constexpr uint32_t kQ = 0;
   static constexpr uint32_t kK = kTile;                    // K stages
   static constexpr uint32_t kE = kK + kStagesK * kTile;    // E slots
