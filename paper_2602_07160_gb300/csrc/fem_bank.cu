@@ -1,7 +1,7 @@
 // Value-bank pre-pass of the FEM read: statistics, shift schedule and the
 // fp16 value bank, written once per key tile for every query tile to share.
 //
-//   tile_stats  (persistent)       max, min and sum of v_.j over each tile of
+//   tile_stats  (block per tile)   max, min and sum of v_.j over each tile of
 //                                  128 keys (valid keys only)
 //   plan        (B*H x 32-channel  per channel: bank mode and linear anchor
 //                groups)           from the whole sequence; the running maximum
@@ -28,10 +28,11 @@ namespace fem {
 
 constexpr float kBankFastBeta = 1.f / 64.f;  // linear bank: (e^y - 1)/beta from here on
 
-// Ring of key tiles a persistent pre-pass block streams through shared
-// memory: kStages slots, one mbarrier each, filled by bulk copies that thread 0
-// issues kStages - 1 tiles ahead.  A block takes the tiles blockIdx.x,
-// blockIdx.x + gridDim.x, ... of the (b, h, key tile) list, key tile fastest.
+// Ring of key tiles a persistent bank block streams through shared memory:
+// kStages slots, one mbarrier each, filled by copies that thread 0 issues
+// kStages - 1 tiles ahead.  A block takes tiles_of_block() tiles, the i-th of
+// them number blockIdx.x + i gridDim.x of the (b, h, key tile) list (key tile
+// fastest), counted from its start or from its end.
 constexpr int kStages = 3;
 
 __device__ __forceinline__ int tiles_of_block(int n_tiles) {
@@ -39,119 +40,88 @@ __device__ __forceinline__ int tiles_of_block(int n_tiles) {
 }
 
 // ---------------------------------------------------------------------------
-// tile_stats: 128 threads; thread (cc, rg) reads 16-byte chunk cc of rows
-// rg*RPG .. rg*RPG + RPG - 1 of the tile (consecutive lanes read consecutive
-// chunks of a row), lanes holding the same chunk combine by shuffles, the four
-// warps through shared memory.  Tiles arrive as plain bulk copies of their
-// rows, which are contiguous in V.
+// tile_stats: one 128-thread block per key tile; thread (cc, rg) loads 16-byte
+// chunk cc of rows rg*RPG .. rg*RPG + RPG - 1 straight from V, all RPG loads in
+// flight at once (consecutive lanes read consecutive chunks of a row), lanes
+// holding the same chunk combine by shuffles, the four warps through shared
+// memory.  Short blocks, many resident per SM: the loads of several tiles per
+// SM are in flight together.
 // ---------------------------------------------------------------------------
 template <int D>
 struct StatsMap {
   static constexpr int CPR = D / 8;        // chunks per row
   static constexpr int RG = 128 / CPR;     // row groups
   static constexpr int RPG = 128 / RG;     // rows per group
-  static constexpr int kTileBytes = kBlockK * D * 2;
 };
 
 template <int D>
-__device__ __forceinline__ void stats_issue(const __nv_bfloat16 *v, int T, int n_kt, int g, uint32_t dst,
-                                            uint32_t bar) {
-  const int bh = g / n_kt, kt = g % n_kt;
-  const uint32_t bytes = static_cast<uint32_t>(min(kBlockK, T - kt * kBlockK) * D * 2);
-  mbar_arrive_expect_tx(bar, bytes);
-  bulk_load(dst, v + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D, bytes, bar);
-}
-
-template <int D>
 __global__ void __launch_bounds__(128) tile_stats_kernel(const __nv_bfloat16 *__restrict__ v, int T, int n_kt,
-                                                          int n_tiles, float4 *__restrict__ tstat,
-                                                          unsigned *__restrict__ err) {
+                                                          float4 *__restrict__ tstat) {
   using M = StatsMap<D>;
-  extern __shared__ __align__(16) uint8_t ring[];  // kStages x [128][D] bf16
-  __shared__ __align__(8) uint64_t s_full[kStages];
-  __shared__ float s_part[2][3][4][D];  // [buffer][max, min, sum][warp][channel]
+  __shared__ float s_part[3][4][D];  // [max, min, sum][warp][channel]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int cc = tid % M::CPR, rg = tid / M::CPR;
-  const int my_n = tiles_of_block(n_tiles);
-  if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&s_full[s]), 1);
-    fence_mbar_init();
-    for (int i = 0; i < kStages && i < my_n; ++i)
-      stats_issue<D>(v, T, n_kt, blockIdx.x + i * gridDim.x, smem_u32(ring + i * M::kTileBytes),
-                     smem_u32(&s_full[i]));
-  }
-  __syncthreads();
-  for (int i = 0; i < my_n; ++i) {
-    const int st = i % kStages, g = blockIdx.x + i * gridDim.x;
-    const int bh = g / n_kt, kt = g % n_kt, rows = min(kBlockK, T - kt * kBlockK);
-    if (!mbar_wait(smem_u32(&s_full[st]), (i / kStages) & 1, err, kErrWaitTma)) return;
-    const uint8_t *tile = ring + st * M::kTileBytes;
-    // the thread's rows into registers, then the slot goes back to the copy engine
-    // before the reductions (rows past T are not read)
-    uint4 rawv[M::RPG];
+  const int g = static_cast<int>(blockIdx.x), bh = g / n_kt, kt = g % n_kt;
+  const int rows = min(kBlockK, T - kt * kBlockK);
+  const uint4 *src = reinterpret_cast<const uint4 *>(v + (static_cast<size_t>(bh) * T + static_cast<size_t>(kt) * kBlockK) * D);
+  uint4 rawv[M::RPG];
 #pragma unroll
-    for (int r = 0; r < M::RPG; ++r) {
-      const int row = rg * M::RPG + r;
-      rawv[r] = row < rows ? *reinterpret_cast<const uint4 *>(tile + (row * D + cc * 8) * 2) : make_uint4(0u, 0u, 0u, 0u);
+  for (int r = 0; r < M::RPG; ++r) {
+    const int row = rg * M::RPG + r;
+    rawv[r] = row < rows ? __ldg(src + row * M::CPR + cc) : make_uint4(0u, 0u, 0u, 0u);
+  }
+  float mx[8], mn[8], sm[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    mx[u] = -INFINITY;
+    mn[u] = INFINITY;
+    sm[u] = 0.f;
+  }
+#pragma unroll
+  for (int r = 0; r < M::RPG; ++r) {
+    const int row = rg * M::RPG + r;
+    if (row < rows) {
+      const uint4 raw = rawv[r];
+      const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float2 f = __bfloat1622float2(p2[u]);
+        mx[2 * u] = fmaxf(mx[2 * u], f.x);
+        mx[2 * u + 1] = fmaxf(mx[2 * u + 1], f.y);
+        mn[2 * u] = fminf(mn[2 * u], f.x);
+        mn[2 * u + 1] = fminf(mn[2 * u + 1], f.y);
+        sm[2 * u] += f.x;
+        sm[2 * u + 1] += f.y;
+      }
     }
-    __syncthreads();  // every read of the slot is done
-    if (tid == 0 && i + kStages < my_n)
-      stats_issue<D>(v, T, n_kt, blockIdx.x + (i + kStages) * gridDim.x, smem_u32(ring + st * M::kTileBytes),
-                     smem_u32(&s_full[st]));
-    float mx[8], mn[8], sm[8];
+  }
+#pragma unroll
+  for (int off = M::CPR; off < 32; off <<= 1) {
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      mx[u] = -INFINITY;
-      mn[u] = INFINITY;
-      sm[u] = 0.f;
+      mx[u] = fmaxf(mx[u], __shfl_xor_sync(0xffffffffu, mx[u], off));
+      mn[u] = fminf(mn[u], __shfl_xor_sync(0xffffffffu, mn[u], off));
+      sm[u] += __shfl_xor_sync(0xffffffffu, sm[u], off);
     }
+  }
+  if (lane < M::CPR) {
 #pragma unroll
-    for (int r = 0; r < M::RPG; ++r) {
-      const int row = rg * M::RPG + r;
-      if (row < rows) {
-        const uint4 raw = rawv[r];
-        const __nv_bfloat162 *p2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const float2 f = __bfloat1622float2(p2[u]);
-          mx[2 * u] = fmaxf(mx[2 * u], f.x);
-          mx[2 * u + 1] = fmaxf(mx[2 * u + 1], f.y);
-          mn[2 * u] = fminf(mn[2 * u], f.x);
-          mn[2 * u + 1] = fminf(mn[2 * u + 1], f.y);
-          sm[2 * u] += f.x;
-          sm[2 * u + 1] += f.y;
-        }
-      }
+    for (int u = 0; u < 8; ++u) {
+      s_part[0][warp][cc * 8 + u] = mx[u];
+      s_part[1][warp][cc * 8 + u] = mn[u];
+      s_part[2][warp][cc * 8 + u] = sm[u];
     }
+  }
+  __syncthreads();  // every partial of the tile is written
+  for (int j = tid; j < D; j += 128) {
+    float a = s_part[0][0][j], b = s_part[1][0][j], c = s_part[2][0][j];
 #pragma unroll
-    for (int off = M::CPR; off < 32; off <<= 1) {
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        mx[u] = fmaxf(mx[u], __shfl_xor_sync(0xffffffffu, mx[u], off));
-        mn[u] = fminf(mn[u], __shfl_xor_sync(0xffffffffu, mn[u], off));
-        sm[u] += __shfl_xor_sync(0xffffffffu, sm[u], off);
-      }
+    for (int w = 1; w < 4; ++w) {
+      a = fmaxf(a, s_part[0][w][j]);
+      b = fminf(b, s_part[1][w][j]);
+      c += s_part[2][w][j];
     }
-    const int buf = i & 1;
-    if (lane < M::CPR) {
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        s_part[buf][0][warp][cc * 8 + u] = mx[u];
-        s_part[buf][1][warp][cc * 8 + u] = mn[u];
-        s_part[buf][2][warp][cc * 8 + u] = sm[u];
-      }
-    }
-    __syncthreads();  // every partial of this tile is written
-    for (int j = tid; j < D; j += 128) {
-      float a = s_part[buf][0][0][j], b = s_part[buf][1][0][j], c = s_part[buf][2][0][j];
-#pragma unroll
-      for (int w = 1; w < 4; ++w) {
-        a = fmaxf(a, s_part[buf][0][w][j]);
-        b = fminf(b, s_part[buf][1][w][j]);
-        c += s_part[buf][2][w][j];
-      }
-      tstat[(static_cast<size_t>(bh) * n_kt + kt) * D + j] = make_float4(a, b, c, 0.f);
-    }
+    tstat[static_cast<size_t>(g) * D + j] = make_float4(a, b, c, 0.f);
   }
 }
 
@@ -327,7 +297,7 @@ template <int D>
 __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CUtensorMap tv,
                                                        const __grid_constant__ CUtensorMap te,
                                                        const float4 *__restrict__ bcoef, int T, int n_kt,
-                                                       int n_tiles, float *__restrict__ colsum,
+                                                       int n_tiles, int reverse, float *__restrict__ colsum,
                                                        unsigned *__restrict__ err) {
   using M = BankMap<D>;
   extern __shared__ uint8_t bank_smem[];
@@ -336,16 +306,22 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
   uint8_t *const ring = bank_smem + (base_addr - smem_u32(bank_smem));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int my_n = tiles_of_block(n_tiles);
+  // reverse: the tiles from the end of the list, for a V larger than L2 -- the last tiles the
+  // statistics pass read are still in L2 when this pass starts, and the bank tiles written last
+  // (the first heads) are the first the read kernel wants
+  auto tile_of = [&](int i) {
+    const int x = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
+    return reverse ? n_tiles - 1 - x : x;
+  };
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&s_full[s]), 1);
     fence_mbar_init();
     for (int i = 0; i < kStages - 1 && i < my_n; ++i)
-      bank_issue<D>(&tv, bcoef, n_kt, blockIdx.x + i * gridDim.x, base_addr + i * M::kSlotBytes,
-                    smem_u32(&s_full[i]));
+      bank_issue<D>(&tv, bcoef, n_kt, tile_of(i), base_addr + i * M::kSlotBytes, smem_u32(&s_full[i]));
   }
   __syncthreads();
   for (int i = 0; i < my_n; ++i) {
-    const int st = i % kStages, g = blockIdx.x + i * gridDim.x;
+    const int st = i % kStages, g = tile_of(i);
     const int bh = g / n_kt, kt = g % n_kt, rows = min(kBlockK, T - kt * kBlockK);
     if (!mbar_wait(smem_u32(&s_full[st]), (i / kStages) & 1, err, kErrWaitTma)) {
       if (tid == 0) bulk_wait_group_read0();
@@ -452,8 +428,8 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
       bulk_wait_group_read<1>();
       if (i + kStages - 1 < my_n) {
         const int sn = (i + kStages - 1) % kStages;
-        bank_issue<D>(&tv, bcoef, n_kt, blockIdx.x + (i + kStages - 1) * gridDim.x,
-                      base_addr + sn * M::kSlotBytes, smem_u32(&s_full[sn]));
+        bank_issue<D>(&tv, bcoef, n_kt, tile_of(i + kStages - 1), base_addr + sn * M::kSlotBytes,
+                      smem_u32(&s_full[sn]));
       }
     }
   }
@@ -466,33 +442,28 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
   const int n_kt = (T + kBlockK - 1) / kBlockK, n_tiles = BH * n_kt;
   const __nv_bfloat16 *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = min(n_tiles, 2 * num_sms);
+  // V larger than half of L2: the bank pass walks the tiles backwards (measured at B4 H16 T8192
+  // d128: 0.7 % per step; at 25 MB, where V stays in L2, forward was 0.5 % faster)
+  const int reverse = static_cast<size_t>(n_tiles) * kBlockK * d * 2 > (size_t{64} << 20) ? 1 : 0;
   cudaError_t e = cudaSuccess;
   if (d == 64) {
-    using SM = StatsMap<64>;
     using BM = BankMap<64>;
-    e = cudaFuncSetAttribute(tile_stats_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kStages * SM::kTileBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(bank_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
+    e = cudaFuncSetAttribute(bank_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
     if (e != cudaSuccess) return e;
     if (!stats_ready)
-      tile_stats_kernel<64><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
+      tile_stats_kernel<64><<<n_tiles, 128, 0, stream>>>(vb, T, n_kt, w.tstat);
     plan_kernel<64><<<dim3(BH, 2), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.shift, w.rfac, w.colmask,
                                                      w.bcoef);
-    bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, w.colsum, err);
+    bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, reverse, w.colsum, err);
   } else if (d == 128) {
-    using SM = StatsMap<128>;
     using BM = BankMap<128>;
-    e = cudaFuncSetAttribute(tile_stats_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kStages * SM::kTileBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(bank_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
+    e = cudaFuncSetAttribute(bank_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
     if (e != cudaSuccess) return e;
     if (!stats_ready)
-      tile_stats_kernel<128><<<grid, 128, kStages * SM::kTileBytes, stream>>>(vb, T, n_kt, n_tiles, w.tstat, err);
+      tile_stats_kernel<128><<<n_tiles, 128, 0, stream>>>(vb, T, n_kt, w.tstat);
     plan_kernel<128><<<dim3(BH, 4), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.shift, w.rfac, w.colmask,
                                                       w.bcoef);
-    bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, w.colsum, err);
+    bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, reverse, w.colsum, err);
   } else {
     return cudaErrorInvalidValue;
   }

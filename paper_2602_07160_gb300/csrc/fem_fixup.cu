@@ -28,7 +28,8 @@
 //
 // Entries come in chunks of kFixChunk = 8 rows of one query tile with the
 // same kt0 (the tensor-core kernel pads each block to a multiple of 8 with
-// rows -1).  One 256-thread block (two per SM) takes a chunk at a time,
+// rows -1).  One 256-thread block (three per SM at d = 128, four at d = 64, their
+// register budgets set for it) takes a chunk at a time,
 // claimed from a counter (the next claim already in flight while the current
 // chunk runs) so that blocks that drew cheap chunks take more of them, and
 // walks its key tiles: it stages the chunk's query rows and the tile's K and V
@@ -136,7 +137,7 @@ __device__ __forceinline__ void fold_tile(float &c, float &A, float &W, float L,
 }
 
 template <int D>
-__global__ void __launch_bounds__(kFixThreads) fixup_kernel(const __nv_bfloat16 *__restrict__ q,
+__global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(const __nv_bfloat16 *__restrict__ q,
                                                             const __nv_bfloat16 *__restrict__ k,
                                                             const __nv_bfloat16 *__restrict__ v,
                                                             const float *__restrict__ beta,
@@ -402,7 +403,7 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
   const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr, nullptr};
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
-  const int grid = num_sms * 3;
+  const int grid = num_sms * (d == 64 ? 4 : 3);
   if (d == 64) {
     const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
     fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, chan, shift, out, H, T, causal, entries,
@@ -411,7 +412,7 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
     const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
     cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
-    // two blocks per SM need the largest shared-memory carveout
+    // three blocks per SM need the largest shared-memory carveout
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                cudaSharedmemCarveoutMaxShared);
