@@ -13,9 +13,11 @@ host-buffer C-ABI call (copies included), the float64 oracle timed on a
 bounded sample on the host cores, and the SM clocks seen during the timed
 region.  ``--impl reference`` times the oracle itself, as the reference arm.
 
-Under torchrun (N > 1) every rank reads its own copy of the workload (weak
-scaling, no collective on the data path); the step time is the maximum over
-ranks.
+Under torchrun (N > 1) the ranks share one global batch of N x B sequences
+(data parallel over the batch, weak scaling): rank r reads sequences r B ..
+r B + B - 1 (``workloads.make_batch_shard``), the read being independent per
+(b, h), so no collective is on the data path; the step time is the maximum
+over ranks.
 """
 from __future__ import annotations
 
@@ -45,11 +47,12 @@ TC_SOURCE = os.path.join(ROOT, "paper_2602_07160_gb300", "csrc", "fem_tc.cu")
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
-    ap.add_argument("--warmup", type=int, default=5)
+    # 1000 steps: about a second of timed work at the headline, so the clock sampler sees it
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["fem", "reference"], default="fem")
     ap.add_argument("--workload", default="lm_causal_d128")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=50)
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle CPU-baseline budget")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -254,7 +257,8 @@ def run_reference(args):
     w = W.WORKLOADS[args.workload]
     q, k, v, beta = W.make_inputs(w)
     s = OracleSampler(w, q, k, v, beta)
-    step_s = max(0.5, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
+    # the whole run about 150 s of oracle time, at least 50 ms per step
+    step_s = max(0.05, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
     n = s.rows_for_seconds(step_s)
     for _ in range(args.warmup):
         s.run(s.rows(n))
@@ -375,7 +379,8 @@ def run_fem(args):
         w = dataclasses.replace(w, B=B_, H=H_, T=T_, name=f"{w.name}@B{B_}H{H_}T{T_}")
     if w.dtype != "bf16":
         raise SystemExit("bench times the bf16 tensor-core read; pick a bf16 workload")
-    q, k, v, beta = W.make_inputs(w, seed=rank)  # sizes come from w (overridable with --shape)
+    # sizes come from w (overridable with --shape); N > 1: this rank's shard of the global batch
+    q, k, v, beta = W.make_inputs(w) if world == 1 else W.make_batch_shard(w, rank, world)
     qd, kd, vd, bd = (x.to(device) for x in (q, k, v, beta))
     out = torch.empty(q.shape, dtype=torch.float32, device=device)
     lse = torch.empty(q.shape[:3], dtype=torch.float32, device=device)
@@ -628,7 +633,8 @@ def run_fem(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
             "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16", "data": "synthetic",
-            "config": dict(w.describe(), pv_operands="fp16", parallelism=f"replicas{world}" if world > 1 else "single",
+            "config": dict(w.describe(), pv_operands="fp16", global_batch=world * w.B,
+                           parallelism=f"dp{world} (batch shards, no exchange)" if world > 1 else "single",
                            l2=f"inputs larger than L2 ({in_bytes / 1e6:.0f} MB of Q/K/V vs 129 MB L2)",
                            parity_sample=parity, fixup_entries=fixup_entries),
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",

@@ -300,6 +300,8 @@ __global__ void __launch_bounds__(256, 2) bank_kernel(const __grid_constant__ CU
                                                        int n_tiles, int reverse, float *__restrict__ colsum,
                                                        unsigned *__restrict__ err) {
   using M = BankMap<D>;
+  // the read kernel, a programmatic dependent launch, may take the SMs this pass's tail leaves
+  grid_dep_launch_dependents();
   extern __shared__ uint8_t bank_smem[];
   __shared__ __align__(8) uint64_t s_full[kStages];
   const uint32_t base_addr = (smem_u32(bank_smem) + 1023u) & ~1023u;  // 128-byte swizzle wants 1024-B alignment
@@ -450,8 +452,7 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
     using BM = BankMap<64>;
     e = cudaFuncSetAttribute(bank_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
     if (e != cudaSuccess) return e;
-    if (!stats_ready)
-      tile_stats_kernel<64><<<n_tiles, 128, 0, stream>>>(vb, T, n_kt, w.tstat);
+    if (!stats_ready) tile_stats_kernel<64><<<n_tiles, 128, 0, stream>>>(vb, T, n_kt, w.tstat);
     plan_kernel<64><<<dim3(BH, 2), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.shift, w.rfac, w.colmask,
                                                      w.bcoef);
     bank_kernel<64><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, reverse, w.colsum, err);
@@ -459,8 +460,7 @@ cudaError_t launch_value_bank(const void *v, const CUtensorMap &tv, const CUtens
     using BM = BankMap<128>;
     e = cudaFuncSetAttribute(bank_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, BM::kSmem);
     if (e != cudaSuccess) return e;
-    if (!stats_ready)
-      tile_stats_kernel<128><<<n_tiles, 128, 0, stream>>>(vb, T, n_kt, w.tstat);
+    if (!stats_ready) tile_stats_kernel<128><<<n_tiles, 128, 0, stream>>>(vb, T, n_kt, w.tstat);
     plan_kernel<128><<<dim3(BH, 4), 128, 0, stream>>>(w.tstat, beta, H, T, n_kt, w.chan, w.shift, w.rfac, w.colmask,
                                                       w.bcoef);
     bank_kernel<128><<<grid, 256, BM::kSmem, stream>>>(tv, te, w.bcoef, T, n_kt, n_tiles, reverse, w.colsum, err);

@@ -153,6 +153,7 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
   // ldmatrix with consecutive rows four banks apart; V rows an odd number of
   // 32-bit words, so one column read across rows is free of bank conflicts
   constexpr int KS = D + 8, VS = D + 2, G = D / 32;
+  grid_dep_wait();  // the entry list and the accumulators the tensor-core kernel left in out
   extern __shared__ __align__(16) uint8_t fix_smem[];
   __nv_bfloat16 *sK = reinterpret_cast<__nv_bfloat16 *>(fix_smem);
   __nv_bfloat16 *sV = sK + kBlockK * KS;
@@ -399,15 +400,16 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const ChanInfo *chan,
                          const float *shift, float *out, int H, int T, int d, int causal, const FixupEntry *entries,
                          const int *count, const int *rows, int *next_chunk, int *last_rows, const TcGate *gate,
-                         int num_sms, cudaStream_t stream) {
+                         int num_sms, cudaStream_t stream, bool pdl) {
   const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr, nullptr};
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = num_sms * (d == 64 ? 4 : 3);
   if (d == 64) {
     const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
-    fixup_kernel<64><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, chan, shift, out, H, T, causal, entries,
-                                                          count, rows, next_chunk, last_rows, g);
+    cudaError_t e = launch_kernel(fixup_kernel<64>, dim3(grid), dim3(kFixThreads), smem, stream, pdl, qb, kb, vb, beta,
+                                  chan, shift, out, H, T, causal, entries, count, rows, next_chunk, last_rows, g);
+    if (e != cudaSuccess) return e;
   } else if (d == 128) {
     const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
     cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -417,8 +419,9 @@ cudaError_t launch_fixup(const void *q, const void *k, const void *v, const floa
       e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
-    fixup_kernel<128><<<grid, kFixThreads, smem, stream>>>(qb, kb, vb, beta, chan, shift, out, H, T, causal, entries,
-                                                           count, rows, next_chunk, last_rows, g);
+    e = launch_kernel(fixup_kernel<128>, dim3(grid), dim3(kFixThreads), smem, stream, pdl, qb, kb, vb, beta, chan, shift,
+                      out, H, T, causal, entries, count, rows, next_chunk, last_rows, g);
+    if (e != cudaSuccess) return e;
   } else {
     return cudaErrorInvalidValue;
   }

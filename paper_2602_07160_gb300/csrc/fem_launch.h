@@ -8,6 +8,25 @@
 
 namespace fem {
 
+// Launches kernel<<<grid, block, smem, stream>>>(args...), with `pdl` as a
+// programmatic dependent launch on the previous kernel of the stream (the
+// kernel then orders itself behind it with grid_dep_wait()).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                                 bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Device workspace of one read (all arrays caller-owned): the value-bank
 // pre-pass's arrays and the exact fix-up's entry list.
 struct BankWorkspace {
@@ -66,9 +85,11 @@ struct TcGate {
 // channels' outputs, their accumulator before that tile.  With te0 (the mean's
 // bank) and gate both given it runs the one-pass gated read; with neither the
 // plain read.
+// pdl: a programmatic dependent launch on the bank kernel before it.
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
                       const CUtensorMap *te0, float *out, const float *beta, const BankWorkspace &w, float *lse,
-                      int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream);
+                      int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream,
+                      bool pdl = false);
 
 // The attention-mode comparator on the same kernel: o = softmax(q k^T / sqrt(d)) v
 // with bf16 P and V on the tensor cores (tv maps V like the bank).
@@ -88,7 +109,7 @@ constexpr int kMaxSeqLen = 8192 * kBlockK;
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const ChanInfo *chan,
                          const float *shift, float *out, int H, int T, int d, int causal, const FixupEntry *entries,
                          const int *count, const int *rows, int *next_chunk, int *last_rows, const TcGate *gate,
-                         int num_sms, cudaStream_t stream);
+                         int num_sms, cudaStream_t stream, bool pdl = false);
 
 
 // Decode read of one query per (b, h) against T cached keys: per-CTA key-chunk

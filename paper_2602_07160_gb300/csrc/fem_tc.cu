@@ -230,10 +230,12 @@ __global__ void __launch_bounds__(384, 1)
   constexpr int kPreK = kStagesK, kPreE = kSlotsE;  // loads the prologue issues (the rings' depths)
   const int ne = nk * kNB;                           // E items
 
+  grid_dep_launch_dependents();
   if (warp == 3) {
     tmem_alloc(sbase + Lay::kTmemSlot, 512);
     tmem_relinquish();
   }
+  grid_dep_wait();  // the value bank, its plan and column sums; the fix-up list's counters
   if (tid == 0) {
     mbar_init(FEM_BAR(kBarQ), 1);
     for (int s = 0; s < kStagesK; ++s) {
@@ -906,7 +908,7 @@ template <int D, bool GATED, bool ATTN = false>
 static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
                                const CUtensorMap &te0, float *out, const float *beta, const BankWorkspace &w,
                                float *lse, int BH, int H, int T, int causal, const TcGate &gate, unsigned *err,
-                               cudaStream_t stream) {
+                               cudaStream_t stream, bool pdl) {
   using Lay = TcLayout<D, GATED>;
   const int n_qt = (T + kBlockQ - 1) / kBlockQ;
   if (n_qt > Lay::kMaxKeyTiles || BH > 65535) return cudaErrorInvalidValue;
@@ -914,25 +916,28 @@ static cudaError_t launch_tc_d(const CUtensorMap &tq, const CUtensorMap &tk, con
   cudaError_t e =
       cudaFuncSetAttribute(fem_tc_kernel<D, GATED, ATTN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const dim3 grid(n_qt, BH);
-  fem_tc_kernel<D, GATED, ATTN>
-      <<<grid, 384, smem, stream>>>(tq, tk, te, te0, out, beta, w, lse, H, T, causal, gate, err);
-  return cudaGetLastError();
+  e = launch_kernel(fem_tc_kernel<D, GATED, ATTN>, dim3(n_qt, BH), dim3(384), smem, stream, pdl, tq, tk, te, te0, out,
+                    beta, w, lse, H, T, causal, gate, err);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_tc(int d, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &te,
                       const CUtensorMap *te0, float *out, const float *beta, const BankWorkspace &w, float *lse,
-                      int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream) {
+                      int BH, int H, int T, int causal, const TcGate *gate, unsigned *err, cudaStream_t stream,
+                      bool pdl) {
   const TcGate none = {nullptr, nullptr, nullptr, nullptr, nullptr};
   if ((te0 != nullptr) != (gate != nullptr)) return cudaErrorInvalidValue;
   if (gate) {
-    if (d == 64) return launch_tc_d<64, true>(tq, tk, te, *te0, out, beta, w, lse, BH, H, T, causal, *gate, err, stream);
+    if (d == 64)
+      return launch_tc_d<64, true>(tq, tk, te, *te0, out, beta, w, lse, BH, H, T, causal, *gate, err, stream, pdl);
     if (d == 128)
-      return launch_tc_d<128, true>(tq, tk, te, *te0, out, beta, w, lse, BH, H, T, causal, *gate, err, stream);
+      return launch_tc_d<128, true>(tq, tk, te, *te0, out, beta, w, lse, BH, H, T, causal, *gate, err, stream, pdl);
     return cudaErrorInvalidValue;
   }
-  if (d == 64) return launch_tc_d<64, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream);
-  if (d == 128) return launch_tc_d<128, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream);
+  if (d == 64)
+    return launch_tc_d<64, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream, pdl);
+  if (d == 128)
+    return launch_tc_d<128, false>(tq, tk, te, te, out, beta, w, lse, BH, H, T, causal, none, err, stream, pdl);
   return cudaErrorInvalidValue;
 }
 
@@ -941,9 +946,11 @@ cudaError_t launch_attn(int d, const CUtensorMap &tq, const CUtensorMap &tk, con
   const TcGate none = {nullptr, nullptr, nullptr, nullptr, nullptr};
   const BankWorkspace w = {};
   if (d == 64)
-    return launch_tc_d<64, false, true>(tq, tk, tv, tv, out, nullptr, w, lse, BH, H, T, causal, none, err, stream);
+    return launch_tc_d<64, false, true>(tq, tk, tv, tv, out, nullptr, w, lse, BH, H, T, causal, none, err, stream,
+                                        false);
   if (d == 128)
-    return launch_tc_d<128, false, true>(tq, tk, tv, tv, out, nullptr, w, lse, BH, H, T, causal, none, err, stream);
+    return launch_tc_d<128, false, true>(tq, tk, tv, tv, out, nullptr, w, lse, BH, H, T, causal, none, err, stream,
+                                         false);
   return cudaErrorInvalidValue;
 }
 

@@ -89,8 +89,14 @@ def make_inputs(w: Workload, seed: int = 0, T: int | None = None, B: int | None 
     B = w.B if B is None else B
     H = w.H if H is None else H
     T = w.T if T is None else T
-    shape = (B, H, T, w.d)
     gen = torch.Generator(device="cpu").manual_seed(seed)
+    q, k, v = _draw_qkv(gen, w, (B, H, T, w.d))
+    beta = _draw_beta(gen, w, H)
+    dt = _dtype(w)
+    return q.to(dt).contiguous(), k.to(dt).contiguous(), v.to(dt).contiguous(), beta.contiguous()
+
+
+def _draw_qkv(gen: torch.Generator, w: Workload, shape):
     q = _normal(gen, shape)
     k = _normal(gen, shape)
     if w.v_dist == "normal":
@@ -101,11 +107,39 @@ def make_inputs(w: Workload, seed: int = 0, T: int | None = None, B: int | None 
         raise ValueError(w.v_dist)
     if w.const_channels:
         c = w.const_channels
-        v[..., :c] = v[:, :, :1, :c]
+        v[..., :c] = v[..., :1, :c]
+    return q, k, v
+
+
+def _draw_beta(gen: torch.Generator, w: Workload, H: int) -> torch.Tensor:
     u = torch.rand((H, w.d), generator=gen, dtype=torch.float64)
-    beta = torch.exp(math.log(w.beta_lo) + u * (math.log(w.beta_hi) - math.log(w.beta_lo))).float()
-    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
-    return q.to(dt).contiguous(), k.to(dt).contiguous(), v.to(dt).contiguous(), beta.contiguous()
+    return torch.exp(math.log(w.beta_lo) + u * (math.log(w.beta_hi) - math.log(w.beta_lo))).float()
+
+
+def _dtype(w: Workload):
+    return torch.bfloat16 if w.dtype == "bf16" else torch.float32
+
+
+def make_batch_shard(w: Workload, rank: int, world: int, seed: int = 0):
+    """Rank ``rank``'s share of one global batch of ``world * w.B`` sequences.
+
+    The read is independent per (b, h), so the global batch shards over the batch
+    dimension with no exchange: rank r holds sequences r*B .. r*B + B - 1, each drawn
+    from its own generator (seeded by ``seed`` and the sequence's global index), and
+    every rank draws the same beta [H, d] (from the generator seeded by ``seed``).  The
+    shards of all ranks, concatenated over the batch, are exactly
+    ``make_batch_shard(w with B = world * w.B, 0, 1, seed)``."""
+    if not 0 <= rank < world:
+        raise ValueError("rank out of range")
+    shape = (1, w.H, w.T, w.d)
+    parts = []
+    for b in range(rank * w.B, (rank + 1) * w.B):
+        gen = torch.Generator(device="cpu").manual_seed((seed * 1_000_003 + 1 + b) % (1 << 63))
+        parts.append(_draw_qkv(gen, w, shape))
+    beta = _draw_beta(torch.Generator(device="cpu").manual_seed(seed), w, w.H)
+    dt = _dtype(w)
+    q, k, v = (torch.cat([p[i] for p in parts]).to(dt).contiguous() for i in range(3))
+    return q, k, v, beta.contiguous()
 
 
 def make_custom(B: int, H: int, T: int, d: int, *, dtype: str = "bf16", beta_lo: float = 0.05,
