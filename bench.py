@@ -49,7 +49,7 @@ def parse_args():
     ap.add_argument("--gpus", type=int, default=1)
     # 1000 steps: about a second of timed work at the headline, so the clock sampler sees it
     ap.add_argument("--steps", type=int, default=1000)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", choices=["fem", "reference"], default="fem")
     ap.add_argument("--workload", default="lm_causal_d128")
     ap.add_argument("--e2e-steps", type=int, default=50)
