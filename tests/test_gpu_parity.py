@@ -118,6 +118,28 @@ def test_deterministic():
     assert np.array_equal(a, b) and np.array_equal(la, lb)
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_timed_launch_matches_dependent_launch(d):
+    """With events around the tensor-core kernel (how bench.py times it) the read and the
+    fix-up are plain launches; without them they are programmatic dependent launches that
+    start in the previous kernel's tail.  Both orders give the same bits, fix-up rows included."""
+    q, k, v, beta = W.make_custom(2, 4, 1000, d, seed=12)
+    dev = torch.device("cuda", 0)
+    qd, kd, vd, bd = (x.to(dev) for x in (q, k, v, beta))
+    o1, l1 = fem.fem_fwd(qd, kd, vd, bd, causal=True)
+    rows1 = fem.last_fixup_rows()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()  # torch creates the CUDA events at their first record
+    e1.record()
+    fem.set_kernel_events(e0, e1)
+    o2, l2 = fem.fem_fwd(qd, kd, vd, bd, causal=True)
+    torch.cuda.synchronize()
+    assert e0.elapsed_time(e1) > 0.0
+    assert rows1 > 0 and fem.last_fixup_rows() == rows1
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    fem.check_device_error()
+
+
 def test_workspace_variant_matches():
     q, k, v, beta = W.make_custom(1, 2, 300, 64, seed=4)
     dev = torch.device("cuda", 0)
