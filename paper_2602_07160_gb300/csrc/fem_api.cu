@@ -120,8 +120,11 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// The counters zeroed before every read: four ints, then the fix-up's split slots.
+constexpr size_t kCountBytes = 256 + kFixPoolSlots * sizeof(FixSlot);
+
 struct WsLayout {
-  size_t tstat, chan, bcoef, shift, rfac, colsum, colmask, bank, fixups, count, total;
+  size_t tstat, chan, bcoef, shift, rfac, colsum, colmask, bank, fixups, count, fixpart, total;
 };
 
 // Head dimensions of the bf16 read that run on CUDA cores (no workspace but the counters).
@@ -157,8 +160,12 @@ bool ws_layout(int B, int H, int T, int d, int causal, WsLayout *w) {
   off += round256(BH * n_kt * 4 * sizeof(unsigned));
   w->fixups = off;
   off += round256(fixup_capacity(BH, static_cast<size_t>(T)) * sizeof(FixupEntry));
-  w->count = off;  // fix-up slots, fix-up rows, the fix-up's chunk counter
-  off += 256;
+  w->count = off;  // fix-up slots, fix-up rows, the fix-up's chunk counter, split chunks; then the split slots
+  off += kCountBytes;
+  w->fixpart = off;
+  if (fix_split_on(static_cast<int>(n_kt)))
+    off += round256(static_cast<size_t>(kFixPoolSlots) * fix_max_segs(static_cast<int>(n_kt)) * kFixChunk *
+                    (2 + 4 * static_cast<size_t>(d)) * sizeof(float));
   w->total = off;
   return true;
 }
@@ -269,6 +276,9 @@ static BankWorkspace bank_workspace(uint8_t *ws, const WsLayout &w) {
   bw.fixup_count = reinterpret_cast<int *>(ws + w.count);
   bw.fixup_rows = reinterpret_cast<int *>(ws + w.count) + 1;
   bw.fixup_next = reinterpret_cast<int *>(ws + w.count) + 2;
+  bw.fix_long = reinterpret_cast<int *>(ws + w.count) + 3;
+  bw.fix_slots = reinterpret_cast<FixSlot *>(ws + w.count + 256);
+  bw.fix_part = w.total > w.fixpart ? reinterpret_cast<float *>(ws + w.fixpart) : nullptr;
   return bw;
 }
 
@@ -315,7 +325,8 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
     gate = TcGate{ga->lam, ga->g, ga->mu_side, bw0.chan, bw0.colsum};
   }
 
-  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, 3 * sizeof(int), s);
+  // the four counters, and the split slots when the fix-up may split
+  cudaError_t e = cudaMemsetAsync(bw.fixup_count, 0, bw.fix_part ? kCountBytes : 4 * sizeof(int), s);
   // the mean's bank (every channel linear at beta = 0: v - c with c the channel mean)
   if (e == cudaSuccess && ga)
     e = launch_value_bank(v, tv, te0, ga->zero_beta, BH, H, T, d, bw0, ds->err, ds->num_sms, s);
@@ -335,7 +346,8 @@ static int fwd_impl(const void *q, const void *k, const void *v, const float *be
   if (e == cudaSuccess && ev1) e = cudaEventRecord(ev1, s);
   if (e == cudaSuccess)
     e = launch_fixup(q, k, v, beta, bw.chan, bw.shift, out, H, T, d, causal, bw.fixups, bw.fixup_count,
-                     bw.fixup_rows, bw.fixup_next, ds->last_fixup, ga ? &gate : nullptr, ds->num_sms, s, pdl);
+                     bw.fixup_rows, bw.fixup_next, ds->last_fixup, ga ? &gate : nullptr, bw.fix_long, bw.fix_slots,
+                     bw.fix_part, ds->num_sms, s, pdl);
   return map_cuda(e);
 }
 

@@ -97,6 +97,31 @@ struct __align__(32) FixupEntry {
   int kt0;
 };
 
+// A fix-up chunk that recomputes its rows from the first key tile over many
+// tiles is split into segments of fix_seg_tiles(n_kt) key tiles that blocks
+// take separately; each leaves its partial state in a pool slot and the last
+// to finish merges them.  At most kFixPoolSlots chunks are split per read
+// (later ones run whole); none when the sequence has fewer than
+// kFixSplitMinTiles key tiles (at 8192 keys the longest such chunks cost no
+// more than the spread of the last claims, and the claims' extra code cost
+// 1 to 2 % of the step).
+constexpr int kFixSegMin = 8;       // key tiles per segment, at least
+constexpr int kFixMaxSeg = 16;      // segments per chunk, at most
+constexpr int kFixPoolSlots = 128;  // chunks split at once
+__host__ __device__ inline int fix_seg_tiles(int n_kt) {
+  const int s = (n_kt + kFixMaxSeg - 1) / kFixMaxSeg;
+  return s > kFixSegMin ? s : kFixSegMin;
+}
+constexpr int kFixSplitMinTiles = 128;
+__host__ __device__ inline bool fix_split_on(int n_kt) { return n_kt >= kFixSplitMinTiles; }
+__host__ __device__ inline int fix_max_segs(int n_kt) { return (n_kt + fix_seg_tiles(n_kt) - 1) / fix_seg_tiles(n_kt); }
+// One split chunk: the chunk, its segment count, the next unclaimed segment,
+// the segments finished, and ready = 1 once the others are written (all zero
+// before the fix-up).
+struct __align__(32) FixSlot {
+  int chunk, n_seg, next, done, ready, pad[3];
+};
+
 // ---------------------------------------------------------------------------
 // Small helpers
 // ---------------------------------------------------------------------------

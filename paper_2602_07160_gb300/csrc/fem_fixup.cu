@@ -40,6 +40,15 @@
 // each listed channel's; a 32-channel group with three or more listed
 // channels is folded with lane = channel instead, walking the keys in turn in
 // one pass.
+//
+// At 128 key tiles or more (SPLIT), a chunk that recomputes its rows from the
+// first key tile over 2 kseg tiles or more (kseg = fix_seg_tiles) is split: the
+// block that draws it registers it in a slot and works through its segments of
+// kseg tiles, other blocks take the remaining segments once the list is
+// exhausted, each segment leaves the rows' partial states (m, L and per listed
+// channel c, A, W, M, all from an empty start) in the slot's pool, and the block
+// that finishes the last segment folds them in key order, each scaled to the
+// common row maximum and shifted like a key tile's sums, and reads the rows out.
 #include "fem_common.cuh"
 #include "fem_launch.h"
 
@@ -136,7 +145,9 @@ __device__ __forceinline__ void fold_tile(float &c, float &A, float &W, float L,
   W += W2;
 }
 
-template <int D>
+// SPLIT: long recomputations go over key-tile segments (part != null); otherwise
+// every chunk runs whole and the kernel carries none of that machinery.
+template <int D, bool SPLIT>
 __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(const __nv_bfloat16 *__restrict__ q,
                                                             const __nv_bfloat16 *__restrict__ k,
                                                             const __nv_bfloat16 *__restrict__ v,
@@ -148,7 +159,9 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
                                                             const int *__restrict__ count,
                                                             const int *__restrict__ rows_listed,
                                                             int *__restrict__ next_chunk,
-                                                            int *__restrict__ last_rows, TcGate gate) {
+                                                            int *__restrict__ last_rows, TcGate gate,
+                                                            int *__restrict__ fix_long, FixSlot *__restrict__ slots,
+                                                            float *__restrict__ part) {
   // staged row strides in bf16 elements: K and Q rows 16-byte aligned for
   // ldmatrix with consecutive rows four banks apart; V rows an odd number of
   // 32-bit words, so one column read across rows is free of bank conflicts
@@ -159,29 +172,128 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
   __nv_bfloat16 *sV = sK + kBlockK * KS;
   __nv_bfloat16 *sQ = sV + kBlockK * VS;  // 16 rows (8 entries, 8 unused) of KS
   __shared__ float sS[kFixChunk][kBlockK];  // the chunk's scores (log2 units), then the tile's P
-  __shared__ int s_ch;
+  __shared__ int s_ch, s_slot, s_seg, s_merge, s_split;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_chunks = *count / kFixChunk;
   if (blockIdx.x == 0 && tid == 0 && last_rows) *last_rows = *rows_listed;
   const float scale = kLog2e * rsqrtf(static_cast<float>(D));
   const int n_kt = (T + kBlockK - 1) / kBlockK;
   const bool gated = gate.lam != nullptr;
+  const int kseg = fix_seg_tiles(n_kt), max_seg = fix_max_segs(n_kt);
+  constexpr int kPart = 2 + 4 * D;  // floats of one row's partial state: m, L, then c, A, W, M per channel
 
-  int claim = 0;  // thread 0: the next chunk, claimed one chunk ahead
+  // warp 0 claims the work; lane 0 keeps the list's next chunk claimed one ahead and the
+  // chunk this block split
+  int claim = n_chunks, my_slot = -1, my_nseg = 0, my_chunk = 0;
   if (tid == 0) claim = atomicAdd(next_chunk, 1);
   for (;;) {
-    if (tid == 0) {
-      s_ch = claim;
-      if (claim < n_chunks) claim = atomicAdd(next_chunk, 1);
+    // the next piece: (1) the next segment of the chunk this block split; (2) the list's
+    // next chunk; (3) once the list is exhausted, a segment of a chunk another block split
+    if (!SPLIT) {
+      if (tid == 0) {
+        s_ch = claim;
+        s_slot = -1;
+        s_seg = 0;
+        if (claim < n_chunks) claim = atomicAdd(next_chunk, 1);
+      }
+    } else if (warp == 0) {
+      int ch = n_chunks, slot = -1, seg = 0;
+      if (lane == 0) {
+        if (my_slot >= 0) {
+          const int sg = atomicAdd(&slots[my_slot].next, 1);
+          if (sg < my_nseg) {
+            ch = my_chunk;
+            slot = my_slot;
+            seg = sg;
+          } else {
+            my_slot = -1;
+          }
+        }
+        if (slot < 0 && claim < n_chunks) {
+          ch = claim;
+          claim = atomicAdd(next_chunk, 1);
+        }
+      }
+      ch = __shfl_sync(0xffffffffu, ch, 0);
+      slot = __shfl_sync(0xffffffffu, slot, 0);
+      seg = __shfl_sync(0xffffffffu, seg, 0);
+      if (slot < 0 && ch >= n_chunks) {
+        // lanes over the slots, 32 at a time; the lowest lane holding one with segments left claims
+        const int nl = min(*reinterpret_cast<volatile int *>(fix_long), kFixPoolSlots);
+        for (int b0 = 0; b0 < nl && slot < 0; b0 += 32) {
+          const int li = b0 + lane;
+          bool cand = false;
+          if (li < nl) {
+            volatile FixSlot *fs = slots + li;
+            if (fs->ready != 0) {
+              __threadfence();  // the slot's fields, written before ready
+              cand = fs->next < fs->n_seg;
+            }
+          }
+          unsigned bal = __ballot_sync(0xffffffffu, cand);
+          while (bal && slot < 0) {
+            const int src = __ffs(bal) - 1;
+            bal &= bal - 1;
+            int got = -1, gch = 0;
+            if (lane == src) {
+              volatile FixSlot *fs = slots + li;
+              const int sg = atomicAdd(&slots[li].next, 1);
+              if (sg < fs->n_seg) {
+                got = sg;
+                gch = fs->chunk;
+              }
+            }
+            got = __shfl_sync(0xffffffffu, got, src);
+            gch = __shfl_sync(0xffffffffu, gch, src);
+            if (got >= 0) {
+              ch = gch;
+              slot = b0 + src;
+              seg = got;
+            }
+          }
+        }
+      }
+      if (lane == 0) {
+        s_ch = ch;
+        s_slot = slot;
+        s_seg = seg;
+      }
     }
     __syncthreads();
     const int ch = s_ch;
+    int slot = SPLIT ? s_slot : -1, seg = SPLIT ? s_seg : 0;
     if (ch >= n_chunks) break;
     const FixupEntry ent = entries[ch * kFixChunk + warp];
     const FixupEntry ent0 = entries[ch * kFixChunk];  // the chunk's first entry is a real row
     const int bh = ent0.row / T, h = bh % H;
     const int qt = (ent0.row % T) / kBlockQ, kt0 = ent0.kt0;
     const int kt_end = causal ? qt : n_kt - 1;
+    if (SPLIT && slot < 0 && kt0 == 0 && kt_end + 1 >= 2 * kseg) {
+      // a recomputation from the first key tile over 2 kseg tiles or more: split into segments
+      // that other blocks may take, this block taking the first (the whole chunk when no slot is free)
+      if (tid == 0) {
+        const int li = atomicAdd(fix_long, 1);
+        int got = -1;
+        if (li < kFixPoolSlots) {
+          FixSlot *fs = slots + li;
+          my_nseg = (kt_end + kseg) / kseg;
+          my_chunk = ch;
+          fs->chunk = ch;
+          fs->n_seg = my_nseg;
+          fs->next = 1;
+          fs->done = 0;
+          __threadfence();
+          atomicExch(&fs->ready, 1);
+          my_slot = got = li;
+        }
+        s_split = got;
+      }
+      __syncthreads();
+      slot = s_split;
+      seg = 0;
+    }
+    // the key tiles of this piece: the whole chunk, or one segment of it
+    const int kt_lo = slot < 0 ? kt0 : seg * kseg, kt_hi = slot < 0 ? kt_end : min(kt_end, kt_lo + kseg - 1);
     const int t = ent.row >= 0 ? ent.row - bh * T : -1;  // this warp's row
     const bool need_mu = gated && kt0 == 0 && ent.l_pre > 0.f;  // the gated read's mean recomputed too
     // the entry's state, lane l holding channels l + 32 g
@@ -229,7 +341,7 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
 #pragma unroll
     for (int off = 16; off; off >>= 1) t_last = max(t_last, __shfl_xor_sync(0xffffffffu, t_last, off));
     t_last -= bh * T;
-    for (int kt = kt0; kt <= kt_end; ++kt) {
+    for (int kt = kt_lo; kt <= kt_hi; ++kt) {
       const int k0 = kt * kBlockK;
       const bool diag = causal && kt == qt;
       // keys k0 .. k0+nk-1 serve every row of the chunk
@@ -372,7 +484,66 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
       }
       __syncthreads();  // the staged rows are rewritten by the next tile or chunk
     }
-    if (t >= 0) {
+    bool read_out = !SPLIT || slot < 0;
+    if (SPLIT && slot >= 0) {
+      // a segment: its partial state to the pool; the last segment to finish merges them all
+      float *pp = part + ((static_cast<size_t>(slot) * max_seg + seg) * kFixChunk + warp) * kPart;
+      if (t >= 0) {
+        if (lane == 0) {
+          pp[0] = m;
+          pp[1] = L;
+        }
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          if (!((ent.mask[g] >> lane) & 1u)) continue;
+          const int j = lane + 32 * g;
+          pp[2 + j] = c_reg[g];
+          pp[2 + D + j] = A_reg[g];
+          pp[2 + 2 * D + j] = W_reg[g];
+          pp[2 + 3 * D + j] = M_reg[g];
+        }
+      }
+      __threadfence();
+      __syncthreads();
+      if (tid == 0) {
+        const int n_seg = reinterpret_cast<volatile FixSlot *>(slots)[slot].n_seg;
+        s_merge = atomicAdd(&slots[slot].done, 1) == n_seg - 1;
+      }
+      __syncthreads();
+      read_out = s_merge != 0;
+      if (read_out && t >= 0) {
+        // every segment's state, in key order, each at its own row maximum and shifts:
+        // scaled to the common maximum and folded like a key tile's sums
+        __threadfence();
+        const int n_seg = reinterpret_cast<volatile FixSlot *>(slots)[slot].n_seg;
+        m = -INFINITY;
+        L = 0.f;
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          c_reg[g] = -INFINITY;
+          A_reg[g] = W_reg[g] = M_reg[g] = 0.f;
+        }
+        for (int sg = 0; sg < n_seg; ++sg) {
+          const float *ps = part + ((static_cast<size_t>(slot) * max_seg + sg) * kFixChunk + warp) * kPart;
+          const float ms = __ldcg(ps), mn = fmaxf(m, ms);
+          const float al = exp2f(m - mn), as = exp2f(ms - mn), ls = __ldcg(ps + 1) * as;
+          L *= al;
+#pragma unroll
+          for (int g = 0; g < G; ++g) {
+            if (!((ent.mask[g] >> lane) & 1u)) continue;
+            const int j = lane + 32 * g;
+            A_reg[g] *= al;
+            W_reg[g] *= al;
+            M_reg[g] = fmaf(M_reg[g], al, __ldcg(ps + 2 + 3 * D + j) * as);
+            fold_tile(c_reg[g], A_reg[g], W_reg[g], L, __ldcg(ps + 2 + j), __ldcg(ps + 2 + D + j) * as,
+                      __ldcg(ps + 2 + 2 * D + j) * as, ls, b_reg[g], rb_reg[g]);
+          }
+          L += ls;
+          m = mn;
+        }
+      }
+    }
+    if (read_out && t >= 0) {
 #pragma unroll
       for (int g = 0; g < G; ++g) {
         if (!((ent.mask[g] >> lane) & 1u)) continue;
@@ -400,27 +571,28 @@ __global__ void __launch_bounds__(kFixThreads, D == 64 ? 4 : 3) fixup_kernel(con
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const ChanInfo *chan,
                          const float *shift, float *out, int H, int T, int d, int causal, const FixupEntry *entries,
                          const int *count, const int *rows, int *next_chunk, int *last_rows, const TcGate *gate,
-                         int num_sms, cudaStream_t stream, bool pdl) {
+                         int *fix_long, FixSlot *fix_slots, float *fix_part, int num_sms, cudaStream_t stream,
+                         bool pdl) {
   const TcGate g = gate ? *gate : TcGate{nullptr, nullptr, nullptr, nullptr, nullptr};
   const __nv_bfloat16 *qb = static_cast<const __nv_bfloat16 *>(q), *kb = static_cast<const __nv_bfloat16 *>(k),
                       *vb = static_cast<const __nv_bfloat16 *>(v);
   const int grid = num_sms * (d == 64 ? 4 : 3);
   if (d == 64) {
     const size_t smem = (kBlockK * (64 + 8) + kBlockK * (64 + 2) + 16 * (64 + 8)) * sizeof(__nv_bfloat16);
-    cudaError_t e = launch_kernel(fixup_kernel<64>, dim3(grid), dim3(kFixThreads), smem, stream, pdl, qb, kb, vb, beta,
-                                  chan, shift, out, H, T, causal, entries, count, rows, next_chunk, last_rows, g);
+    cudaError_t e = launch_kernel(fix_part ? fixup_kernel<64, true> : fixup_kernel<64, false>, dim3(grid),
+                                  dim3(kFixThreads), smem, stream, pdl, qb, kb, vb, beta, chan, shift, out, H, T,
+                                  causal, entries, count, rows, next_chunk, last_rows, g, fix_long, fix_slots, fix_part);
     if (e != cudaSuccess) return e;
   } else if (d == 128) {
     const size_t smem = (kBlockK * (128 + 8) + kBlockK * (128 + 2) + 16 * (128 + 8)) * sizeof(__nv_bfloat16);
-    cudaError_t e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    const auto kern = fix_part ? fixup_kernel<128, true> : fixup_kernel<128, false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     // three blocks per SM need the largest shared-memory carveout
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(fixup_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                               cudaSharedmemCarveoutMaxShared);
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
-    e = launch_kernel(fixup_kernel<128>, dim3(grid), dim3(kFixThreads), smem, stream, pdl, qb, kb, vb, beta, chan, shift,
-                      out, H, T, causal, entries, count, rows, next_chunk, last_rows, g);
+    e = launch_kernel(kern, dim3(grid), dim3(kFixThreads), smem, stream, pdl, qb, kb, vb, beta, chan, shift, out, H, T,
+                      causal, entries, count, rows, next_chunk, last_rows, g, fix_long, fix_slots, fix_part);
     if (e != cudaSuccess) return e;
   } else {
     return cudaErrorInvalidValue;

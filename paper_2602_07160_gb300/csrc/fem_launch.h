@@ -42,6 +42,9 @@ struct BankWorkspace {
   int *fixup_count;         // its length in slots, a multiple of 8 (zeroed before the pre-pass)
   int *fixup_rows;          // rows listed (zeroed before the pre-pass)
   int *fixup_next;          // the fix-up's next unclaimed chunk (zeroed before the pre-pass)
+  int *fix_long;            // chunks registered for splitting (zeroed before the pre-pass)
+  FixSlot *fix_slots;       // [kFixPoolSlots] (zeroed before the pre-pass)
+  float *fix_part;          // [kFixPoolSlots, fix_max_segs, kFixChunk, 2 + 4 d] partial states; null: no split
 };
 
 // Capacity of the fix-up list in entries: every row, plus the padding of each
@@ -109,7 +112,8 @@ constexpr int kMaxSeqLen = 8192 * kBlockK;
 cudaError_t launch_fixup(const void *q, const void *k, const void *v, const float *beta, const ChanInfo *chan,
                          const float *shift, float *out, int H, int T, int d, int causal, const FixupEntry *entries,
                          const int *count, const int *rows, int *next_chunk, int *last_rows, const TcGate *gate,
-                         int num_sms, cudaStream_t stream, bool pdl = false);
+                         int *fix_long, FixSlot *fix_slots, float *fix_part, int num_sms, cudaStream_t stream,
+                         bool pdl = false);
 
 
 // Decode read of one query per (b, h) against T cached keys: per-CTA key-chunk

@@ -93,6 +93,25 @@ def test_student_t_values_wide_beta(d):
     _assert_close(out, ref, what="student-t")
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_long_recomputations_over_key_tile_segments(d):
+    """T = 16384 has 128 key tiles, so fix-up chunks that recompute rows from the first key
+    tile over 16 or more tiles are split into segments of 8 tiles taken by different blocks
+    and merged by the last one (heavy-tailed values and beta up to 100 list such rows, at
+    every query tile).  Compared with the oracle: every row of the last two query tiles of
+    each head, where the segments are most, and rows drawn at random."""
+    B, H, T = 1, 2, 16384
+    q, k, v, beta = W.make_custom(B, H, T, d, beta_lo=1e-3, beta_hi=100.0, v_dist="student_t3",
+                                  const_channels=4, seed=21)
+    out, lse = _gpu_bf16(q, k, v, beta, True)
+    assert fem.last_fixup_rows() > 0
+    late = np.concatenate([np.arange(hh * T + T - 256, hh * T + T) for hh in range(B * H)])
+    rows = np.unique(np.concatenate([late, np.random.default_rng(5).choice(B * H * T, size=256, replace=False)]))
+    ref, ref_lse = oracle.fem_read_rows(q, k, v, beta, True, rows)
+    _assert_close(out.reshape(-1, d)[rows], ref, what="segments")
+    assert np.abs(lse.reshape(-1)[rows] - ref_lse).max() <= LSE_MAX
+
+
 def test_first_row_is_first_value_and_constant_channels():
     """P1 and P2 on the device: row 0 reads v_0; constant channels read the constant."""
     q, k, v, beta = W.make_custom(2, 2, 260, 128, beta_lo=1e-3, beta_hi=100.0, const_channels=4, seed=3)
