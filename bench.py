@@ -585,26 +585,29 @@ def run_fem(args):
                                "what": "fem_tdc_conv: h_t = exp(-s_t) h_(t-1) + u_t, segmented scan; algorithmic "
                                        "bytes s + u + h (fp32)"}
         del ts, tu, th
-        # gradients of the fp32 read (fem_bwd_f32) on B1 H4 T2048 d64 causal
-        qb, kb, vb, bb = (x.to(device) for x in W.make_custom(1, 4, 2048, 64, dtype="f32", seed=3))
-        ob, lb = fem.fem_fwd_f32(qb, kb, vb, bb, causal=True)
-        gb = torch.randn(qb.shape, device=device, generator=gen)
-        fem.fem_bwd_f32(qb, kb, vb, bb, ob, lb, gb, causal=True)
-        b0, b1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        b0.record(stream)
-        for _ in range(3):
-            fem.fem_bwd_f32(qb, kb, vb, bb, ob, lb, gb, causal=True, stream=stream)
-        b1.record(stream)
-        torch.cuda.synchronize(device)
-        fem.check_device_error(stream)
-        bwd_ms = b0.elapsed_time(b1) / 3
-        bwd_flops = 2.5 * 4.0 * 1 * 4 * 2048 * 2048 * 64 / 2  # flash-attention backward convention, causal
-        context["backward_f32"] = {"ms": bwd_ms, "tflops": bwd_flops / (bwd_ms * 1e-3) / 1e12,
-                                   "fp32_peak_tflops": fp32_peak,
-                                   "shape": {"B": 1, "H": 4, "T": 2048, "d": 64, "causal": True},
-                                   "what": "fem_bwd_f32: dq, dk, dv, dbeta of the fp32 read, two O(T^2 d) passes on "
-                                           "CUDA cores; FLOPs 2.5 x the forward's attention count"}
-        del qb, kb, vb, bb, ob, lb, gb
+        # gradients of the fp32 read (fem_bwd_f32), causal: a small shape and one head-batch of the
+        # headline shape (B1 H16 T8192 d128), where every SM holds enough rows
+        for key, (Bb, Hb, Tb, db, reps) in (("backward_f32", (1, 4, 2048, 64, 3)),
+                                            ("backward_f32_large", (1, 16, 8192, 128, 2))):
+            qb, kb, vb, bb = (x.to(device) for x in W.make_custom(Bb, Hb, Tb, db, dtype="f32", seed=3))
+            ob, lb = fem.fem_fwd_f32(qb, kb, vb, bb, causal=True)
+            gb = torch.randn(qb.shape, device=device, generator=gen)
+            fem.fem_bwd_f32(qb, kb, vb, bb, ob, lb, gb, causal=True)
+            b0, b1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            b0.record(stream)
+            for _ in range(reps):
+                fem.fem_bwd_f32(qb, kb, vb, bb, ob, lb, gb, causal=True, stream=stream)
+            b1.record(stream)
+            torch.cuda.synchronize(device)
+            fem.check_device_error(stream)
+            bwd_ms = b0.elapsed_time(b1) / reps
+            bwd_flops = 2.5 * 4.0 * Bb * Hb * Tb * Tb * db / 2  # flash-attention backward convention, causal
+            context[key] = {"ms": bwd_ms, "tflops": bwd_flops / (bwd_ms * 1e-3) / 1e12,
+                            "fp32_peak_tflops": fp32_peak,
+                            "shape": {"B": Bb, "H": Hb, "T": Tb, "d": db, "causal": True},
+                            "what": "fem_bwd_f32: dq, dk, dv, dbeta of the fp32 read, two O(T^2 d) passes on "
+                                    "CUDA cores; FLOPs 2.5 x the forward's attention count"}
+            del qb, kb, vb, bb, ob, lb, gb
 
     # ---- end to end through the host-buffer C ABI call
     e2e = None
