@@ -289,6 +289,32 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def time_graph(fn, iters):
+    """Mean ms per replay of a CUDA graph holding one fn(stream) call (the library's launches
+    captured as they are), replayed back to back: the call's device time without the host's
+    per-call overhead."""
+    import torch
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        fn(side)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn(torch.cuda.current_stream())
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(iters):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / iters
+
+
 def time_cuda(fn, stream, warmup, iters):
     """Mean ms per call of fn() over iters calls after warmup calls (CUDA events on stream)."""
     import torch
@@ -329,7 +355,11 @@ def workload_records(args, device, stream):
             def call():
                 fem.fem_fwd_f32(qd, kd, vd, bd, causal=w.causal, out=out, lse=lse, stream=stream)
             ms = time_cuda(call, stream, 5, 200)
+            gms = time_graph(lambda st: fem.fem_fwd_f32(qd, kd, vd, bd, causal=w.causal, out=out, lse=lse, stream=st),
+                             200)
             rec.update({"path": "fem_fwd_f32 (CUDA cores, fp32)", "ms": ms, "us": ms * 1e3,
+                        # the eager loop is bound by the Python call's overhead; a graph replay is not
+                        "graph_us": gms * 1e3,
                         "tflops": w.flops / (ms * 1e-3) / 1e12,
                         "roofline": {"bound": "latency", "note": "a few microseconds of launch and one "
                                      "dependent key loop per row; no throughput roofline applies"}})
@@ -343,6 +373,12 @@ def workload_records(args, device, stream):
             rec.update({"path": "fem_fwd (pre-pass, tcgen05 read, exact fix-up)", "ms": ms, "tflops": tf,
                         "fixup_rows": fem.last_fixup_rows(stream)})
             if name == "vit_s_full_prior":
+                # the whole call (counters, pre-pass, read, fix-up) captured once and replayed
+                ws = torch.empty(fem.workspace_bytes(w.B, w.H, w.T, w.d, w.causal), dtype=torch.uint8,
+                                 device=device)
+                rec["graph_ms"] = time_graph(
+                    lambda st: fem.fem_fwd_ws(qd, kd, vd, bd, ws, causal=w.causal, out=out, lse=lse, stream=st), iters)
+                del ws
                 gbs = io_bytes / (ms * 1e-3) / 1e9
                 rec["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
                                    "note": "algorithmic bytes Q, K, V in, out and lse out; tensor fraction "
