@@ -12,7 +12,12 @@
  *
  * beta_j = 0 is the continuous beta -> 0 limit, the prior mean
  * sum_i p_t(i) v_{i,j} (Prop. "app-baseline").  beta_j < 0 is outside the
- * method and a precondition violation (device memory is not inspected).
+ * method and a precondition violation: device memory is not inspected unless
+ * the environment variable FEM_DEBUG is set (to anything but "0") when the
+ * library first checks it.  Then every entry point that takes beta checks it
+ * first (one small kernel and a synchronisation of `stream`) and returns
+ * FEM_ERR_INVALID_ARG, with nothing of the computation enqueued, when an entry
+ * is negative, NaN or infinite.  Debug mode is not for stream capture.
  *
  * Conventions for every entry point:
  *  - Layout: q, k, v are [B, H, T, d] contiguous, d fastest; beta is [H, d]

@@ -11,6 +11,8 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdlib>
+#include <cstring>
 #include <mutex>
 #include <vector>
 
@@ -22,6 +24,7 @@ namespace {
 
 __device__ unsigned g_error_word;
 __device__ int g_last_fixup;
+__device__ unsigned g_beta_bad;  // FEM_DEBUG: set when a beta entry is negative, NaN or infinite
 
 constexpr int kMaxDevices = 64;
 
@@ -33,6 +36,7 @@ struct DeviceState {
   // stream-ordered workspaces come from this pool, which keeps freed memory for
   // the next call instead of returning it to the driver at every synchronisation
   cudaMemPool_t pool = nullptr;
+  unsigned *beta_bad = nullptr;
   // copy streams of fem_fwd_host, created on its first call
   cudaStream_t copy_in = nullptr, copy_out = nullptr;
 };
@@ -60,6 +64,7 @@ int device_state(DeviceState **out) {
     if (cudaGetSymbolAddress(reinterpret_cast<void **>(&s.last_fixup), g_last_fixup) != cudaSuccess)
       return FEM_ERR_CUDA;
     if (cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return FEM_ERR_CUDA;
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&s.beta_bad), g_beta_bad) != cudaSuccess) return FEM_ERR_CUDA;
     if (!g_encode) {
       cudaDriverEntryPointQueryResult q;
       void *fn = nullptr;
@@ -72,6 +77,49 @@ int device_state(DeviceState **out) {
     s.ready = true;
   }
   *out = &s;
+  return FEM_OK;
+}
+
+// FEM_DEBUG=1 (read once, at the first check): the entry points that take beta check it (beta >= 0
+// and finite) before they enqueue the computation, a synchronisation of the stream each.
+bool fem_debug() {
+  static const bool on = [] {
+    const char *e = std::getenv("FEM_DEBUG");
+    return e != nullptr && *e != 0 && std::strcmp(e, "0") != 0;
+  }();
+  return on;
+}
+
+__global__ void beta_check_kernel(const float *__restrict__ beta, int n, unsigned *bad) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+    const float b = beta[i];
+    if (!(b >= 0.f) || b == INFINITY) atomicOr(bad, 1u);
+  }
+}
+
+// FEM_OK unless FEM_DEBUG is on and beta [n] (device) holds a negative, NaN or infinite entry
+// (FEM_ERR_INVALID_ARG); a failing CUDA call gives FEM_ERR_CUDA.
+int debug_check_beta(const float *beta, long long n, DeviceState *ds, cudaStream_t s) {
+  if (!fem_debug()) return FEM_OK;
+  if (n <= 0 || n > (1ll << 30)) return FEM_ERR_INVALID_ARG;
+  unsigned bad = 0;
+  cudaError_t e = cudaMemsetAsync(ds->beta_bad, 0, sizeof(unsigned), s);
+  if (e == cudaSuccess) {
+    beta_check_kernel<<<static_cast<int>(std::min<long long>((n + 255) / 256, 1024)), 256, 0, s>>>(
+        beta, static_cast<int>(n), ds->beta_bad);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&bad, ds->beta_bad, sizeof(unsigned), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return FEM_ERR_CUDA;
+  return bad ? FEM_ERR_INVALID_ARG : FEM_OK;
+}
+
+// the same for beta in host memory
+int debug_check_beta_host(const float *beta, long long n) {
+  if (!fem_debug()) return FEM_OK;
+  for (long long i = 0; i < n; ++i)
+    if (!(beta[i] >= 0.f) || beta[i] == INFINITY) return FEM_ERR_INVALID_ARG;
   return FEM_OK;
 }
 
@@ -362,6 +410,8 @@ int fem_fwd_ws(const void *q, const void *k, const void *v, const float *beta, f
   if (workspace_bytes < w.total) return FEM_ERR_NO_MEMORY;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   return fwd_impl(q, k, v, beta, out, lse, B, H, T, d, causal, static_cast<uint8_t *>(workspace), nullptr, ds,
                   static_cast<cudaStream_t>(stream));
 }
@@ -373,6 +423,8 @@ int fem_fwd(const void *q, const void *k, const void *v, const float *beta, floa
   if ((rc = check_read_sizes(T, d)) != FEM_OK) return rc;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   const size_t bytes = fem_fwd_workspace_bytes(B, H, T, d, causal);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
@@ -392,6 +444,8 @@ int fem_fwd_gated(const void *q, const void *k, const void *v, const float *beta
   if ((rc = check_tc_sizes(T, d)) != FEM_OK) return rc;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta_max, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   // workspace: the beta_max read's, the mean's pre-pass (non-causal layout),
   // a zero beta [H, d], and mu_side [B, H, T, d] fp32 for the fix-up's entries
   // (the guard can list entries of either mask)
@@ -432,6 +486,8 @@ int fem_bwd_f32(const float *q, const float *k, const float *v, const float *bet
   if (d > 256) return FEM_ERR_UNSUPPORTED;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   return map_cuda(launch_bwd_f32(q, k, v, beta, out, lse, dout, dq, dk, dv, dbeta, B, H, T, d, causal,
                                  static_cast<cudaStream_t>(stream)));
 }
@@ -469,6 +525,8 @@ int fem_gla_fwd_tc(const float *qf, const float *kf, const float *v, const float
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   return map_cuda(launch_gla_tc(qf, kf, v, logdecay, beta, out, logz, B, H, T, ds->err,
                                 static_cast<cudaStream_t>(stream)));
 }
@@ -488,6 +546,8 @@ int fem_gla_fwd(const float *qf, const float *kf, const float *v, const float *l
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   const size_t bytes = gla_workspace_bytes(B * H, T, m, d, ds->num_sms, nullptr, nullptr);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
@@ -512,6 +572,8 @@ int fem_decode(const void *q, const void *k, const void *v, const float *beta, f
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   const int BH = B * H;
   const size_t bytes = decode_workspace_bytes(BH, T, d, ds->num_sms);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -536,6 +598,8 @@ int fem_fwd_f32(const float *q, const float *k, const float *v, const float *bet
   if (d > 256) return FEM_ERR_UNSUPPORTED;
   DeviceState *ds = nullptr;
   if ((rc = device_state(&ds)) != FEM_OK) return rc;
+  if ((rc = debug_check_beta(beta, static_cast<long long>(H) * d, ds, static_cast<cudaStream_t>(stream))) != FEM_OK)
+    return rc;
   return map_cuda(launch_f32(q, k, v, beta, out, lse, B, H, T, d, causal, static_cast<cudaStream_t>(stream)));
 }
 
@@ -544,6 +608,7 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
   if (!q || !k || !v || !beta || !out) return FEM_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || T <= 0 || d <= 0 || (causal != 0 && causal != 1)) return FEM_ERR_INVALID_ARG;
   if (check_read_sizes(T, d) != FEM_OK) return FEM_ERR_UNSUPPORTED;
+  if (debug_check_beta_host(beta, static_cast<long long>(H) * d) != FEM_OK) return FEM_ERR_INVALID_ARG;
   DeviceState *ds = nullptr;
   int rc = device_state(&ds);
   if (rc != FEM_OK) return rc;
