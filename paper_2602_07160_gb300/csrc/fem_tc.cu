@@ -56,6 +56,7 @@
 // next use always waits for the previous one.
 #include "fem_common.cuh"
 #include "fem_launch.h"
+#include "fem_order.h"
 
 namespace fem {
 
@@ -126,7 +127,6 @@ enum : int {
   kBarSide = 33      // + side slot (8): tile k's rescale factors and moved-channel mask are in shared memory
 };
 
-constexpr int kHeadGroup = 8;  // heads whose query tiles the launch order interleaves
 
 __device__ __forceinline__ int pad_chunk(int n) { return (n + kFixChunk - 1) / kFixChunk * kFixChunk; }
 
@@ -188,10 +188,9 @@ __global__ void __launch_bounds__(384, 1)
   // CTAs in flight share the K and E of at most two groups (64 MB at d = 128,
   // T = 8192) in L2: sixteen-head groups doubled that and raised the DRAM reads by 60 %
   const int rank = static_cast<int>(blockIdx.y * gridDim.x + blockIdx.x), BH = static_cast<int>(gridDim.y);
-  const int g0 = rank / (kHeadGroup * n_qt) * kHeadGroup, gsz = min(kHeadGroup, BH - g0);
-  const int idx = rank - g0 * n_qt;
-  const int bh = g0 + idx % gsz, h = bh % H;
-  const int qt = causal ? n_qt - 1 - idx / gsz : idx / gsz;
+  int bh, qt;
+  tc_tile_of_rank(rank, BH, n_qt, causal, bh, qt);
+  const int h = bh % H;
   const int nk = causal ? qt + 1 : n_kt_all;  // key tiles this query tile reads
   // causal with earlier key tiles: the diagonal tile's P E (of the beta bank)
   // goes to the score buffer no other tile uses from then on, so acc keeps
