@@ -112,6 +112,27 @@ def test_long_recomputations_over_key_tile_segments(d):
     assert np.abs(lse.reshape(-1)[rows] - ref_lse).max() <= LSE_MAX
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_maximum_sequence_length(d):
+    """T = 2^20, the longest sequence the tensor-core read takes (8192 key tiles; the fix-up
+    splits at 512 tiles per segment there).  Sampled rows against the oracle: the first rows,
+    rows around key-tile edges, the last rows and rows drawn at random."""
+    T = 1 << 20
+    q, k, v, beta = W.make_custom(1, 1, T, d, seed=31)
+    dev = torch.device("cuda", 0)
+    qd, kd, vd, bd = (x.to(dev) for x in (q, k, v, beta))
+    out, lse = fem.fem_fwd(qd, kd, vd, bd, causal=True)
+    fem.check_device_error()
+    rows = np.unique(np.concatenate([np.arange(8), [127, 128, 129, 65535, 65536, 524288],
+                                     np.arange(T - 8, T),
+                                     np.random.default_rng(7).choice(T, size=8, replace=False)]))
+    ref, ref_lse = oracle.fem_read_rows(q, k, v, beta, True, rows)
+    got = out.reshape(-1, d)[torch.from_numpy(rows).to(dev)].double().cpu().numpy()
+    _assert_close(got, ref, what="T = 2^20")
+    got_lse = lse.reshape(-1)[torch.from_numpy(rows).to(dev)].double().cpu().numpy()
+    assert np.abs(got_lse - ref_lse).max() <= LSE_MAX
+
+
 def test_first_row_is_first_value_and_constant_channels():
     """P1 and P2 on the device: row 0 reads v_0; constant channels read the constant."""
     q, k, v, beta = W.make_custom(2, 2, 260, 128, beta_lo=1e-3, beta_hi=100.0, const_channels=4, seed=3)
