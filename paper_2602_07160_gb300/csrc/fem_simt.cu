@@ -28,6 +28,9 @@ namespace fem {
 
 constexpr int kSimtMaxPerLane = 8;  // d <= 256
 
+// rows up to which a row gets a block of its own (its keys split over the warps)
+constexpr long long kSimtSplitRows = 2048;
+
 // keys per staged tile: K and V of a tile take 32 KB at most (8 KB at d = 16)
 inline __host__ __device__ int fem_simt_tile(int d) {
   const int kt = 4096 / d;
@@ -43,22 +46,26 @@ __device__ __forceinline__ float ld_in(const float *p) { return *p; }
 __device__ __forceinline__ float ld_in(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
 
 // PER: channel slots per lane, d <= 32 PER (the unrolled per-slot code costs
-// issue slots even where a slot is empty)
-template <typename In, int PER>
+// issue slots even where a slot is empty).  SPLIT (few rows): one row per
+// block, each warp folding a quarter of every staged tile's keys from an empty
+// state, the four states merged at the end (each scaled to the common row
+// maximum, each channel's moved to the larger shift as when a key raises it),
+// so that a row's dependent chain is a quarter as long.
+template <typename In, int PER, bool SPLIT>
 __global__ void __launch_bounds__(128) fem_simt_kernel(const In *__restrict__ q, const In *__restrict__ k,
                                                         const In *__restrict__ v, const float *__restrict__ beta,
                                                         float *__restrict__ out, float *__restrict__ lse, int H,
                                                         int T, int d, int causal) {
   extern __shared__ float simt_smem[];  // [tile][d] K, then [tile][d] V
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int bpr = (T + 3) / 4;  // blocks per (b, h)
+  const int bpr = SPLIT ? T : (T + 3) / 4;  // blocks per (b, h)
   const long long bh = blockIdx.x / bpr;
-  const int t0 = static_cast<int>(blockIdx.x % bpr) * 4, t = t0 + warp;
+  const int t0 = static_cast<int>(blockIdx.x % bpr) * (SPLIT ? 1 : 4), t = SPLIT ? t0 : t0 + warp;
   const bool valid = t < T;
   const long long row = bh * T + t;
   const int h = static_cast<int>(bh % H);
-  const int n = !valid ? 0 : (causal ? t + 1 : T);  // keys this row sees
-  const int n_blk = causal ? min(T, t0 + 4) : T;    // keys any row of the block sees
+  const int n = !valid ? 0 : (causal ? t + 1 : T);                // keys this row sees
+  const int n_blk = SPLIT ? n : (causal ? min(T, t0 + 4) : T);    // keys any row of the block sees
   const int per = (d + 31) / 32;  // <= PER
   const int tile = fem_simt_tile(d);
   const float inv_sqrt_d = rsqrtf(static_cast<float>(d));
@@ -88,7 +95,10 @@ __global__ void __launch_bounds__(128) fem_simt_kernel(const In *__restrict__ q,
     }
     __syncthreads();
     const int n_here = min(nt, n - i0);  // this row's keys in the tile
-    for (int ii = 0; ii < n_here; ++ii) {
+    // SPLIT: this warp's quarter of them
+    const int quarter = (n_here + 3) / 4;
+    const int ii0 = SPLIT ? min(n_here, warp * quarter) : 0, ii1 = SPLIT ? min(n_here, ii0 + quarter) : n_here;
+    for (int ii = ii0; ii < ii1; ++ii) {
       const float *kr = sk + ii * d;
       float part = 0.f;
 #pragma unroll
@@ -131,6 +141,69 @@ __global__ void __launch_bounds__(128) fem_simt_kernel(const In *__restrict__ q,
       L += p;
     }
   }
+  if (SPLIT) {
+    // warps 1..3 leave their states in shared memory (m, L, then c, A, W per channel); warp 0
+    // folds them into its own in key order
+    __syncthreads();  // the last tile is consumed
+    float *st = simt_smem + (warp - 1) * (2 + 3 * d);
+    if (warp > 0) {
+      if (lane == 0) {
+        st[0] = m;
+        st[1] = L;
+      }
+#pragma unroll
+      for (int u = 0; u < PER; ++u) {
+        const int j = lane + 32 * u;
+        if (!(u < per && j < d)) continue;
+        st[2 + j] = c[u];
+        st[2 + d + j] = A[u];
+        st[2 + 2 * d + j] = W[u];
+      }
+    }
+    __syncthreads();
+    if (warp > 0) return;
+    for (int w = 1; w < 4; ++w) {
+      const float *sw = simt_smem + (w - 1) * (2 + 3 * d);
+      const float m2 = sw[0], L2 = sw[1];
+      if (m2 == -INFINITY) continue;  // a warp that saw no key
+      if (m == -INFINITY) {           // this one saw none: take the other state
+        m = m2;
+        L = L2;
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+          const int j = lane + 32 * u;
+          if (!(u < per && j < d)) continue;
+          c[u] = sw[2 + j];
+          A[u] = sw[2 + d + j];
+          W[u] = sw[2 + 2 * d + j];
+        }
+        continue;
+      }
+      const float mn = fmaxf(m, m2), a1 = expf(m - mn), a2 = expf(m2 - mn);
+      const float L1 = L * a1, Ls = L2 * a2;
+#pragma unroll
+      for (int u = 0; u < PER; ++u) {
+        const int j = lane + 32 * u;
+        if (!(u < per && j < d)) continue;
+        const float b = bj[u], c2 = sw[2 + j];
+        float A1 = A[u] * a1, W1 = W[u] * a1, A2 = sw[2 + d + j] * a2, W2 = sw[2 + 2 * d + j] * a2;
+        if (c2 > c[u]) {
+          const float r = expf(b * (c[u] - c2));
+          W1 = r * W1 + expm1_over_beta(b, c[u] - c2) * L1;
+          A1 *= r;
+          c[u] = c2;
+        } else if (c2 < c[u]) {
+          const float r = expf(b * (c2 - c[u]));
+          W2 = r * W2 + expm1_over_beta(b, c2 - c[u]) * Ls;
+          A2 *= r;
+        }
+        A[u] = A1 + A2;
+        W[u] = W1 + W2;
+      }
+      L = L1 + Ls;
+      m = mn;
+    }
+  }
   if (!valid) return;
 
 #pragma unroll
@@ -154,17 +227,25 @@ template <typename In>
 static cudaError_t launch_simt(const In *q, const In *k, const In *v, const float *beta, float *out, float *lse, int B,
                                int H, int T, int d, int causal, cudaStream_t stream) {
   if (d > 32 * kSimtMaxPerLane) return cudaErrorInvalidValue;
-  const unsigned blocks = static_cast<unsigned>(static_cast<long long>(B) * H * ((T + 3) / 4));
+  // few rows: a block per row, its keys split over the four warps (the merge area of three
+  // states fits in the staging space: 3 (2 + 3 d) <= 2 tile d floats)
+  const long long rows = static_cast<long long>(B) * H * T;
+  const bool split = rows <= kSimtSplitRows;
+  const unsigned blocks = static_cast<unsigned>(split ? rows : static_cast<long long>(B) * H * ((T + 3) / 4));
   const size_t smem = 2 * static_cast<size_t>(fem_simt_tile(d)) * d * sizeof(float);
   const int per = (d + 31) / 32;
+#define FEM_SIMT_LAUNCH(P)                                                                                          \
+  (split ? fem_simt_kernel<In, P, true><<<blocks, 128, smem, stream>>>(q, k, v, beta, out, lse, H, T, d, causal)     \
+         : fem_simt_kernel<In, P, false><<<blocks, 128, smem, stream>>>(q, k, v, beta, out, lse, H, T, d, causal))
   if (per == 1)
-    fem_simt_kernel<In, 1><<<blocks, 128, smem, stream>>>(q, k, v, beta, out, lse, H, T, d, causal);
+    FEM_SIMT_LAUNCH(1);
   else if (per == 2)
-    fem_simt_kernel<In, 2><<<blocks, 128, smem, stream>>>(q, k, v, beta, out, lse, H, T, d, causal);
+    FEM_SIMT_LAUNCH(2);
   else if (per <= 4)
-    fem_simt_kernel<In, 4><<<blocks, 128, smem, stream>>>(q, k, v, beta, out, lse, H, T, d, causal);
+    FEM_SIMT_LAUNCH(4);
   else
-    fem_simt_kernel<In, 8><<<blocks, 128, smem, stream>>>(q, k, v, beta, out, lse, H, T, d, causal);
+    FEM_SIMT_LAUNCH(8);
+#undef FEM_SIMT_LAUNCH
   return cudaGetLastError();
 }
 
