@@ -447,16 +447,27 @@ __global__ void __launch_bounds__(256, 1)
           const float b = c_beta[j];
           const float *vcol = v + r0 * kVD + jo + j;
           float m = -INFINITY, acc = 0.f;
+          // 32 keys' values in flight at a time (the chunk's staged values already hold the next
+          // chunk's), then the walk over them
 #pragma unroll
-          for (int i = 0; i < kGC; ++i) {
-            if (i <= t) {
-              const float x = b * __ldg(vcol + static_cast<size_t>(i) * kVD);
-              const float a = __uint_as_float(sr[i >> 5][i & 31]) * expf(gt - gam[i]);
-              if (x > m) {
-                acc = fmaf(acc, expf(m - x), a);
-                m = x;
-              } else {
-                acc = fmaf(a, expf(x - m), acc);
+          for (int i0 = 0; i0 < kGC; i0 += 32) {
+            if (i0 > t) break;
+            float xv[32];
+#pragma unroll
+            for (int k2 = 0; k2 < 32; ++k2)
+              xv[k2] = i0 + k2 < rows ? __ldg(vcol + static_cast<size_t>(i0 + k2) * kVD) : 0.f;
+#pragma unroll
+            for (int k2 = 0; k2 < 32; ++k2) {
+              const int i = i0 + k2;
+              if (i <= t) {
+                const float x = b * xv[k2];
+                const float a = __uint_as_float(sr[i >> 5][i & 31]) * expf(gt - gam[i]);
+                if (x > m) {
+                  acc = fmaf(acc, expf(m - x), a);
+                  m = x;
+                } else {
+                  acc = fmaf(a, expf(x - m), acc);
+                }
               }
             }
           }
