@@ -59,6 +59,9 @@ SMALL = [
     (2, 2, 129, 64, False),
     (2, 3, 197, 64, False),
     (1, 2, 300, 128, False),
+    # the last length of the one-launch pre-pass (four key tiles) and the first of the three launches
+    (1, 2, 512, 64, True),
+    (1, 2, 513, 128, False),
 ]
 
 
