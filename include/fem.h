@@ -239,7 +239,9 @@ int fem_gla_fwd_tc(const float *qf, const float *kf, const float *v, const float
  *   s, u : device, float32 [B, T, Hc]; s >= 0 (the softplus rates)
  *   h    : device, float32 [B, T, Hc]
  * A segmented scan in fp32 (segment end states, a combine over segments, then
- * the outputs).  Allocates its workspace stream-ordered on `stream`.
+ * the outputs).  Up to T = 16384 one launch of 8-CTA clusters that combine
+ * through distributed shared memory and allocates nothing; beyond, three
+ * launches with a workspace allocated stream-ordered on `stream`.
  */
 int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc, void *stream);
 

@@ -503,7 +503,9 @@ int fem_tdc_conv(const float *s, const float *u, float *h, int B, int T, int Hc,
   if (rc != FEM_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   void *ws = nullptr;
-  cudaError_t e = ws_alloc(ds, &ws, tdc_workspace_bytes(B, T, Hc), st);
+  const size_t bytes = tdc_workspace_bytes(B, T, Hc);  // 0: the one-launch form, no workspace
+  if (bytes == 0) return map_cuda(launch_tdc(s, u, h, B, T, Hc, nullptr, st));
+  cudaError_t e = ws_alloc(ds, &ws, bytes, st);
   if (e != cudaSuccess) return map_cuda(e);
   rc = map_cuda(launch_tdc(s, u, h, B, T, Hc, ws, st));
   e = cudaFreeAsync(ws, st);

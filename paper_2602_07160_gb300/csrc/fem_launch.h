@@ -137,7 +137,8 @@ cudaError_t launch_gla_tc(const float *qf, const float *kf, const float *v, cons
                           float *out, float *logz, int B, int H, int T, unsigned *err, cudaStream_t stream);
 
 // Time-decay conditioner convolution h_t = exp(-s_t) h_{t-1} + u_t over [B, T, Hc]
-// (segmented scan); `ws` holds tdc_workspace_bytes() bytes.
+// (segmented scan: one launch of 8-CTA clusters up to T = 16384, no workspace, then
+// tdc_workspace_bytes() is 0; three launches beyond); `ws` holds tdc_workspace_bytes() bytes.
 size_t tdc_workspace_bytes(int B, int T, int Hc);
 cudaError_t launch_tdc(const float *s, const float *u, float *h, int B, int T, int Hc, void *ws, cudaStream_t stream);
 

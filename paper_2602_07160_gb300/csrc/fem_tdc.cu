@@ -18,10 +18,13 @@
 // lanes.  (A single pass with a decoupled look-back over segments measured
 // slower: 44 us against 27 us for the three kernels at B4 T8192 Hc64, its
 // look-back walking one dependent load at a time.)
+#include <cooperative_groups.h>
+
 #include "fem_common.cuh"
 #include "fem_launch.h"
 
 namespace fem {
+namespace cg = cooperative_groups;
 
 constexpr int kTdcSeg = 32;  // steps per segment
 
@@ -107,12 +110,114 @@ __global__ void tdc_combine_kernel(int B, int n_seg, int Hc, float *__restrict__
   }
 }
 
+// ---------------------------------------------------------------------------
+// One-launch form for T <= kTdcClusterMaxT: a cluster of n CTAs per (b, 32
+// channels), n = 1, 2, 4 or 8 so that a thread has about kTdcSubLen steps, CTA r
+// taking the r-th n-th of the time axis, warp w of a CTA the w-th of its 32
+// sub-segments, lane = channel (each warp load is one 128-byte step of 32
+// channels).  (1) every thread's sub-segment map x -> exp(-S) x + a from zero
+// (S its summed rate); (2) warp 0 composes the CTA's 32 maps in order (each
+// sub-segment's prefix kept in shared memory), the cluster barrier publishes
+// the CTA's total map, and warp 0 composes the totals of the CTAs before it,
+// read from their shared memory, into the CTA's start state; (3) every thread
+// runs its sub-segment again from its start state and writes h.  The second
+// read of s and u finds them in L2.  No workspace and one launch instead of
+// three; the maps compose exactly like the combine kernel's.
+// ---------------------------------------------------------------------------
+constexpr int kTdcCtas = 8;           // CTAs per cluster at most (portable cluster size)
+constexpr int kTdcSubs = 32;          // sub-segments (warps) per CTA
+constexpr int kTdcSubLen = 32;        // steps per sub-segment the cluster size aims at
+constexpr int kTdcClusterMaxT = 16384;
+
+__global__ void __launch_bounds__(32 * kTdcSubs, 1)
+    tdc_cluster_kernel(const float *__restrict__ s, const float *__restrict__ u, float *__restrict__ h, int T, int Hc,
+                       int len_sub) {
+  __shared__ float s_S[kTdcSubs][32], s_a[kTdcSubs][32];  // sub-segment maps, then their exclusive prefixes
+  __shared__ float s_tot[2][32];                           // the CTA's total map (S, a) per channel
+  __shared__ float s_start[32];                            // the state before the CTA's first step
+  cg::cluster_group cluster = cg::this_cluster();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int rank = static_cast<int>(cluster.block_rank());  // the block's part of the time axis
+  const int c = static_cast<int>(blockIdx.y) * 32 + lane, b = static_cast<int>(blockIdx.z);
+  const bool valid = c < Hc;
+  const int t0 = min(T, (rank * kTdcSubs + w) * len_sub), t1 = min(T, t0 + len_sub);
+  const size_t base = static_cast<size_t>(b) * T * Hc + c;
+
+  // (1) the sub-segment's map from a zero state; the loads do not depend on the recurrence
+  float acc = 0.f, S = 0.f;
+  if (valid) {
+#pragma unroll 16
+    for (int t = t0; t < t1; ++t) {
+      const size_t e = base + static_cast<size_t>(t) * Hc;
+      const float st = s[e];
+      acc = fmaf(ex2_approx(-st * kLog2e), acc, u[e]);
+      S += st;
+    }
+  }
+  s_S[w][lane] = S;
+  s_a[w][lane] = acc;
+  __syncthreads();
+  // (2) exclusive prefixes of the CTA's maps in order, and its total
+  if (w == 0) {
+    float PS = 0.f, Pa = 0.f;  // the map of sub-segments 0 .. i-1
+    for (int i = 0; i < kTdcSubs; ++i) {
+      const float Si = s_S[i][lane], ai = s_a[i][lane];
+      s_S[i][lane] = PS;
+      s_a[i][lane] = Pa;
+      Pa = fmaf(ex2_approx(-Si * kLog2e), Pa, ai);
+      PS += Si;
+    }
+    s_tot[0][lane] = PS;
+    s_tot[1][lane] = Pa;
+  }
+  cluster.sync();  // every CTA's total map is in its shared memory
+  if (w == 0) {
+    float x = 0.f;  // h before step 0 is zero
+    for (int q = 0; q < rank; ++q) {
+      const float *tot = cluster.map_shared_rank(&s_tot[0][0], q);
+      x = fmaf(ex2_approx(-tot[lane] * kLog2e), x, tot[32 + lane]);
+    }
+    s_start[lane] = x;
+  }
+  cluster.sync();  // the remote reads are done (no CTA leaves while another reads it); start states ready
+  // (3) the sub-segment again from its start state, writing h
+  acc = fmaf(ex2_approx(-s_S[w][lane] * kLog2e), s_start[lane], s_a[w][lane]);
+  if (valid) {
+#pragma unroll 16
+    for (int t = t0; t < t1; ++t) {
+      const size_t e = base + static_cast<size_t>(t) * Hc;
+      acc = fmaf(ex2_approx(-s[e] * kLog2e), acc, u[e]);
+      h[e] = acc;
+    }
+  }
+}
+
+bool tdc_one_launch(int B, int T, int Hc) { return T <= kTdcClusterMaxT && (Hc + 31) / 32 <= 65535 && B <= 65535; }
+
 size_t tdc_workspace_bytes(int B, int T, int Hc) {
+  if (tdc_one_launch(B, T, Hc)) return 0;
   const size_t n_seg = (static_cast<size_t>(T) + kTdcSeg - 1) / kTdcSeg;
   return 2 * static_cast<size_t>(B) * n_seg * Hc * sizeof(float);
 }
 
 cudaError_t launch_tdc(const float *s, const float *u, float *h, int B, int T, int Hc, void *ws, cudaStream_t stream) {
+  if (tdc_one_launch(B, T, Hc)) {
+    int n = 1;  // CTAs per cluster: the smallest power of two giving sub-segments of at most kTdcSubLen steps
+    while (n < kTdcCtas && n * kTdcSubs * kTdcSubLen < T) n *= 2;
+    const int len_sub = (T + n * kTdcSubs - 1) / (n * kTdcSubs);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(n, (Hc + 31) / 32, B);
+    cfg.blockDim = dim3(32 * kTdcSubs);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = n;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tdc_cluster_kernel, s, u, h, T, Hc, len_sub);
+  }
   const int n_seg = (T + kTdcSeg - 1) / kTdcSeg;
   float *state = static_cast<float *>(ws);
   float *rate = state + static_cast<size_t>(B) * n_seg * Hc;

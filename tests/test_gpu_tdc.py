@@ -23,7 +23,10 @@ def lib():
                                             (1, 1000, 48, 0.2), (4, 2000, 64, 0.01),
                                             # 157 segments (several per combine lane) and more
                                             # channels than a block's threads
-                                            (1, 5000, 40, 0.01), (1, 1200, 300, 0.05)])
+                                            (1, 5000, 40, 0.01), (1, 1200, 300, 0.05),
+                                            # the longest sequence of the one-launch form, and the
+                                            # first of the three launches
+                                            (1, 16384, 4, 0.01), (1, 16385, 4, 0.01)])
 def test_tdc_matches_oracle(B, T, Hc, s_scale):
     g = torch.Generator().manual_seed(T + Hc)
     s = s_scale * torch.nn.functional.softplus(torch.randn((B, T, Hc), generator=g))
