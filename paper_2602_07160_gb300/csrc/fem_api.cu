@@ -624,10 +624,30 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
   // Chunks of consecutive heads of one batch element (contiguous in every
   // [B, H, T, d] array): the copies in of chunk c+1, the read of chunk c and
   // the copies out of chunk c-1 overlap (two copy streams, the caller's stream
-  // computing).  About eight chunks in all.
+  // computing).  About eight chunks in all, the first and the last of them
+  // split into a quarter and the rest: only the first chunk's copies in run
+  // before any read and only the last chunk's read and copies out after the
+  // last copy in, so small end chunks shorten the pipeline's fill and drain.
   const int per_b = std::max(1, std::min(H, 8 / B));
-  const int hc = (H + per_b - 1) / per_b;  // heads per chunk
-  const int n_chunks = B * ((H + hc - 1) / hc);
+  const int hc = (H + per_b - 1) / per_b;  // heads per chunk (at most)
+  struct Chunk {
+    int b, h0, nh;
+  };
+  std::vector<Chunk> chunks;
+  for (int b = 0; b < B; ++b)
+    for (int h0 = 0; h0 < H; h0 += hc) chunks.push_back({b, h0, std::min(hc, H - h0)});
+  const int edge = std::max(1, hc / 4);
+  if (chunks.front().nh > edge) {
+    const Chunk f = chunks.front();
+    chunks.front() = {f.b, f.h0 + edge, f.nh - edge};
+    chunks.insert(chunks.begin(), Chunk{f.b, f.h0, edge});
+  }
+  if (chunks.back().nh > edge) {
+    const Chunk l = chunks.back();
+    chunks.back() = {l.b, l.h0, l.nh - edge};
+    chunks.push_back({l.b, l.h0 + l.nh - edge, edge});
+  }
+  const int n_chunks = static_cast<int>(chunks.size());
   const size_t n = static_cast<size_t>(B) * H * T * d;
   const size_t rows = static_cast<size_t>(B) * H * T;
   const size_t in_b = round256(n * 2), beta_b = round256(static_cast<size_t>(H) * d * 4), out_b = round256(n * 4),
@@ -649,35 +669,32 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(db, beta, static_cast<size_t>(H) * d * 4, cudaMemcpyHostToDevice, ds->copy_in);
   rc = map_cuda(e);
-  int c = 0;
-  for (int b = 0; b < B && rc == FEM_OK; ++b) {
-    for (int h0 = 0; h0 < H && rc == FEM_OK; h0 += hc, ++c) {
-      const int nh = std::min(hc, H - h0);
-      const size_t e0 = (static_cast<size_t>(b) * H + h0) * T * d, ne = static_cast<size_t>(nh) * T * d;
-      const size_t r0 = (static_cast<size_t>(b) * H + h0) * T, nr = static_cast<size_t>(nh) * T;
-      const uint8_t *hq = static_cast<const uint8_t *>(q), *hk = static_cast<const uint8_t *>(k),
-                    *hv = static_cast<const uint8_t *>(v);
-      e = cudaMemcpyAsync(dq + e0 * 2, hq + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
-      if (e == cudaSuccess) e = cudaMemcpyAsync(dk + e0 * 2, hk + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
-      if (e == cudaSuccess) e = cudaMemcpyAsync(dv + e0 * 2, hv + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
-      if (e == cudaSuccess) e = cudaEventRecord(ev[2 * c], ds->copy_in);
-      if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[2 * c], 0);
-      rc = map_cuda(e);
-      if (rc == FEM_OK)
-        rc = fem_fwd_ws(dq + e0 * 2, dk + e0 * 2, dv + e0 * 2, reinterpret_cast<const float *>(db) + h0 * d,
-                        reinterpret_cast<float *>(dout) + e0, lse ? reinterpret_cast<float *>(dlse) + r0 : nullptr, 1,
-                        nh, T, d, causal, dws, ws_b, stream);
-      if (rc != FEM_OK) break;
-      e = cudaEventRecord(ev[2 * c + 1], s);
-      if (e == cudaSuccess) e = cudaStreamWaitEvent(ds->copy_out, ev[2 * c + 1], 0);
-      if (e == cudaSuccess)
-        e = cudaMemcpyAsync(out + e0, reinterpret_cast<float *>(dout) + e0, ne * 4, cudaMemcpyDeviceToHost,
-                            ds->copy_out);
-      if (e == cudaSuccess && lse)
-        e = cudaMemcpyAsync(lse + r0, reinterpret_cast<float *>(dlse) + r0, nr * 4, cudaMemcpyDeviceToHost,
-                            ds->copy_out);
-      rc = map_cuda(e);
-    }
+  for (int c = 0; c < n_chunks && rc == FEM_OK; ++c) {
+    const int b = chunks[c].b, h0 = chunks[c].h0, nh = chunks[c].nh;
+    const size_t e0 = (static_cast<size_t>(b) * H + h0) * T * d, ne = static_cast<size_t>(nh) * T * d;
+    const size_t r0 = (static_cast<size_t>(b) * H + h0) * T, nr = static_cast<size_t>(nh) * T;
+    const uint8_t *hq = static_cast<const uint8_t *>(q), *hk = static_cast<const uint8_t *>(k),
+                  *hv = static_cast<const uint8_t *>(v);
+    e = cudaMemcpyAsync(dq + e0 * 2, hq + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dk + e0 * 2, hk + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dv + e0 * 2, hv + e0 * 2, ne * 2, cudaMemcpyHostToDevice, ds->copy_in);
+    if (e == cudaSuccess) e = cudaEventRecord(ev[2 * c], ds->copy_in);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev[2 * c], 0);
+    rc = map_cuda(e);
+    if (rc == FEM_OK)
+      rc = fem_fwd_ws(dq + e0 * 2, dk + e0 * 2, dv + e0 * 2, reinterpret_cast<const float *>(db) + h0 * d,
+                      reinterpret_cast<float *>(dout) + e0, lse ? reinterpret_cast<float *>(dlse) + r0 : nullptr, 1,
+                      nh, T, d, causal, dws, ws_b, stream);
+    if (rc != FEM_OK) break;
+    e = cudaEventRecord(ev[2 * c + 1], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(ds->copy_out, ev[2 * c + 1], 0);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(out + e0, reinterpret_cast<float *>(dout) + e0, ne * 4, cudaMemcpyDeviceToHost,
+                          ds->copy_out);
+    if (e == cudaSuccess && lse)
+      e = cudaMemcpyAsync(lse + r0, reinterpret_cast<float *>(dlse) + r0, nr * 4, cudaMemcpyDeviceToHost,
+                          ds->copy_out);
+    rc = map_cuda(e);
   }
   // the caller's stream frees the buffers once every copy out has landed
   cudaError_t ej = cudaEventRecord(ev[2 * n_chunks + 1], ds->copy_out);
