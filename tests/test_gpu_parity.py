@@ -205,7 +205,8 @@ def test_host_entry_point_matches():
 @pytest.mark.parametrize("causal", [True, False])
 def test_host_entry_point_chunks(causal):
     """B = 3, H = 5: the host entry point copies and reads chunks of three and two heads per
-    batch element, overlapped; every chunk matches the device entry point."""
+    batch element (the very first and last chunks split into one head and the rest),
+    overlapped; every chunk matches the device entry point."""
     q, k, v, beta = W.make_custom(3, 5, 200, 64, seed=9)
     dev = torch.device("cuda", 0)
     o1, l1 = fem.fem_fwd(*(x.to(dev) for x in (q, k, v, beta)), causal=causal)
