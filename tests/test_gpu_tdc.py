@@ -31,7 +31,8 @@ def test_tdc_matches_oracle(B, T, Hc, s_scale):
     g = torch.Generator().manual_seed(T + Hc)
     s = s_scale * torch.nn.functional.softplus(torch.randn((B, T, Hc), generator=g))
     u = torch.randn((B, T, Hc), generator=g)
-    h = fem.fem_tdc_conv(s.cuda(), u.cuda())
+    h = torch.full((B, T, Hc), float("nan"), device="cuda")  # poisoned: every element must be written
+    fem.fem_tdc_conv(s.cuda(), u.cuda(), out=h)
     fem.check_device_error()
     ref = oracle.tdc_conv(s, u)
     err = np.abs(h.cpu().double().numpy() - ref)
