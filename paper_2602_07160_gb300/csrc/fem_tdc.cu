@@ -116,13 +116,14 @@ __global__ void tdc_combine_kernel(int B, int n_seg, int Hc, float *__restrict__
 // taking the r-th n-th of the time axis, warp w of a CTA the w-th of its 32
 // sub-segments, lane = channel (each warp load is one 128-byte step of 32
 // channels).  (1) every thread's sub-segment map x -> exp(-S) x + a from zero
-// (S its summed rate); (2) warp 0 composes the CTA's 32 maps in order (each
-// sub-segment's prefix kept in shared memory), the cluster barrier publishes
-// the CTA's total map, and warp 0 composes the totals of the CTAs before it,
-// read from their shared memory, into the CTA's start state; (3) every thread
-// runs its sub-segment again from its start state and writes h.  The second
-// read of s and u finds them in L2.  No workspace and one launch instead of
-// three; the maps compose exactly like the combine kernel's.
+// (S its summed rate); (2) warp c scans channel c's 32 maps in order, lane =
+// sub-segment, with shuffles (the exclusive prefixes back in shared memory),
+// the cluster barrier publishes the CTA's total maps, and warp 0 loads the
+// totals of the CTAs before it from their shared memory and composes them into
+// the CTA's start state; (3) every thread runs its sub-segment again from its
+// start state and writes h.  The second read of s and u finds them in L2.  No
+// workspace and one launch instead of three; the maps compose like the combine
+// kernel's.
 // ---------------------------------------------------------------------------
 constexpr int kTdcCtas = 8;           // CTAs per cluster at most (portable cluster size)
 constexpr int kTdcSubs = 32;          // sub-segments (warps) per CTA
@@ -132,7 +133,7 @@ constexpr int kTdcClusterMaxT = 16384;
 __global__ void __launch_bounds__(32 * kTdcSubs, 1)
     tdc_cluster_kernel(const float *__restrict__ s, const float *__restrict__ u, float *__restrict__ h, int T, int Hc,
                        int len_sub) {
-  __shared__ float s_S[kTdcSubs][32], s_a[kTdcSubs][32];  // sub-segment maps, then their exclusive prefixes
+  __shared__ float s_S[kTdcSubs][33], s_a[kTdcSubs][33];  // [sub-segment][channel]: maps, then their exclusive prefixes
   __shared__ float s_tot[2][32];                           // the CTA's total map (S, a) per channel
   __shared__ float s_start[32];                            // the state before the CTA's first step
   cg::cluster_group cluster = cg::this_cluster();
@@ -157,26 +158,42 @@ __global__ void __launch_bounds__(32 * kTdcSubs, 1)
   s_S[w][lane] = S;
   s_a[w][lane] = acc;
   __syncthreads();
-  // (2) exclusive prefixes of the CTA's maps in order, and its total
-  if (w == 0) {
-    float PS = 0.f, Pa = 0.f;  // the map of sub-segments 0 .. i-1
-    for (int i = 0; i < kTdcSubs; ++i) {
-      const float Si = s_S[i][lane], ai = s_a[i][lane];
-      s_S[i][lane] = PS;
-      s_a[i][lane] = Pa;
-      Pa = fmaf(ex2_approx(-Si * kLog2e), Pa, ai);
-      PS += Si;
+  // (2) warp w scans channel w's maps over the sub-segments (lane = sub-segment): an
+  // earlier map (Sp, ap) followed by a later one (S, a) is (Sp + S, exp(-S) ap + a)
+  {
+    float SS = s_S[lane][w], A = s_a[lane][w];
+#pragma unroll
+    for (int off = 1; off < kTdcSubs; off <<= 1) {
+      const float Sp = __shfl_up_sync(0xffffffffu, SS, off), ap = __shfl_up_sync(0xffffffffu, A, off);
+      if (lane >= off) {
+        A = fmaf(ex2_approx(-SS * kLog2e), ap, A);
+        SS += Sp;
+      }
     }
-    s_tot[0][lane] = PS;
-    s_tot[1][lane] = Pa;
+    float exS = __shfl_up_sync(0xffffffffu, SS, 1), exA = __shfl_up_sync(0xffffffffu, A, 1);
+    if (lane == 0) exS = exA = 0.f;
+    s_S[lane][w] = exS;
+    s_a[lane][w] = exA;
+    if (lane == kTdcSubs - 1) {
+      s_tot[0][w] = SS;
+      s_tot[1][w] = A;
+    }
   }
-  cluster.sync();  // every CTA's total map is in its shared memory
+  cluster.sync();  // every CTA's total maps are in its shared memory
   if (w == 0) {
-    float x = 0.f;  // h before step 0 is zero
-    for (int q = 0; q < rank; ++q) {
-      const float *tot = cluster.map_shared_rank(&s_tot[0][0], q);
-      x = fmaf(ex2_approx(-tot[lane] * kLog2e), x, tot[32 + lane]);
+    float tS[kTdcCtas], tA[kTdcCtas];  // the totals of the CTAs before this one, loaded together
+#pragma unroll
+    for (int q = 0; q < kTdcCtas; ++q) {
+      if (q < rank) {
+        const float *tot = cluster.map_shared_rank(&s_tot[0][0], q);
+        tS[q] = tot[lane];
+        tA[q] = tot[32 + lane];
+      }
     }
+    float x = 0.f;  // h before step 0 is zero
+#pragma unroll
+    for (int q = 0; q < kTdcCtas; ++q)
+      if (q < rank) x = fmaf(ex2_approx(-tS[q] * kLog2e), x, tA[q]);
     s_start[lane] = x;
   }
   cluster.sync();  // the remote reads are done (no CTA leaves while another reads it); start states ready
