@@ -17,6 +17,7 @@
 #include <vector>
 
 #include "fem.h"
+#include "fem_chunks.h"
 #include "fem_launch.h"
 
 namespace fem {
@@ -621,32 +622,9 @@ int fem_fwd_host(const void *q, const void *k, const void *v, const float *beta,
     if (!ds->copy_out && cudaStreamCreateWithFlags(&ds->copy_out, cudaStreamNonBlocking) != cudaSuccess)
       return FEM_ERR_CUDA;
   }
-  // Chunks of consecutive heads of one batch element (contiguous in every
-  // [B, H, T, d] array): the copies in of chunk c+1, the read of chunk c and
-  // the copies out of chunk c-1 overlap (two copy streams, the caller's stream
-  // computing).  About eight chunks in all, the first and the last of them
-  // split into a quarter and the rest: only the first chunk's copies in run
-  // before any read and only the last chunk's read and copies out after the
-  // last copy in, so small end chunks shorten the pipeline's fill and drain.
-  const int per_b = std::max(1, std::min(H, 8 / B));
-  const int hc = (H + per_b - 1) / per_b;  // heads per chunk (at most)
-  struct Chunk {
-    int b, h0, nh;
-  };
-  std::vector<Chunk> chunks;
-  for (int b = 0; b < B; ++b)
-    for (int h0 = 0; h0 < H; h0 += hc) chunks.push_back({b, h0, std::min(hc, H - h0)});
-  const int edge = std::max(1, hc / 4);
-  if (chunks.front().nh > edge) {
-    const Chunk f = chunks.front();
-    chunks.front() = {f.b, f.h0 + edge, f.nh - edge};
-    chunks.insert(chunks.begin(), Chunk{f.b, f.h0, edge});
-  }
-  if (chunks.back().nh > edge) {
-    const Chunk l = chunks.back();
-    chunks.back() = {l.b, l.h0, l.nh - edge};
-    chunks.push_back({l.b, l.h0 + l.nh - edge, edge});
-  }
+  // chunks of heads whose copies in, reads and copies out overlap (fem_chunks.h)
+  const int hc = host_chunk_heads(B, H);  // heads per chunk, at most
+  const std::vector<HostChunk> chunks = host_chunks(B, H);
   const int n_chunks = static_cast<int>(chunks.size());
   const size_t n = static_cast<size_t>(B) * H * T * d;
   const size_t rows = static_cast<size_t>(B) * H * T;
